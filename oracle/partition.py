@@ -1,0 +1,118 @@
+"""Chunk-boundary oracle for Latency-Balanced Chunk Partitioning (TEST INFRASTRUCTURE).
+
+Test infrastructure only (see ``oracle/__init__.py``); the product path never
+imports this module.
+
+What the paper fixes
+--------------------
+Sec. 3.2, Eq. 1: the attention cost of chunk ``i`` with length ``c_i`` and
+prefix ``p_i = c_1 + ... + c_{i-1}`` grows with ``c_i`` times the number of keys
+it sees, while the GEMM part grows with ``c_i`` alone.  Sec. 3.2 (Insight) and
+Sec. 4.2: later chunks are made shorter so that chunk costs are balanced;
+stage 1 of Algorithm 1 builds a compute-balanced split.
+
+Readings taken here (the paper gives no closed rule):
+
+* cost_i = c_i * (p_i + c_i / 2), the number of (query, key) pairs of a causal
+  chunk up to the O(c_i) diagonal term.  Then
+  ``2 * cost_i = b_{i+1}^2 - b_i^2`` with ``b_i = p_i`` the chunk start, so the
+  total cost telescopes to ``S^2 / 2`` for ANY split and equal costs give the
+  closed form ``b_i = S * sqrt(i / M)``.
+* Boundaries are multiples of the granularity ``g``: with ``U = S // g``,
+  ``n_i = round_half_up(U * sqrt(i / M))`` (computed exactly in integers as the
+  largest ``n >= 0`` with ``n == 0`` or ``M * (2n - 1)^2 <= 4 * i * U^2``),
+  ``b_i = g * n_i``.
+* Clamp in one forward pass so every chunk has at least ``g`` tokens:
+  ``b_i = min(max(b_i, b_{i-1} + g), g * (U - (M - i)))``; ``b_0 = 0``,
+  ``b_M = S`` (the last chunk absorbs ``S % g``).
+* Uniform mode (used for the two small configurations): ``n_i =
+  round_half_up(i * U / M)`` with the same clamps.
+
+Everything is exact Python integer arithmetic (``math.isqrt``), so the result
+is bit-exact by construction.
+"""
+
+from __future__ import annotations
+
+import math
+from typing import List
+
+UNIFORM = 0
+LBCP = 1
+
+
+def _check(seq_len: int, num_chunks: int, granularity: int) -> int:
+    if seq_len <= 0 or num_chunks < 1 or granularity < 1:
+        raise ValueError("seq_len > 0, num_chunks >= 1, granularity >= 1 required")
+    if num_chunks * granularity > seq_len:
+        raise ValueError("num_chunks * granularity must not exceed seq_len")
+    return seq_len // granularity
+
+
+def _round_half_up_sqrt(i: int, num_chunks: int, units: int) -> int:
+    """round_half_up(units * sqrt(i / num_chunks)) exactly.
+
+    round_half_up(x) = n  <=>  n - 1/2 <= x < n + 1/2.  For n >= 1 the left
+    side is (2n - 1)^2 <= 4 x^2 = 4 i U^2 / M; the largest odd q = 2n - 1 with
+    q^2 <= 4 i U^2 / M is isqrt(floor(4 i U^2 / M)).
+    """
+    q = math.isqrt((4 * i * units * units) // num_chunks)
+    return (q + 1) // 2
+
+
+def _round_half_up_ratio(i: int, num_chunks: int, units: int) -> int:
+    """round_half_up(i * units / num_chunks) exactly."""
+    return (2 * i * units + num_chunks) // (2 * num_chunks)
+
+
+def boundaries(seq_len: int, num_chunks: int, granularity: int = 128,
+               mode: int = LBCP) -> List[int]:
+    """Chunk boundaries ``[b_0 = 0, b_1, ..., b_M = seq_len]``.
+
+    ``mode`` is ``LBCP`` (equal cost_i, Sec. 3.2 / Sec. 4.2) or ``UNIFORM``.
+    """
+    units = _check(seq_len, num_chunks, granularity)
+    if mode == LBCP:
+        raw = [_round_half_up_sqrt(i, num_chunks, units) for i in range(num_chunks)]
+    elif mode == UNIFORM:
+        raw = [_round_half_up_ratio(i, num_chunks, units) for i in range(num_chunks)]
+    else:
+        raise ValueError("unknown partition mode")
+    out = [0]
+    for i in range(1, num_chunks):
+        b = granularity * raw[i]
+        b = max(b, out[-1] + granularity)
+        b = min(b, granularity * (units - (num_chunks - i)))
+        out.append(b)
+    out.append(seq_len)
+    return out
+
+
+def chunk_cost_x2(bounds: List[int]) -> List[int]:
+    """Twice the per-chunk attention cost, ``2 * c_i * (p_i + c_i / 2)``.
+
+    Written with the chunk length and prefix of Eq. 1 (not with the
+    telescoped squares) so that the telescoping identity can be tested.
+    """
+    costs = []
+    for i in range(len(bounds) - 1):
+        p = bounds[i]
+        c = bounds[i + 1] - bounds[i]
+        costs.append(c * (2 * p + c))
+    return costs
+
+
+def eq1_cost(bounds: List[int]) -> List[int]:
+    """Eq. 1 as printed, ``c_i * (p_i + c_i)`` (used only for comparison)."""
+    return [(bounds[i + 1] - bounds[i]) * (bounds[i + 1]) for i in range(len(bounds) - 1)]
+
+
+def causal_pairs(bounds: List[int]) -> List[int]:
+    """Exact number of causal (query, key) pairs per chunk,
+    ``c_i * p_i + c_i * (c_i + 1) / 2`` (the attention FLOP count / (4 H d))."""
+    out = []
+    for i in range(len(bounds) - 1):
+        p = bounds[i]
+        c = bounds[i + 1] - bounds[i]
+        out.append(c * p + c * (c + 1) // 2)
+    return out
