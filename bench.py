@@ -1,0 +1,479 @@
+#!/usr/bin/env python3
+"""Benchmark: chunked causal prefill attention (MOCAP's hot path) on GB300.
+
+One step = one pass of the whole hot path over one prompt: LBCP boundaries
+(host), then for every chunk the KV append and the chunk attention.  The
+default workload is the 131072-token Llama-3-70B attention shape (64 q-heads,
+8 kv-heads, d=128) in 32 LBCP chunks.  Inputs are larger than L2 (Q 2 GiB,
+K/V 256 MiB each), so no flush is needed between steps.
+
+Prints ONE JSON line (rank 0).  ``--impl reference`` times the float64 CPU
+oracle instead, on a bounded row sample of the same workload.
+
+Under torchrun each rank runs an independent replica on its own GPU (the
+path has no exchange step); value = all ranks' work / the slowest rank.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "chunk-attn TFLOP/s & % GB300 BF16 tensor peak; prefill tokens/s"
+FALLBACK_PEAK_TFLOPS = 1700.0  # sustained bf16, used only without MEASURED_PEAKS.json
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", type=int, default=4)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-rows-per-chunk", type=int, default=2)
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------ helpers --
+def attn_flops(bounds_list, n_q_heads, head_dim):
+    """Algorithmic FLOP: 4 * Hq * d per causal (query, key) pair; pairs per
+    chunk c_i * p_i + c_i (c_i + 1) / 2 (exact, no masked-tile waste)."""
+    per_chunk = []
+    for bounds in bounds_list:
+        per_chunk.append([4 * n_q_heads * head_dim *
+                          ((b1 - b0) * b0 + (b1 - b0) * (b1 - b0 + 1) // 2)
+                          for b0, b1 in zip(bounds[:-1], bounds[1:])])
+    return per_chunk
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    except Exception:
+        return {"bf16_tflops_sustained": FALLBACK_PEAK_TFLOPS, "hbm_gbs": FALLBACK_HBM_GBS}, \
+            "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in ("chunk_attn.cu", "sm103_ptx.cuh"):
+        with open(os.path.join(ROOT, "paper_2606_22968_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(workload_name):
+    """DRAM bytes per launch of the attention kernel from the committed ncu
+    summary, if it was taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "chunk_attn_dram_traffic.txt")
+    try:
+        vals = {}
+        with open(path) as f:
+            for line in f:
+                if ":" in line and not line.startswith("#"):
+                    k, v = line.split(":", 1)
+                    vals[k.strip()] = v.strip()
+        if vals.get("kernel_source_sha256_16") != kernel_source_hash():
+            return None
+        if vals.get("workload") != workload_name:
+            return None
+        return float(vals["dram_bytes_per_launch_full_workload"])
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            import tempfile
+            fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.out, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.out.close()
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax = float(parts[2])
+                except ValueError:
+                    continue
+                for name, val in zip(names, parts[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------- CPU oracle --
+def oracle_sample_plan(bounds, rows_per_chunk, step_index):
+    """(chunk, rows) items the oracle evaluates in one sampled step: for every
+    chunk, the last row plus evenly spread rows shifted by the step index;
+    chunks are visited last-first, then first, then alternating inwards so a
+    time-bounded prefix of the plan still spans short and long prefixes."""
+    n_chunks = len(bounds) - 1
+    order, lo, hi = [], 0, n_chunks - 1
+    while lo <= hi:
+        order.append(hi)
+        if lo != hi:
+            order.append(lo)
+        lo, hi = lo + 1, hi - 1
+    plan = []
+    for i in order:
+        n = bounds[i + 1] - bounds[i]
+        rows = {n - 1}
+        for r in range(1, rows_per_chunk):
+            rows.add((r * n // rows_per_chunk + 37 * step_index) % n)
+        plan.append((i, sorted(rows)))
+    return plan
+
+
+def _oracle_worker(args):
+    """Runs in a spawned process: times the oracle over sampled rows, each
+    step stopping after `budget_s` seconds (at least one item)."""
+    (q_items, k_bits, v_bits, bounds, plans, scale, budget_s, threads) = args
+    import numpy as np
+    from oracle import attention as A
+    k = A.bf16_bits_to_f64(k_bits)
+    v = A.bf16_bits_to_f64(v_bits)
+    times, flops, done = [], [], []
+    for plan, qs in zip(plans, q_items):
+        t0 = time.perf_counter()
+        fl, n_done = 0, 0
+        for (i, rows), q_bits in zip(plan, qs):
+            b0, b1 = bounds[i], bounds[i + 1]
+            r = np.array(rows)
+            q_rows = A.bf16_bits_to_f64(q_bits)
+            q_full = np.zeros((int(r.max()) + 1,) + q_rows.shape[1:])
+            q_full[r] = q_rows
+            A.chunk_attention(q_full, k[:b1], v[:b1], b0, scale, rows=r)
+            fl += sum(4 * q_rows.shape[1] * q_rows.shape[2] * (b0 + x + 1) for x in rows)
+            n_done += 1
+            if time.perf_counter() - t0 > budget_s:
+                break
+        times.append(time.perf_counter() - t0)
+        flops.append(fl)
+        done.append(n_done)
+    return times, flops, done
+
+
+def run_oracle_sample(q, k, v, bounds, scale, n_steps, rows_per_chunk, budget_s):
+    """Time the oracle on sampled rows (q/k/v: torch tensors on any device)."""
+    import multiprocessing as mp
+    import torch
+    threads = os.cpu_count() or 1
+    plans = [oracle_sample_plan(bounds, rows_per_chunk, s) for s in range(n_steps)]
+    q_items = []
+    for plan in plans:
+        items = []
+        for i, rows in plan:
+            idx = torch.as_tensor([bounds[i] + x for x in rows], device=q.device)
+            items.append(q[idx].cpu().view(torch.int16).numpy())
+        q_items.append(items)
+    k_bits = k.cpu().view(torch.int16).numpy()
+    v_bits = v.cpu().view(torch.int16).numpy()
+    env_keys = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS")
+    saved = {x: os.environ.get(x) for x in env_keys}
+    for x in env_keys:
+        os.environ[x] = str(threads)  # inherited by the spawned worker
+    try:
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(1) as pool:
+            times, flops, done = pool.apply(
+                _oracle_worker, ((q_items, k_bits, v_bits, bounds, plans, scale, budget_s,
+                                  threads),))
+    finally:
+        for x, val in saved.items():
+            if val is None:
+                os.environ.pop(x, None)
+            else:
+                os.environ[x] = val
+    return times, flops, done, threads
+
+
+# --------------------------------------------------------------- main arms --
+def init_dist(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world, device):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def reference_arm(args, rank, world):
+    """The float64 oracle, timed on the host cores on a bounded sample."""
+    import torch
+    from paper_2606_22968_gb300 import workloads
+    from oracle import partition as P
+    if rank != 0:
+        return 0
+    w = workloads.get(args.workload)
+    bounds = P.boundaries(w.seq_lens[0], w.num_chunks[0], 128, w.mode)
+    q, k, v = workloads.make_qkv(w, "cpu")
+    n = args.steps + args.warmup
+    budget = max(2.0, min(15.0, 150.0 / n))
+    times, flops, done, threads = run_oracle_sample(q, k, v, bounds, w.scale, n,
+                                                    args.cpu_rows_per_chunk, budget)
+    t = sum(times[args.warmup:])
+    fl = sum(flops[args.warmup:])
+    value = fl / t / 1e12
+    sample = (f"per step: up to {args.cpu_rows_per_chunk} rows x all {w.n_q_heads} heads of "
+              f"each chunk, chunks visited last/first alternately until ~{budget:.0f} s "
+              f"(chunks done per step: {done}); float64 oracle")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000 * t / max(1, args.steps), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {**w.describe(), "workload": w.name},
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def ours_arm(args, rank, world, local):
+    import torch
+    import paper_2606_22968_gb300 as m
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+
+    m._lib.load()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = workloads.get(args.workload)
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev)
+    steps_plan = pf.steps()
+    n_chunks = len(steps_plan)
+    stream = torch.cuda.current_stream(dev)
+
+    flops_chunks = attn_flops(pf.bounds, w.n_q_heads, w.head_dim)
+    # per step (chunk index k): attention FLOP of every (request, k)
+    step_flops = [sum(flops_chunks[r][c] for r, c in st) for st in steps_plan]
+    total_flops = sum(step_flops)
+    append_bytes = 2 * 2 * w.total_tokens * w.n_kv_heads * w.head_dim * 2  # K,V x (rd+wr)
+
+    def one_step(ev=None):
+        pf.partition()
+        pf.run(q, k, v, stream, ev)
+
+    for _ in range(args.warmup):
+        one_step()
+    torch.cuda.synchronize(dev)
+    if m.mocap_last_device_status() != m.MOCAP_OK:
+        raise RuntimeError("device wait expired during warm-up")
+
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n_chunks)]
+           for _ in range(args.steps)]
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    time.sleep(0.3)  # let the sampler start before load
+    start.record(stream)
+    for s in range(args.steps):
+        one_step(evs[s])
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop()
+    status = m.mocap_last_device_status()
+    if status != m.MOCAP_OK:
+        raise RuntimeError(f"device status {m.mocap_status_string(status)}")
+
+    ms_total = start.elapsed_time(end)
+    ms_total = max_over_ranks(ms_total, world, dev)
+    ms_step = ms_total / args.steps
+    attn_ms = [[evs[s][c][1].elapsed_time(evs[s][c][2]) for c in range(n_chunks)]
+               for s in range(args.steps)]
+    app_ms = [[evs[s][c][0].elapsed_time(evs[s][c][1]) for c in range(n_chunks)]
+              for s in range(args.steps)]
+    attn_step_ms = [sum(x) for x in attn_ms]
+    app_step_ms = [sum(x) for x in app_ms]
+    per_chunk = [statistics.median(attn_ms[s][c] for s in range(args.steps))
+                 for c in range(n_chunks)]
+    cv = statistics.pstdev(per_chunk) / statistics.mean(per_chunk) if n_chunks > 1 else 0.0
+
+    value = world * total_flops / (ms_step * 1e-3) / 1e12
+    tokens_per_s = world * w.total_tokens / (ms_step * 1e-3)
+    peaks, peak_src = load_peaks()
+    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAK_TFLOPS))
+    attn_avg_ms = statistics.mean(attn_step_ms)
+    achieved = total_flops / (attn_avg_ms * 1e-3) / 1e12
+    launches_per_step = n_chunks  # attention launches
+    traffic_full = ncu_traffic(w.name)
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    app_gbs = append_bytes / (statistics.mean(app_step_ms) * 1e-3) / 1e9
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {**w.describe(), "workload": w.name,
+                   "l2": "inputs larger than L2 (no flush): Q %.1f GiB, K+V %.2f GiB" % (
+                       q.numel() * 2 / 2**30, 2 * k.numel() * 2 / 2**30),
+                   "parallelism": "replicas" if world > 1 else "single-gpu"},
+        "prefill_tokens_per_s": tokens_per_s,
+        "attn_tflops_kernel_only": achieved,
+        "attn_frac_of_peak": achieved / peak,
+        "per_chunk_attn_ms": {"min": min(per_chunk), "max": max(per_chunk),
+                              "max_over_min": max(per_chunk) / min(per_chunk), "cv": cv},
+        "append": {"gb_per_s": app_gbs, "frac_of_hbm": app_gbs / hbm,
+                   "ms_per_step": statistics.mean(app_step_ms)},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak,
+                     "peak_source": f"bf16_tflops_sustained ({peak_src})",
+                     "kernel": "chunk_attn_kernel",
+                     "traffic": None if traffic_full is None else traffic_full / launches_per_step,
+                     "traffic_unit": "bytes per launch (avg over the step's launches)"},
+        "clocks": clk,
+        # our kernels per timed region: one append per (request, chunk) and
+        # one attention launch per step
+        "gpu_launches": args.steps * sum(1 + len(st) for st in steps_plan),
+    }
+
+    if not args.no_e2e:
+        line["e2e"] = measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        times, flops, done, threads = run_oracle_sample(
+            q, k, v, pf.bounds[0], w.scale, 1, args.cpu_rows_per_chunk, 20.0)
+        line["cpu_baseline"] = {
+            "value": flops[0] / times[0] / 1e12, "unit": "TFLOP/s", "cores": threads,
+            "kind": "oracle",
+            "sample": f"up to {args.cpu_rows_per_chunk} rows x all {w.n_q_heads} heads of "
+                      f"{done[0]} of {len(pf.bounds[0]) - 1} chunks (last/first alternately, "
+                      f"~20 s budget): {flops[0]:.3e} FLOP in {times[0]:.1f} s, float64 oracle"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
+    """The same metric through the public API with host buffers: each step
+    copies Q/K/V from pinned host memory, runs the hot path and copies O and
+    LSE back."""
+    import torch
+    hq, hk, hv = (t.cpu().pin_memory() for t in (q, k, v))
+    ho = torch.empty(pf.out.shape, dtype=pf.out.dtype).pin_memory()
+    hl = torch.empty(pf.lse.shape, dtype=pf.lse.dtype).pin_memory()
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv))
+    d2h = ho.numel() * ho.element_size() + hl.numel() * hl.element_size()
+
+    def step():
+        dq.copy_(hq, non_blocking=True)
+        dk.copy_(hk, non_blocking=True)
+        dv.copy_(hv, non_blocking=True)
+        pf.partition()
+        pf.run(dq, dk, dv, stream)
+        ho.copy_(pf.out, non_blocking=True)
+        hl.copy_(pf.lse, non_blocking=True)
+
+    step()
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.e2e_steps):
+        step()
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    ms = max_over_ranks(t0.elapsed_time(t1) / args.e2e_steps, world, dev)
+    if not torch.equal(ho.to(dev), pf.out):
+        raise RuntimeError("e2e: host copy of O differs")
+    return {"value": world * total_flops / (ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+
+def main():
+    args = parse_args()
+    rank, world, local = init_dist(args)
+    try:
+        if args.impl == "reference":
+            return reference_arm(args, rank, world)
+        return ours_arm(args, rank, world, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,198 @@
+/*
+ * mocap.h -- C ABI of the GB300 (sm_103a) chunked causal prefill attention
+ * library: the data-parallel hot path of MOCAP's prefill-only method
+ * (arXiv 2606.22968).
+ *
+ * The method (Sec. 2.2, Sec. 3.2 / Eq. 1, Sec. 4.2): a long prompt of S
+ * tokens is split into M chunks with boundaries 0 = b_0 < b_1 < ... < b_M = S.
+ * Chunk i (rows [b_i, b_{i+1})) attends to the keys/values of all earlier
+ * chunks plus a causal block over itself, so its attention cost grows with
+ * its prefix; Latency-Balanced Chunk Partitioning picks boundaries that
+ * balance that cost.  The library exposes:
+ *
+ *   mocap_lbcp_partition      chunk boundaries (host, exact integers)
+ *   mocap_kv_append           chunk K/V -> contiguous bf16 KV cache (device)
+ *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
+ *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
+ *   mocap_last_device_status  bounded-wait timeouts reported by the kernels
+ *   mocap_status_string       text for a status code
+ *
+ * Conventions for every entry point:
+ *   - Tensor pointers are DEVICE pointers owned by the caller.  The library
+ *     never allocates, frees or retains caller memory.
+ *   - Layouts are dense row-major with no padding:
+ *       Q, O      bf16 [rows, n_q_heads, head_dim]
+ *       K, V      bf16 [rows, n_kv_heads, head_dim]   (chunk input or cache)
+ *       LSE       fp32 [n_q_heads, rows]
+ *     Device pointers must be 16-byte aligned.
+ *   - Work is enqueued on `stream` (NULL = legacy default stream) and the
+ *     call returns without synchronising.  No hidden host<->device traffic.
+ *   - Arguments are validated before any launch; on MOCAP_EINVAL or
+ *     MOCAP_EUNSUPPORTED nothing was enqueued.  MOCAP_ECUDA reports a failed
+ *     launch (the CUDA error is left for cudaGetLastError()).
+ */
+#ifndef MOCAP_H_
+#define MOCAP_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *mocap_stream_t; /* same object as cudaStream_t */
+
+typedef enum {
+  MOCAP_OK = 0,
+  MOCAP_EINVAL = 1,        /* bad argument (null, range, alignment, shape)   */
+  MOCAP_ECUDA = 2,         /* a CUDA runtime/driver call failed              */
+  MOCAP_EUNSUPPORTED = 3,  /* valid request this build does not implement    */
+  MOCAP_ETIMEOUT = 4       /* a device-side bounded wait expired             */
+} mocap_status;
+
+typedef enum {
+  MOCAP_PART_UNIFORM = 0,  /* n_i = round_half_up(i * U / M)                 */
+  MOCAP_PART_LBCP = 1      /* n_i = round_half_up(U * sqrt(i / M))           */
+} mocap_part_mode;
+
+/*
+ * mocap_lbcp_partition -- chunk boundaries with equal attention cost.
+ *
+ * Sec. 3.2, Eq. 1: chunk i of length c_i with prefix p_i costs attention work
+ * that grows with c_i * (keys seen).  We balance cost_i = c_i * (p_i + c_i/2),
+ * the causal pair count up to its O(c_i) term; since 2 * cost_i =
+ * b_{i+1}^2 - b_i^2 the equal-cost split is b_i = S * sqrt(i / M) (the
+ * compute-balanced initialisation of Sec. 4.2 / Algorithm 1 stage 1, for the
+ * attention term).  Boundaries are snapped to multiples of `granularity` g:
+ * with U = seq_len / g (floor), n_i = round_half_up(U * sqrt(i / M)) computed
+ * exactly in integers, b_i = g * n_i, then in one forward pass
+ * b_i = min(max(b_i, b_{i-1} + g), g * (U - (M - i))), b_0 = 0, b_M = seq_len.
+ * MOCAP_PART_UNIFORM uses n_i = round_half_up(i * U / M) with the same clamps.
+ * Every chunk has at least g tokens; the last absorbs seq_len % g.
+ *
+ *   seq_len      S, tokens, 1 <= S
+ *   num_chunks   M >= 1, with M * granularity <= S and S / g < 2^31
+ *   granularity  g >= 1 (128 matches the attention kernel's row tile)
+ *   boundaries   HOST array of num_chunks + 1 int64, written on success
+ *
+ * Pure host integer code: deterministic and bit-exact, no CUDA calls.
+ * Returns MOCAP_EINVAL for a null pointer or out-of-range argument.
+ */
+mocap_status mocap_lbcp_partition(int64_t seq_len, int32_t num_chunks,
+                                  int32_t granularity, mocap_part_mode mode,
+                                  int64_t *boundaries);
+
+/*
+ * mocap_kv_append -- write a chunk's K and V into the KV cache.
+ *
+ * Sec. 2.2 / Sec. 3.1: the KV of every earlier chunk stays live for later
+ * chunks.  Copies rows [0, len) of k_chunk/v_chunk (bf16 [len, n_kv_heads,
+ * head_dim]) to rows [offset, offset + len) of k_cache/v_cache (bf16
+ * [cache_capacity, n_kv_heads, head_dim]), bit-exact; no other cache byte is
+ * touched.  Source and destination must not overlap.
+ *
+ * MOCAP_EINVAL: null pointer, misaligned pointer, offset < 0, len < 0,
+ * offset + len > cache_capacity, n_kv_heads < 1, head_dim < 1 or
+ * n_kv_heads * head_dim not a multiple of 8.  len == 0 is a no-op.
+ */
+mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk,
+                             void *k_cache, void *v_cache,
+                             int64_t cache_capacity, int64_t offset, int64_t len,
+                             int32_t n_kv_heads, int32_t head_dim,
+                             mocap_stream_t stream);
+
+/*
+ * mocap_chunk_attn -- attention of one chunk against its KV prefix.
+ *
+ * Sec. 2.2 / Eq. 1: the chunk's queries (global rows prefix .. prefix+len-1)
+ * attend to cache rows 0 .. prefix+len-1 with a causal mask: query row t sees
+ * key rows j <= t.  For query head h the KV head is h / (n_q_heads /
+ * n_kv_heads) (contiguous GQA groups).  With s_j = scale * q_t . k_j:
+ *   out[i, h, :] = sum_j softmax(s)_j * v[j, kv(h), :]       (bf16, RNE)
+ *   lse[h, i]    = ln sum_j exp(s_j)                          (fp32)
+ * Softmax statistics and accumulation are fp32; the probabilities are
+ * rounded to bf16 for the P.V product.
+ *
+ *   q         bf16 [len, n_q_heads, head_dim]
+ *   k_cache   bf16 [>= prefix+len, n_kv_heads, head_dim]; rows >= prefix+len
+ *   v_cache   are never read (their contents may be anything, NaN included)
+ *   out       bf16 [len, n_q_heads, head_dim]
+ *   lse       fp32 [n_q_heads, len]
+ *   workspace, workspace_bytes: caller-owned device scratch of at least
+ *             mocap_chunk_attn_workspace_size(...) bytes (may be NULL when
+ *             that size is 0).
+ *
+ * Requirements: head_dim in {64, 128} (else MOCAP_EUNSUPPORTED); n_q_heads a
+ * multiple of n_kv_heads; scale > 0 and finite; prefix >= 0; len >= 0
+ * (0 = no-op); prefix + len < 2^31; 16-byte aligned pointers.
+ * Device-side bounded waits that expire are reported by
+ * mocap_last_device_status(); the kernel never traps.
+ */
+mocap_status mocap_chunk_attn(const void *q, const void *k_cache, const void *v_cache,
+                              int64_t prefix, int64_t len,
+                              int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
+                              float scale, void *out, float *lse,
+                              void *workspace, size_t workspace_bytes,
+                              mocap_stream_t stream);
+
+/* Bytes of device scratch mocap_chunk_attn needs for this shape (0 today:
+ * the single-pass kernel keeps all intermediates on chip). */
+size_t mocap_chunk_attn_workspace_size(int64_t prefix, int64_t len,
+                                       int32_t n_q_heads, int32_t head_dim);
+
+/*
+ * One (request, chunk) item of a varlen launch.  All offsets are in rows.
+ *   q_row     first row of this chunk's queries in the packed q / out buffers
+ *   kv_row    first cache row of the item's request (its key 0)
+ *   prefix    keys of earlier chunks of the request (cache rows kv_row ..
+ *             kv_row + prefix - 1)
+ *   len       the chunk's length; its own keys are cache rows
+ *             kv_row + prefix .. kv_row + prefix + len - 1
+ */
+typedef struct {
+  int64_t q_row;
+  int64_t kv_row;
+  int64_t prefix;
+  int64_t len;
+} mocap_varlen_item;
+
+#define MOCAP_VARLEN_MAX_ITEMS 64
+
+/*
+ * mocap_chunk_attn_varlen -- mocap_chunk_attn over up to
+ * MOCAP_VARLEN_MAX_ITEMS independent items in a single launch (e.g. chunk k
+ * of every request of a prefill batch).  Semantics per item are exactly
+ * mocap_chunk_attn with q = q + q_row rows, k/v_cache = cache + kv_row rows,
+ * out = out + q_row rows, and lse row block [h, q_row .. q_row+len) of the
+ * packed fp32 [n_q_heads, q_rows_total] array.
+ *
+ *   items        HOST array of n_items descriptors (read during the call only)
+ *   q_rows_total rows of the packed q / out buffers and row stride of lse
+ *   kv_rows_total rows of the packed caches (bounds check only)
+ * Items must not write overlapping output rows.  Same requirements and
+ * errors as mocap_chunk_attn; n_items == 0 is a no-op.
+ */
+mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const void *v_cache,
+                                     const mocap_varlen_item *items, int32_t n_items,
+                                     int64_t q_rows_total, int64_t kv_rows_total,
+                                     int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
+                                     float scale, void *out, float *lse,
+                                     mocap_stream_t stream);
+
+/*
+ * mocap_last_device_status -- synchronises `stream`, then reads and clears
+ * the device status word that the kernels set when a bounded wait expires
+ * (MOCAP_ETIMEOUT) instead of hanging.  MOCAP_OK when nothing was recorded;
+ * MOCAP_ECUDA if the synchronisation itself failed.
+ */
+mocap_status mocap_last_device_status(mocap_stream_t stream);
+
+/* Static, NUL-terminated name of a status code. */
+const char *mocap_status_string(mocap_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOCAP_H_ */

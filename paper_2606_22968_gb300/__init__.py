@@ -1,0 +1,110 @@
+"""GB300-native (sm_103a) chunked causal prefill attention -- the hot path of
+MOCAP's prefill-only method (arXiv 2606.22968), behind a C ABI.
+
+The functions below carry the C entry points' names and only marshal
+arguments (torch tensors -> device pointers, streams -> handles); all work
+runs in ``libmocap.so``.  There is no CPU fallback: a missing or unbuildable
+library raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+from typing import List, Sequence
+
+from . import _lib
+from ._lib import VarlenItem
+
+MOCAP_OK, MOCAP_EINVAL, MOCAP_ECUDA, MOCAP_EUNSUPPORTED, MOCAP_ETIMEOUT = 0, 1, 2, 3, 4
+MOCAP_PART_UNIFORM, MOCAP_PART_LBCP = 0, 1
+MOCAP_VARLEN_MAX_ITEMS = 64
+
+
+class MocapError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        msg = _lib.load().mocap_status_string(status)
+        super().__init__(f"{where}: {msg.decode() if msg else status}")
+
+
+def _check(status: int, where: str):
+    if status != MOCAP_OK:
+        raise MocapError(status, where)
+
+
+def _ptr(t) -> int:
+    if t is None:
+        return 0
+    if isinstance(t, int):
+        return t
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def mocap_lbcp_partition(seq_len: int, num_chunks: int, granularity: int = 128,
+                         mode: int = MOCAP_PART_LBCP) -> List[int]:
+    out = (ctypes.c_int64 * (num_chunks + 1))()
+    _check(_lib.load().mocap_lbcp_partition(seq_len, num_chunks, granularity, mode, out),
+           "mocap_lbcp_partition")
+    return list(out)
+
+
+def mocap_kv_append(k_chunk, v_chunk, k_cache, v_cache, offset: int, stream=None):
+    """Copy chunk K/V ([len, Hkv, d] bf16) into cache rows [offset, offset+len)."""
+    length, n_kv, d = k_chunk.shape
+    _check(_lib.load().mocap_kv_append(_ptr(k_chunk), _ptr(v_chunk), _ptr(k_cache), _ptr(v_cache),
+                                       k_cache.shape[0], offset, length, n_kv, d,
+                                       _stream(stream)), "mocap_kv_append")
+
+
+def mocap_chunk_attn_workspace_size(prefix: int, length: int, n_q_heads: int, head_dim: int) -> int:
+    return int(_lib.load().mocap_chunk_attn_workspace_size(prefix, length, n_q_heads, head_dim))
+
+
+def mocap_chunk_attn(q, k_cache, v_cache, prefix: int, out, lse, scale: float,
+                     workspace=None, stream=None):
+    """One chunk's causal GQA attention over cache rows [0, prefix+len).
+
+    q/out [len, Hq, d] bf16, caches [>= prefix+len, Hkv, d] bf16, lse [Hq, len] fp32.
+    """
+    length, n_q, d = q.shape
+    n_kv = k_cache.shape[1]
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(_lib.load().mocap_chunk_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), prefix, length,
+                                        n_q, n_kv, d, scale, _ptr(out), _ptr(lse),
+                                        _ptr(workspace), ws_bytes, _stream(stream)),
+           "mocap_chunk_attn")
+
+
+def mocap_chunk_attn_varlen(q, k_cache, v_cache, items: Sequence[tuple], out, lse, scale: float,
+                            stream=None):
+    """Many (q_row, kv_row, prefix, len) items in one launch; lse is [Hq, q_rows_total]."""
+    q_rows, n_q, d = q.shape
+    n_kv = k_cache.shape[1]
+    arr = (VarlenItem * max(1, len(items)))()
+    for i, (q_row, kv_row, prefix, length) in enumerate(items):
+        arr[i] = VarlenItem(q_row, kv_row, prefix, length)
+    _check(_lib.load().mocap_chunk_attn_varlen(_ptr(q), _ptr(k_cache), _ptr(v_cache), arr,
+                                               len(items), q_rows, k_cache.shape[0], n_q, n_kv,
+                                               d, scale, _ptr(out), _ptr(lse), _stream(stream)),
+           "mocap_chunk_attn_varlen")
+
+
+def mocap_last_device_status(stream=None) -> int:
+    return int(_lib.load().mocap_last_device_status(_stream(stream)))
+
+
+def mocap_status_string(status: int) -> str:
+    return _lib.load().mocap_status_string(status).decode()

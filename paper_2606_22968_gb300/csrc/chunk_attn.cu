@@ -1,0 +1,593 @@
+// chunk_attn.cu -- chunked causal GQA prefill attention on sm_103a.
+//
+// Sec. 2.2 / Eq. 1: chunk i's queries (global rows prefix .. prefix+len-1)
+// attend to the KV of every earlier chunk plus a causal block over their own
+// chunk; the attention work grows with the prefix, which is what LBCP
+// balances.  The kernel computes, for query head h (KV head h / group) and
+// global row t, O_t = softmax_{j<=t}(scale q_t.k_j) V and LSE_t = ln sum exp.
+//
+// Design (one CTA = 128 query rows x up to two query heads of one KV group):
+//   warp 0        TMA producer: Q tiles once, then K_j, V_j tiles (128 keys)
+//                 through a 4-deep ring of 128-byte-swizzled smem stages.
+//   warp 1        MMA issuer (one thread): S_s = Q_s K_j^T into TMEM, then
+//                 O_s += P_s V_j with P_s read from TMEM; tcgen05.commit
+//                 signals S ready / stage free / O final.
+//   warps 2-5     softmax for head slot 0, warps 6-9 for slot 1: a warp may
+//                 touch only TMEM lanes 32*(warp%4) .. +31, and any 4
+//                 consecutive warps cover all 128.  Thread r
+//                 owns TMEM lane r = query row r, so row max / row sum are
+//                 thread-local (no shuffles).  Online softmax in fp32, log2
+//                 domain; O is rescaled in TMEM only when the running max grows
+//                 by more than 2^8 (exact: the final 1/l uses the same max).
+//                 P is written back to TMEM as packed bf16 (aliasing S).
+//   TMEM (512 columns): S0 [0,128) S1 [128,256) O0 [256,256+D) O1 [256+D, ..).
+// The two slots share every K/V tile (two heads of one GQA group), so the
+// tensor core alternates between them while the other slot's softmax runs.
+// Key tiles entirely below the chunk's diagonal are unmasked; only the last
+// one or two tiles apply the causal mask.  Rows and keys past the chunk end
+// are zero-filled by TMA (the tensor maps end at prefix+len), so cache rows
+// beyond the prefix are never read.
+#include <cmath>
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "internal.h"
+#include "sm103_ptx.cuh"
+
+namespace mocap {
+namespace {
+
+constexpr int kBlockM = 128;   // query rows per tile = TMEM lanes
+constexpr int kBlockN = 128;   // keys per K/V tile
+constexpr int kStages = 4;     // ring stages, each holds one K or one V tile
+constexpr int kThreads = 320;  // 10 warps: producer, MMA, 2 x 4 softmax
+constexpr int kBoxCols = 64;   // bf16 per 128-byte swizzled row
+constexpr int kBoxBytes = kBlockM * kBoxCols * 2;  // 16 KB: one TMA box
+constexpr uint32_t kTmemCols = 512;
+constexpr float kMaxGrowthLog2 = 8.0f;  // rescale O only past a 2^8 max increase
+constexpr uint64_t kDrainLimitNs = 20000000ull;  // 20 ms for in-flight copies
+
+struct ItemDesc {
+  int64_t q_row;      // first packed Q/O row of the item
+  int32_t prefix;     // keys before the chunk
+  int32_t len;        // chunk rows
+  int32_t q_blocks;   // ceil(len / 128)
+  int32_t cta_begin;  // first CTA index of the item
+};
+
+template <int MAXI>
+struct AttnParams {
+  CUtensorMap tq[MAXI];  // Q  [len, Hq, D]           box {64, 1, 128}
+  CUtensorMap tk[MAXI];  // K  [prefix+len, Hkv, D]   box {64, 1, 128}
+  CUtensorMap tv[MAXI];  // V  [prefix+len, Hkv, D]   box {64, 1, 128}
+  ItemDesc items[MAXI];
+  __nv_bfloat16 *out;
+  float *lse;
+  uint32_t *status;
+  int64_t lse_stride;
+  int32_t n_items;
+  int32_t n_q_heads;
+  int32_t n_kv_heads;
+  int32_t heads_per_group;
+  int32_t pairs_per_group;
+  float scale_log2;  // scale * log2(e)
+};
+
+template <int D>
+struct Layout {
+  static constexpr int kTileBytes = kBlockM * D * 2;  // one Q, K or V tile
+  static constexpr int kQ = 0;                         // 2 Q tiles
+  static constexpr int kRing = 2 * kTileBytes;
+  static constexpr int kBars = kRing + kStages * kTileBytes;
+  // barrier slots (8 bytes each)
+  static constexpr int kBarQ = 0;
+  static constexpr int kBarFull = 1;               // kStages
+  static constexpr int kBarEmpty = 1 + kStages;    // kStages
+  static constexpr int kBarS = 1 + 2 * kStages;    // 2
+  static constexpr int kBarP = 3 + 2 * kStages;    // 2
+  static constexpr int kBarO = 5 + 2 * kStages;    // 2
+  static constexpr int kBarDrain = 7 + 2 * kStages;
+  static constexpr int kNumBars = 8 + 2 * kStages;
+  static constexpr int kTmemSlot = kBars + 8 * kNumBars;
+  static constexpr int kFlag = kTmemSlot + 4;
+  static constexpr int kBytes = kFlag + 4 + 1024;  // + slack for 1024-byte alignment
+};
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// S = Q K^T for one head slot: M=128, N=128, K=D; both operands K-major.
+template <int D>
+__device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint32_t q_smem, uint32_t k_smem) {
+  constexpr uint32_t idesc = idesc_bf16_f32(kBlockM, kBlockN, false, false);
+#pragma unroll
+  for (int kk = 0; kk < D / 16; ++kk) {
+    const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;  // 16 bf16 = 32 bytes
+    mma_ss(s_tmem, sdesc_sw128(q_smem + off, 16, 1024), sdesc_sw128(k_smem + off, 16, 1024),
+           idesc, kk > 0 ? 1u : 0u);
+  }
+}
+
+// O += P V for one head slot: M=128, N=D, K=128 keys.  P (A operand) lives in
+// TMEM, 2 bf16 per column; V (B operand) is MN-major: d is contiguous, two
+// 64-wide d halves 16 KB apart (LBO), 8-key groups 1024 bytes apart (SBO).
+template <int D>
+__device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint32_t v_smem,
+                                         bool accumulate) {
+  constexpr uint32_t idesc = idesc_bf16_f32(kBlockM, D, false, true);
+#pragma unroll
+  for (int kk = 0; kk < kBlockN / 16; ++kk) {
+    mma_ts(o_tmem, p_tmem + kk * 8, sdesc_sw128(v_smem + kk * 16 * 128, kBoxBytes, 1024), idesc,
+           (accumulate || kk > 0) ? 1u : 0u);
+  }
+}
+
+template <int D>
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, float (&x)[128]) {
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    uint32_t r[32];
+    tmem_ld32(taddr + c * 32, r);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) x[c * 32 + e] = __uint_as_float(r[e]);
+  }
+}
+
+template <int D, int MAXI>
+__global__ void __launch_bounds__(kThreads, 1)
+    chunk_attn_kernel(const __grid_constant__ AttnParams<MAXI> p) {
+  using L = Layout<D>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t *gbase = smem_raw + (base - raw);
+  const uint32_t bars = base + L::kBars;
+  auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
+  volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(gbase + L::kTmemSlot);
+  volatile uint32_t *flag = reinterpret_cast<volatile uint32_t *>(gbase + L::kFlag);
+
+  const uint32_t warp = threadIdx.x >> 5;
+  const uint32_t lane = threadIdx.x & 31u;
+
+  // A launch after an expired wait does nothing (CTA-uniform decision).
+  if (threadIdx.x == 0) *flag = *reinterpret_cast<volatile uint32_t *>(p.status);
+  __syncthreads();
+  if (*flag != 0u) return;
+
+  // ---- work item --------------------------------------------------------
+  int item = 0;
+  const int cta = static_cast<int>(blockIdx.x);
+  while (item + 1 < p.n_items && cta >= p.items[item + 1].cta_begin) ++item;
+  const ItemDesc it = p.items[item];
+  int w = cta - it.cta_begin;
+  const int pair = w % p.pairs_per_group;
+  w /= p.pairs_per_group;
+  const int g = w % p.n_kv_heads;
+  w /= p.n_kv_heads;
+  const int qblock = it.q_blocks - 1 - w;  // heaviest (latest) row blocks first
+  const int r0 = qblock * kBlockM;
+  const int h0 = g * p.heads_per_group + 2 * pair;
+  const int nslots = min(2, p.heads_per_group - 2 * pair);
+  const int qpos0 = it.prefix + r0;
+  const int kv_len = it.prefix + it.len;
+  const int kv_end = min(qpos0 + kBlockM, kv_len);
+  const int n_kv = (kv_end + kBlockN - 1) / kBlockN;
+  const int n_unmasked = (qpos0 + 1) / kBlockN;  // tiles wholly at or below the diagonal
+
+  // ---- setup --------------------------------------------------------------
+  if (warp == 1) {
+    tmem_alloc(base + L::kTmemSlot, kTmemCols);
+    tmem_relinquish();
+  }
+  if (threadIdx.x == 0) {
+    mbar_init(bar(L::kBarQ), 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(bar(L::kBarFull + s), 1);
+      mbar_init(bar(L::kBarEmpty + s), 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(bar(L::kBarS + s), 1);
+      mbar_init(bar(L::kBarP + s), 4);  // one arrive per softmax warp
+      mbar_init(bar(L::kBarO + s), 1);
+    }
+    mbar_init(bar(L::kBarDrain), 1);
+    fence_mbar_init();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ===================== TMA producer =====================================
+    if (lane == 0) {
+      const CUtensorMap *mq = &p.tq[item];
+      const CUtensorMap *mk = &p.tk[item];
+      const CUtensorMap *mv = &p.tv[item];
+      prefetch_tmap(mq);
+      prefetch_tmap(mk);
+      prefetch_tmap(mv);
+      mbar_arrive_expect_tx(bar(L::kBarQ), nslots * L::kTileBytes);
+      for (int s = 0; s < nslots; ++s)
+        for (int c = 0; c < D / kBoxCols; ++c)
+          tma_load_3d(base + L::kQ + s * L::kTileBytes + c * kBoxBytes, mq, bar(L::kBarQ),
+                      c * kBoxCols, h0 + s, r0);
+      const int n_seq = 2 * n_kv;  // K_0, V_0, K_1, V_1, ...
+      bool ok = true;
+      int seq = 0;
+      for (; seq < n_seq; ++seq) {
+        const int st = seq % kStages;
+        if (seq >= kStages &&
+            !mbar_wait(bar(L::kBarEmpty + st), ((seq / kStages) - 1) & 1, p.status)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(bar(L::kBarFull + st), L::kTileBytes);
+        const CUtensorMap *m = (seq & 1) ? mv : mk;
+        const int key0 = (seq >> 1) * kBlockN;
+        for (int c = 0; c < D / kBoxCols; ++c)
+          tma_load_3d(base + L::kRing + st * L::kTileBytes + c * kBoxBytes, m,
+                      bar(L::kBarFull + st), c * kBoxCols, g, key0);
+      }
+      // Copies still in flight land before the CTA may exit.
+      mbar_wait(bar(L::kBarQ), 0, p.status, kDrainLimitNs, false);
+      for (int s2 = max(0, seq - kStages); s2 < seq; ++s2)
+        mbar_wait(bar(L::kBarFull + s2 % kStages), (s2 / kStages) & 1, p.status, kDrainLimitNs,
+                  false);
+      // Normal exit: the last stage releases (tcgen05.commit arrivals) landed.
+      if (ok)
+        for (int s2 = max(0, n_seq - kStages); s2 < n_seq; ++s2)
+          if (!mbar_wait(bar(L::kBarEmpty + s2 % kStages), (s2 / kStages) & 1, p.status)) break;
+    }
+  } else if (warp == 1) {
+    // ===================== MMA issuer =======================================
+    if (lane == 0) {
+      const uint32_t q_smem = base + L::kQ;
+      auto stage_smem = [&](int seq) -> uint32_t {
+        return base + L::kRing + (seq % kStages) * L::kTileBytes;
+      };
+      bool ok = mbar_wait(bar(L::kBarQ), 0, p.status) &&
+                mbar_wait(bar(L::kBarFull + 0), 0, p.status);
+      if (ok) {
+        tc_fence_after();
+        for (int s = 0; s < nslots; ++s) {
+          issue_qk<D>(tmem + s * kBlockN, q_smem + s * L::kTileBytes, stage_smem(0));
+          tc_commit(bar(L::kBarS + s));
+        }
+        tc_commit(bar(L::kBarEmpty + 0));
+        for (int j = 0; j < n_kv && ok; ++j) {
+          const int sv = 2 * j + 1;
+          const int sk = 2 * j + 2;
+          const bool has_next = j + 1 < n_kv;
+          ok = mbar_wait(bar(L::kBarFull + sv % kStages), (sv / kStages) & 1, p.status);
+          if (ok && has_next)
+            ok = mbar_wait(bar(L::kBarFull + sk % kStages), (sk / kStages) & 1, p.status);
+          if (!ok) break;
+          tc_fence_after();
+          for (int s = 0; s < nslots; ++s) {
+            ok = mbar_wait(bar(L::kBarP + s), j & 1, p.status);
+            if (!ok) break;
+            tc_fence_after();
+            issue_pv<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, stage_smem(sv), j > 0);
+            if (has_next) {
+              issue_qk<D>(tmem + s * kBlockN, q_smem + s * L::kTileBytes, stage_smem(sk));
+              tc_commit(bar(L::kBarS + s));
+            } else {
+              tc_commit(bar(L::kBarO + s));
+            }
+          }
+          if (!ok) break;
+          tc_commit(bar(L::kBarEmpty + sv % kStages));
+          if (has_next) tc_commit(bar(L::kBarEmpty + sk % kStages));
+        }
+      }
+      // Every issued MMA completes before TMEM is released.
+      tc_commit(bar(L::kBarDrain));
+      mbar_wait(bar(L::kBarDrain), 0, p.status, kDrainLimitNs, false);
+    }
+  } else {
+    // ===================== softmax / epilogue ===============================
+    const int s = static_cast<int>(warp - 2) / 4;
+    if (s < nslots) {
+      const uint32_t quarter = warp & 3u;
+      const int row = static_cast<int>(quarter * 32 + lane);
+      const uint32_t lane_addr = tmem + ((quarter * 32u) << 16);
+      const uint32_t s_addr = lane_addr + s * kBlockN;
+      const uint32_t o_addr = lane_addr + 2 * kBlockN + s * D;
+      const int qpos = qpos0 + row;
+      const float sl2 = p.scale_log2;
+      float m = -INFINITY;  // running max of scale*log2(e)*s, possibly stale by < 2^8
+      float l = 0.f;        // running sum of fp32 probabilities
+      bool ok = true;
+      for (int j = 0; j < n_kv; ++j) {
+        if (!mbar_wait_warp(bar(L::kBarS + s), j & 1, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float x[128];
+        tmem_ld128<D>(s_addr, x);
+        if (j >= n_unmasked) {
+          const int lim = qpos - j * kBlockN;  // last visible column of this row
+#pragma unroll
+          for (int c = 0; c < 128; ++c)
+            if (c > lim) x[c] = -INFINITY;
+        }
+        float tmax = x[0];
+#pragma unroll
+        for (int c = 1; c < 128; ++c) tmax = fmaxf(tmax, x[c]);
+        const float mt = tmax * sl2;
+        if (j == 0) {
+          m = mt;  // key 0 is visible to every row: finite
+        } else if (__any_sync(0xffffffffu, mt > m + kMaxGrowthLog2)) {
+          // Rare: the running max grew by more than 2^8.  Rescale O and l,
+          // then re-read S so its registers are free during the rescale.
+          const float mn = fmaxf(m, mt);
+          const float f = ex2_approx(m - mn);
+          l *= f;
+          m = mn;
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld32(o_addr + c * 32, r);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * f);
+            tmem_st32(o_addr + c * 32, r);
+          }
+          tmem_st_wait();
+          tmem_ld128<D>(s_addr, x);
+          if (j >= n_unmasked) {
+            const int lim = qpos - j * kBlockN;
+#pragma unroll
+            for (int c = 0; c < 128; ++c)
+              if (c > lim) x[c] = -INFINITY;
+          }
+        }
+        const float neg_m = -m;
+        float sum0 = 0.f, sum1 = 0.f;
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const float a = ex2_approx(fmaf(x[cc * 32 + 2 * e], sl2, neg_m));
+            const float b = ex2_approx(fmaf(x[cc * 32 + 2 * e + 1], sl2, neg_m));
+            sum0 += a;
+            sum1 += b;
+            pk[e] = pack_bf16(a, b);
+          }
+          tmem_st16(s_addr + cc * 16, pk);  // P columns 16cc .. 16cc+15 alias S
+        }
+        l += sum0 + sum1;
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(L::kBarP + s));
+      }
+      if (ok) ok = mbar_wait_warp(bar(L::kBarO + s), 0, p.status);
+      if (ok) {
+        tc_fence_after();
+        const float inv = 1.0f / l;
+        const bool valid = r0 + row < it.len;
+        const int64_t orow = it.q_row + r0 + row;
+        __nv_bfloat16 *dst = p.out + (orow * p.n_q_heads + h0 + s) * D;
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(o_addr + c * 32, r);
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e)
+            pk[e] = pack_bf16(__uint_as_float(r[2 * e]) * inv, __uint_as_float(r[2 * e + 1]) * inv);
+          if (valid) {
+            uint4 *d4 = reinterpret_cast<uint4 *>(dst + c * 32);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              d4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+          }
+        }
+        if (valid)
+          p.lse[static_cast<int64_t>(h0 + s) * p.lse_stride + orow] =
+              (m + log2f(l)) * 0.69314718055994530942f;
+      }
+    }
+  }
+
+  // ---- teardown -------------------------------------------------------------
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ host --
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *ptr = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// [rows, heads, d] bf16 tensor, box = 64 columns x 1 head x 128 rows, 128B swizzle.
+bool make_map(CUtensorMap *map, const void *ptr, int64_t rows, int heads, int d) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(heads),
+                        static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2,
+                           static_cast<cuuint64_t>(heads) * static_cast<cuuint64_t>(d) * 2};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(kBoxCols), 1u, static_cast<cuuint32_t>(kBlockM)};
+  cuuint32_t elem[3] = {1u, 1u, 1u};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box,
+            elem, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct Shape {
+  int n_q_heads, n_kv_heads, head_dim;
+};
+
+mocap_status check_shape(const Shape &sh, float scale) {
+  if (sh.n_q_heads < 1 || sh.n_kv_heads < 1 || sh.n_q_heads % sh.n_kv_heads != 0)
+    return MOCAP_EINVAL;
+  if (!(scale > 0.0f) || !std::isfinite(scale)) return MOCAP_EINVAL;
+  if (sh.head_dim != 64 && sh.head_dim != 128) return MOCAP_EUNSUPPORTED;
+  return MOCAP_OK;
+}
+
+struct HostItem {
+  int64_t q_row, kv_row, prefix, len;
+};
+
+template <int D, int MAXI>
+mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
+                    const std::vector<HostItem> &items, int64_t lse_stride, const Shape &sh,
+                    float scale, void *out, float *lse, cudaStream_t stream) {
+  using L = Layout<D>;
+  static AttnParams<MAXI> prm;  // large: build in static storage, guarded below
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lock(mu);
+  std::memset(&prm, 0, sizeof(prm));
+  uint32_t *status = device_status_ptr();
+  if (status == nullptr) return MOCAP_ECUDA;
+  const int group = sh.n_q_heads / sh.n_kv_heads;
+  const int pairs = (group + 1) / 2;
+  int64_t ctas = 0;
+  int n = 0;
+  const size_t qrow_bytes = static_cast<size_t>(sh.n_q_heads) * D * 2;
+  const size_t kvrow_bytes = static_cast<size_t>(sh.n_kv_heads) * D * 2;
+  for (const HostItem &h : items) {
+    const auto *qb = static_cast<const uint8_t *>(q) + h.q_row * qrow_bytes;
+    const auto *kb = static_cast<const uint8_t *>(k_cache) + h.kv_row * kvrow_bytes;
+    const auto *vb = static_cast<const uint8_t *>(v_cache) + h.kv_row * kvrow_bytes;
+    if (!make_map(&prm.tq[n], qb, h.len, sh.n_q_heads, D) ||
+        !make_map(&prm.tk[n], kb, h.prefix + h.len, sh.n_kv_heads, D) ||
+        !make_map(&prm.tv[n], vb, h.prefix + h.len, sh.n_kv_heads, D))
+      return MOCAP_ECUDA;
+    ItemDesc &d = prm.items[n];
+    d.q_row = h.q_row;
+    d.prefix = static_cast<int32_t>(h.prefix);
+    d.len = static_cast<int32_t>(h.len);
+    d.q_blocks = static_cast<int32_t>((h.len + kBlockM - 1) / kBlockM);
+    d.cta_begin = static_cast<int32_t>(ctas);
+    ctas += static_cast<int64_t>(d.q_blocks) * sh.n_kv_heads * pairs;
+    ++n;
+  }
+  if (n == 0) return MOCAP_OK;
+  if (ctas > 0x7fffffff) return MOCAP_EINVAL;
+  prm.out = static_cast<__nv_bfloat16 *>(out);
+  prm.lse = lse;
+  prm.status = status;
+  prm.lse_stride = lse_stride;
+  prm.n_items = n;
+  prm.n_q_heads = sh.n_q_heads;
+  prm.n_kv_heads = sh.n_kv_heads;
+  prm.heads_per_group = group;
+  prm.pairs_per_group = pairs;
+  prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
+
+  auto kern = chunk_attn_kernel<D, MAXI>;
+  static bool attr_done[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
+  if (!attr_done[dev]) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes) !=
+        cudaSuccess)
+      return MOCAP_ECUDA;
+    attr_done[dev] = true;
+  }
+  kern<<<static_cast<unsigned>(ctas), kThreads, L::kBytes, stream>>>(prm);
+  return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+}
+
+template <int MAXI>
+mocap_status dispatch(const void *q, const void *k_cache, const void *v_cache,
+                      const std::vector<HostItem> &items, int64_t lse_stride, const Shape &sh,
+                      float scale, void *out, float *lse, cudaStream_t stream) {
+  if (sh.head_dim == 128)
+    return launch<128, MAXI>(q, k_cache, v_cache, items, lse_stride, sh, scale, out, lse, stream);
+  return launch<64, MAXI>(q, k_cache, v_cache, items, lse_stride, sh, scale, out, lse, stream);
+}
+
+bool pointers_ok(const void *q, const void *k, const void *v, const void *out, const float *lse) {
+  if (!q || !k || !v || !out || !lse) return false;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out)) return false;
+  return (reinterpret_cast<uintptr_t>(lse) & 3u) == 0;
+}
+
+constexpr int64_t kMaxRows = 0x7fffffffLL;
+
+}  // namespace
+}  // namespace mocap
+
+using mocap::HostItem;
+
+extern "C" size_t mocap_chunk_attn_workspace_size(int64_t, int64_t, int32_t, int32_t) { return 0; }
+
+extern "C" mocap_status mocap_chunk_attn(const void *q, const void *k_cache, const void *v_cache,
+                                         int64_t prefix, int64_t len, int32_t n_q_heads,
+                                         int32_t n_kv_heads, int32_t head_dim, float scale,
+                                         void *out, float *lse, void *workspace,
+                                         size_t workspace_bytes, mocap_stream_t stream) {
+  (void)workspace;
+  (void)workspace_bytes;
+  const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
+  const mocap_status st = mocap::check_shape(sh, scale);
+  if (st != MOCAP_OK) return st;
+  if (prefix < 0 || len < 0 || prefix > mocap::kMaxRows - len) return MOCAP_EINVAL;
+  if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
+  if (len == 0) return MOCAP_OK;
+  std::vector<HostItem> items{{0, 0, prefix, len}};
+  return mocap::dispatch<1>(q, k_cache, v_cache, items, len, sh, scale, out, lse,
+                            reinterpret_cast<cudaStream_t>(stream));
+}
+
+extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache,
+                                                const void *v_cache,
+                                                const mocap_varlen_item *items, int32_t n_items,
+                                                int64_t q_rows_total, int64_t kv_rows_total,
+                                                int32_t n_q_heads, int32_t n_kv_heads,
+                                                int32_t head_dim, float scale, void *out,
+                                                float *lse, mocap_stream_t stream) {
+  const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
+  const mocap_status st = mocap::check_shape(sh, scale);
+  if (st != MOCAP_OK) return st;
+  if (n_items < 0 || n_items > MOCAP_VARLEN_MAX_ITEMS) return MOCAP_EINVAL;
+  if (n_items > 0 && items == nullptr) return MOCAP_EINVAL;
+  if (q_rows_total < 0 || kv_rows_total < 0) return MOCAP_EINVAL;
+  if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
+  std::vector<HostItem> list;
+  for (int i = 0; i < n_items; ++i) {
+    const mocap_varlen_item &x = items[i];
+    if (x.q_row < 0 || x.kv_row < 0 || x.prefix < 0 || x.len < 0) return MOCAP_EINVAL;
+    if (x.prefix > mocap::kMaxRows - x.len) return MOCAP_EINVAL;
+    if (x.q_row > q_rows_total - x.len) return MOCAP_EINVAL;
+    if (x.kv_row > kv_rows_total - (x.prefix + x.len)) return MOCAP_EINVAL;
+    if (x.len > 0) list.push_back({x.q_row, x.kv_row, x.prefix, x.len});
+  }
+  if (list.empty()) return MOCAP_OK;
+  // Heaviest items first (their last row blocks see the most keys).
+  std::stable_sort(list.begin(), list.end(), [](const HostItem &a, const HostItem &b) {
+    return a.prefix + a.len > b.prefix + b.len;
+  });
+  return mocap::dispatch<MOCAP_VARLEN_MAX_ITEMS>(q, k_cache, v_cache, list, q_rows_total, sh,
+                                                 scale, out, lse,
+                                                 reinterpret_cast<cudaStream_t>(stream));
+}

@@ -1,0 +1,91 @@
+// kv_append.cu -- append one chunk's K and V rows to the contiguous KV cache.
+//
+// Sec. 2.2 / Sec. 3.1: every chunk's KV stays live for the chunks after it.
+// The cache is [capacity, n_kv_heads, head_dim] bf16 row-major, so rows
+// [offset, offset + len) of the cache are one contiguous byte range and the
+// append is a straight 16-byte-vector copy of two ranges (K and V) in a single
+// launch.  HBM-bound: 2 tensors x (read + write) x len x Hkv x d x 2 bytes.
+#include <algorithm>
+
+#include "internal.h"
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kUnroll = 4;
+
+__device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+// Vectors [0, n) come from k_src -> k_dst, vectors [n, 2n) from v_src -> v_dst.
+__global__ void __launch_bounds__(kThreads) kv_append_kernel(const uint4 *__restrict__ k_src,
+                                                             const uint4 *__restrict__ v_src,
+                                                             uint4 *__restrict__ k_dst,
+                                                             uint4 *__restrict__ v_dst,
+                                                             int64_t n) {
+  const int64_t total = 2 * n;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads * kUnroll;
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * kThreads * kUnroll + threadIdx.x;
+       base < total; base += stride) {
+    uint4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = base + static_cast<int64_t>(u) * kThreads;
+      if (i < total) v[u] = ld_stream(i < n ? k_src + i : v_src + (i - n));
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = base + static_cast<int64_t>(u) * kThreads;
+      if (i < total) {
+        if (i < n) k_dst[i] = v[u];
+        else v_dst[i - n] = v[u];
+      }
+    }
+  }
+}
+
+int sm_count() {
+  static int cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+}  // namespace
+
+extern "C" mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk, void *k_cache,
+                                        void *v_cache, int64_t cache_capacity, int64_t offset,
+                                        int64_t len, int32_t n_kv_heads, int32_t head_dim,
+                                        mocap_stream_t stream) {
+  if (!k_chunk || !v_chunk || !k_cache || !v_cache) return MOCAP_EINVAL;
+  if (!mocap::aligned16(k_chunk) || !mocap::aligned16(v_chunk) || !mocap::aligned16(k_cache) ||
+      !mocap::aligned16(v_cache))
+    return MOCAP_EINVAL;
+  if (n_kv_heads < 1 || head_dim < 1 || offset < 0 || len < 0 || cache_capacity < 0)
+    return MOCAP_EINVAL;
+  const int64_t row_elems = static_cast<int64_t>(n_kv_heads) * head_dim;
+  if (row_elems % 8 != 0) return MOCAP_EINVAL;  // rows must be whole 16-byte vectors
+  if (offset > cache_capacity || len > cache_capacity - offset) return MOCAP_EINVAL;
+  if (len == 0) return MOCAP_OK;
+
+  const int64_t n = len * row_elems / 8;  // 16-byte vectors per tensor
+  const int64_t dst_off = offset * row_elems / 8;
+  const int64_t want = (2 * n + kThreads * kUnroll - 1) / (kThreads * kUnroll);
+  const int64_t cap = static_cast<int64_t>(sm_count()) * 8;
+  const int blocks = static_cast<int>(std::max<int64_t>(1, std::min(want, cap)));
+  kv_append_kernel<<<blocks, kThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      static_cast<const uint4 *>(k_chunk), static_cast<const uint4 *>(v_chunk),
+      static_cast<uint4 *>(k_cache) + dst_off, static_cast<uint4 *>(v_cache) + dst_off, n);
+  return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+}

@@ -1,0 +1,51 @@
+// status.cu -- device status word for bounded-wait timeouts, status strings.
+#include <mutex>
+
+#include "internal.h"
+
+namespace {
+__device__ uint32_t g_device_status;  // 0 = OK, MOCAP_ETIMEOUT after an expired wait
+
+constexpr int kMaxDevices = 64;
+uint32_t *g_status_ptr[kMaxDevices] = {};
+std::mutex g_status_mu;
+}  // namespace
+
+namespace mocap {
+
+uint32_t *device_status_ptr() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_status_mu);
+  if (g_status_ptr[dev] == nullptr) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
+    g_status_ptr[dev] = static_cast<uint32_t *>(p);
+  }
+  return g_status_ptr[dev];
+}
+
+}  // namespace mocap
+
+extern "C" mocap_status mocap_last_device_status(mocap_stream_t stream) {
+  uint32_t *p = mocap::device_status_ptr();
+  if (p == nullptr) return MOCAP_ECUDA;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t value = 0;
+  if (cudaMemcpyAsync(&value, p, sizeof(value), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return MOCAP_ECUDA;
+  if (cudaMemsetAsync(p, 0, sizeof(uint32_t), s) != cudaSuccess) return MOCAP_ECUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return MOCAP_ECUDA;
+  return value == 0 ? MOCAP_OK : static_cast<mocap_status>(value);
+}
+
+extern "C" const char *mocap_status_string(mocap_status status) {
+  switch (status) {
+    case MOCAP_OK: return "MOCAP_OK";
+    case MOCAP_EINVAL: return "MOCAP_EINVAL: invalid argument";
+    case MOCAP_ECUDA: return "MOCAP_ECUDA: CUDA call failed";
+    case MOCAP_EUNSUPPORTED: return "MOCAP_EUNSUPPORTED: unsupported shape";
+    case MOCAP_ETIMEOUT: return "MOCAP_ETIMEOUT: device wait expired";
+  }
+  return "MOCAP_UNKNOWN";
+}

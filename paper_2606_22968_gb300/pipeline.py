@@ -1,0 +1,106 @@
+"""Chunked prefill over a whole prompt on one GPU: partition, append, attend.
+
+This walks the chunks of each request in order, exactly as one stage of the
+chunked pipeline does (Sec. 2.2): chunk i's K/V are appended to the request's
+KV cache and its queries attend to everything cached so far.  Boundaries come
+from LBCP (Sec. 3.2 / Sec. 4.2) or the uniform split.  Every step is a call
+into libmocap.so; torch only allocates memory and provides the stream.
+"""
+
+from __future__ import annotations
+
+from typing import List, Optional
+
+import torch
+
+from . import (MOCAP_PART_LBCP, MOCAP_PART_UNIFORM, mocap_chunk_attn, mocap_chunk_attn_varlen,
+               mocap_kv_append, mocap_lbcp_partition)
+from .workloads import GRANULARITY, Workload, request_offsets
+
+
+class ChunkedPrefill:
+    """Buffers and launch sequence for one workload on one device.
+
+    Single-request workloads launch ``mocap_chunk_attn`` once per chunk, with
+    chunk i's LSE in its own ``[Hq, c_i]`` block of ``lse`` (offset Hq*b_i).
+    Multi-request workloads launch ``mocap_chunk_attn_varlen`` once per chunk
+    index k over every request that has a chunk k; ``lse`` is then one
+    ``[Hq, T]`` array over the packed rows.
+    """
+
+    def __init__(self, w: Workload, device, mode: Optional[int] = None):
+        self.w = w
+        self.device = torch.device(device)
+        self.mode = w.mode if mode is None else mode
+        self.bounds: List[List[int]] = []
+        self.partition()
+        self.cu = request_offsets(w)
+        total = w.total_tokens
+        kw = dict(device=self.device, dtype=torch.bfloat16)
+        self.k_cache = torch.empty((total, w.n_kv_heads, w.head_dim), **kw)
+        self.v_cache = torch.empty((total, w.n_kv_heads, w.head_dim), **kw)
+        self.out = torch.empty((total, w.n_q_heads, w.head_dim), **kw)
+        self.lse = torch.empty((w.n_q_heads * total,), device=self.device, dtype=torch.float32)
+        self.single = len(w.seq_lens) == 1
+
+    def partition(self):
+        """Chunk boundaries of every request (host call into the library)."""
+        part_mode = MOCAP_PART_LBCP if self.mode == 1 else MOCAP_PART_UNIFORM
+        self.bounds = [mocap_lbcp_partition(s, m, GRANULARITY, part_mode)
+                       for s, m in zip(self.w.seq_lens, self.w.num_chunks)]
+        return self.bounds
+
+    # -- launch plan -----------------------------------------------------------
+    def steps(self):
+        """List of launch steps; each is a list of (request, chunk index)."""
+        n_steps = max(len(b) - 1 for b in self.bounds)
+        return [[(r, k) for r in range(len(self.bounds)) if k < len(self.bounds[r]) - 1]
+                for k in range(n_steps)]
+
+    def chunk_lse(self, i: int) -> torch.Tensor:
+        """Single request: chunk i's LSE block [Hq, c_i]."""
+        b = self.bounds[0]
+        hq = self.w.n_q_heads
+        return self.lse[hq * b[i]:hq * b[i + 1]].view(hq, b[i + 1] - b[i])
+
+    def lse_packed(self) -> torch.Tensor:
+        """Multi-request: the [Hq, T] LSE array."""
+        return self.lse.view(self.w.n_q_heads, self.w.total_tokens)
+
+    # -- execution ----------------------------------------------------------------
+    def run_step(self, q, k, v, step, stream=None, events=None):
+        """Append + attention for one step (one chunk index).  ``events`` is
+        an optional triple of CUDA events recorded before the appends, between
+        appends and attention, and after the attention."""
+        w = self.w
+        if events is not None:
+            events[0].record(stream)
+        for r, c in step:
+            b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
+            base = self.cu[r]
+            mocap_kv_append(k[base + b0:base + b1], v[base + b0:base + b1],
+                            self.k_cache[base:base + w.seq_lens[r]],
+                            self.v_cache[base:base + w.seq_lens[r]], b0, stream=stream)
+        if events is not None:
+            events[1].record(stream)
+        if self.single:
+            (_, c), = step
+            b0, b1 = self.bounds[0][c], self.bounds[0][c + 1]
+            mocap_chunk_attn(q[b0:b1], self.k_cache, self.v_cache, b0, self.out[b0:b1],
+                             self.chunk_lse(c), w.scale, stream=stream)
+        else:
+            items = []
+            for r, c in step:
+                b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
+                items.append((self.cu[r] + b0, self.cu[r], b0, b1 - b0))
+            mocap_chunk_attn_varlen(q, self.k_cache, self.v_cache, items, self.out,
+                                    self.lse_packed(), w.scale, stream=stream)
+        if events is not None:
+            events[2].record(stream)
+
+    def run(self, q, k, v, stream=None, chunk_events=None):
+        """The whole prompt: every step in order.  ``chunk_events`` optionally
+        holds one event triple per step (see run_step)."""
+        for i, step in enumerate(self.steps()):
+            self.run_step(q, k, v, step, stream,
+                          None if chunk_events is None else chunk_events[i])

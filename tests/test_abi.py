@@ -1,0 +1,156 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds and
+exports every entry point include/mocap.h declares, the host partition is
+bit-exact against the oracle, and invalid arguments are rejected before any
+CUDA call."""
+
+import ctypes
+import os
+import random
+import re
+
+import pytest
+
+from oracle import partition as P
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    names = set()
+    inc = os.path.join(ROOT, "include")
+    for f in os.listdir(inc):
+        if f.endswith(".h"):
+            text = open(os.path.join(inc, f)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names |= set(re.findall(r"\b(mocap_[a-z0-9_]+)\s*\(", text))
+    return names
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ["mocap_lbcp_partition", "mocap_kv_append", "mocap_chunk_attn",
+              "mocap_chunk_attn_workspace_size", "mocap_chunk_attn_varlen",
+              "mocap_last_device_status", "mocap_status_string"]:
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared():
+        assert hasattr(lib, name), name
+
+
+def test_build_entry_compiles_for_sm103a():
+    import __graft_entry__  # noqa: F401
+    from paper_2606_22968_gb300 import _build
+    assert "arch=compute_103a,code=sm_103a" in " ".join(_build.ARCH)
+    assert os.path.exists(_build.build())
+
+
+def _c_partition(lib, s, m, g, mode):
+    out = (ctypes.c_int64 * (m + 1))()
+    st = lib.mocap_lbcp_partition(s, m, g, mode, out)
+    return st, list(out)
+
+
+def test_partition_bit_exact_vs_oracle_sweep(lib):
+    for units in range(1, 2049, 7):
+        for m in (1, 2, 3, 4, 5, 8, 16, 31, 32, 64):
+            if m > units:
+                continue
+            for mode in (0, 1):
+                s = units * 128
+                st, b = _c_partition(lib, s, m, 128, mode)
+                assert st == 0
+                assert b == P.boundaries(s, m, 128, mode), (s, m, mode)
+
+
+def test_partition_random_ragged_vs_oracle(lib):
+    rnd = random.Random(1)
+    for _ in range(3000):
+        g = rnd.choice([1, 16, 64, 128, 256])
+        s = rnd.randint(1, 1 << 24)
+        m = rnd.randint(1, 200)
+        if m * g > s:
+            continue
+        mode = rnd.randint(0, 1)
+        st, b = _c_partition(lib, s, m, g, mode)
+        assert st == 0 and b == P.boundaries(s, m, g, mode)
+
+
+def test_partition_large_sequences(lib):
+    for s, m in [(1 << 30, 1000), ((1 << 37) - 5, 4096), (131072, 32)]:
+        st, b = _c_partition(lib, s, m, 128, 1)
+        assert st == 0 and b == P.boundaries(s, m, 128, 1)
+
+
+def test_partition_invalid(lib):
+    out = (ctypes.c_int64 * 10)()
+    assert lib.mocap_lbcp_partition(0, 1, 128, 1, out) == 1
+    assert lib.mocap_lbcp_partition(1024, 0, 128, 1, out) == 1
+    assert lib.mocap_lbcp_partition(1024, 9, 128, 1, out) == 1
+    assert lib.mocap_lbcp_partition(1024, 2, 0, 1, out) == 1
+    assert lib.mocap_lbcp_partition(1024, 2, 128, 7, out) == 1
+    assert lib.mocap_lbcp_partition(1024, 2, 128, 1, None) == 1
+    assert lib.mocap_lbcp_partition(1 << 40, 2, 1, 1, out) == 1  # U >= 2^30
+
+
+def test_status_strings(lib):
+    for code in range(5):
+        assert lib.mocap_status_string(code).startswith(b"MOCAP_")
+
+
+FAKE = 1 << 20  # a 16-byte-aligned non-null value; never dereferenced
+
+
+def test_kv_append_rejects_bad_arguments_before_launch(lib):
+    f = lib.mocap_kv_append
+    assert f(None, FAKE, FAKE, FAKE, 10, 0, 1, 8, 128, None) == 1
+    assert f(FAKE + 2, FAKE, FAKE, FAKE, 10, 0, 1, 8, 128, None) == 1      # misaligned
+    assert f(FAKE, FAKE, FAKE, FAKE, 10, 8, 3, 8, 128, None) == 1           # past capacity
+    assert f(FAKE, FAKE, FAKE, FAKE, 10, -1, 1, 8, 128, None) == 1
+    assert f(FAKE, FAKE, FAKE, FAKE, 10, 0, -1, 8, 128, None) == 1
+    assert f(FAKE, FAKE, FAKE, FAKE, 10, 0, 1, 1, 4, None) == 1             # 4 elems: not 16 B
+    assert f(FAKE, FAKE, FAKE, FAKE, 10, 3, 0, 8, 128, None) == 0           # empty: no-op
+
+
+def test_chunk_attn_rejects_bad_arguments_before_launch(lib):
+    f = lib.mocap_chunk_attn
+    ok = dict(prefix=0, length=128, hq=8, hkv=2, d=128, scale=0.088)
+
+    def call(**kw):
+        a = dict(ok, **kw)
+        return f(kw.get("q", FAKE), FAKE, FAKE, a["prefix"], a["length"], a["hq"], a["hkv"], a["d"],
+                 a["scale"], FAKE, kw.get("lse", FAKE), None, 0, None)
+
+    assert call(q=None) == 1
+    assert call(q=FAKE + 8) == 1
+    assert call(lse=FAKE + 2) == 1
+    assert call(hq=6, hkv=4) == 1
+    assert call(hkv=0) == 1
+    assert call(scale=0.0) == 1
+    assert call(scale=float("nan")) == 1
+    assert call(scale=-1.0) == 1
+    assert call(prefix=-1) == 1
+    assert call(length=-5) == 1
+    assert call(prefix=(1 << 31) - 10, length=20) == 1
+    assert call(d=96) == 3
+    assert call(d=256) == 3
+    assert call(length=0) == 0
+
+
+def test_varlen_rejects_bad_items_before_launch(lib):
+    from paper_2606_22968_gb300._lib import VarlenItem
+    f = lib.mocap_chunk_attn_varlen
+
+    def call(items, q_rows=1000, kv_rows=1000, n=None):
+        arr = (VarlenItem * max(1, len(items)))(*[VarlenItem(*x) for x in items])
+        return f(FAKE, FAKE, FAKE, arr, len(items) if n is None else n, q_rows, kv_rows, 8, 2, 128,
+                 0.1, FAKE, FAKE, None)
+
+    assert call([(0, 0, 0, 10)], q_rows=5) == 1          # q rows past the buffer
+    assert call([(0, 0, 995, 10)]) == 1                  # kv rows past the cache
+    assert call([(-1, 0, 0, 10)]) == 1
+    assert call([(0, 0, 0, 10)], n=65) == 1              # too many items
+    assert call([(0, 0, 0, 10)], n=-1) == 1
+    assert call([]) == 0
+    assert call([(0, 0, 5, 0)]) == 0                     # empty item: no-op

@@ -1,0 +1,251 @@
+"""GPU parity: the CUDA path (through the C ABI) against the float64 oracle.
+
+Small cases compare every output element; the five workloads at full size
+compare sampled rows of every chunk (first/last rows, rows around every
+128-row tile boundary, a stride and random rows).  Tolerances: O max-abs
+2e-2 and mean-abs 2e-3, LSE max-abs 1e-3.  KV-cache contents are compared
+bit for bit.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import attention as A
+from oracle import partition as P
+from tests.parity_utils import (LSE_MAX_ABS, O_MAX_ABS, assert_close, check_single_request,
+                                chunk_rows_oracle, f64, sample_rows)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def m():
+    import paper_2606_22968_gb300 as mod
+    mod._lib.load()
+    return mod
+
+
+def _randn(shape, gen, dev):
+    return torch.randn(shape, generator=gen, device=dev, dtype=torch.bfloat16)
+
+
+def run_explicit(m, q, k, v, bounds, scale, k_cache=None, v_cache=None):
+    """Append + attend chunk by chunk with explicit boundaries."""
+    s, hq, d = q.shape
+    hkv = k.shape[1]
+    dev = q.device
+    if k_cache is None:
+        k_cache = torch.zeros((s, hkv, d), device=dev, dtype=torch.bfloat16)
+        v_cache = torch.zeros((s, hkv, d), device=dev, dtype=torch.bfloat16)
+    out = torch.full((s, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    lses = []
+    for i in range(len(bounds) - 1):
+        b0, b1 = bounds[i], bounds[i + 1]
+        m.mocap_kv_append(k[b0:b1], v[b0:b1], k_cache, v_cache, b0)
+        lse = torch.full((hq, b1 - b0), float("nan"), device=dev, dtype=torch.float32)
+        m.mocap_chunk_attn(q[b0:b1], k_cache, v_cache, b0, out[b0:b1], lse, scale)
+        lses.append(lse)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    return out, lses, k_cache, v_cache
+
+
+SMALL_CASES = [
+    # (bounds, Hq, Hkv, d)
+    ([0, 256, 512, 768, 1024], 4, 4, 64),
+    ([0, 1, 130, 300, 513], 8, 2, 128),          # 1-row chunk, unaligned prefixes
+    ([0, 700], 6, 2, 128),                        # one chunk, GQA 3:1 (odd head slot)
+    ([0, 127, 128, 129, 383, 640], 4, 1, 64),     # around tile edges, GQA 4:1
+    ([0, 200, 455], 1, 1, 128),                   # single head
+    ([0, 384, 385, 1000], 16, 2, 128),            # GQA 8:1
+    ([0, 50, 99], 2, 2, 64),                      # everything inside one tile
+]
+
+
+@pytest.mark.parametrize("bounds,hq,hkv,d", SMALL_CASES)
+def test_small_cases_all_elements(m, bounds, hq, hkv, d):
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(1234 + hq * 7 + d)
+    s = bounds[-1]
+    q, k, v = _randn((s, hq, d), gen, dev), _randn((s, hkv, d), gen, dev), _randn((s, hkv, d), gen, dev)
+    scale = 1.0 / math.sqrt(d)
+    out, lses, kc, vc = run_explicit(m, q, k, v, bounds, scale)
+    assert torch.equal(kc, k) and torch.equal(vc, v)
+    o_ref, l_ref, _, _ = A.chunked_prefill(f64(q), f64(k), f64(v), bounds, scale)
+    lse = np.concatenate([x.cpu().numpy() for x in lses], axis=1)
+    assert_close(out.float().cpu().numpy(), lse, o_ref, np.concatenate(l_ref, axis=1))
+
+
+def test_large_scale_logits(m):
+    """Peaked softmax (scores of +-40): exercises the running-max rescale."""
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(99)
+    s, hq, hkv, d = 1100, 4, 2, 128
+    q = (_randn((s, hq, d), gen, dev).float() * 3).bfloat16()
+    k = (_randn((s, hkv, d), gen, dev).float() * 3).bfloat16()
+    v = _randn((s, hkv, d), gen, dev)
+    # increasing key norms make the running max grow along the sequence
+    ramp = torch.linspace(0.2, 1.5, s, device=dev).view(s, 1, 1)
+    k = (k.float() * ramp).bfloat16()
+    bounds = [0, 300, 1100]
+    scale = 1.0 / math.sqrt(d)
+    out, lses, _, _ = run_explicit(m, q, k, v, bounds, scale)
+    o_ref, l_ref, _, _ = A.chunked_prefill(f64(q), f64(k), f64(v), bounds, scale)
+    lse = np.concatenate([x.cpu().numpy() for x in lses], axis=1)
+    assert_close(out.float().cpu().numpy(), lse, o_ref, np.concatenate(l_ref, axis=1))
+
+
+def test_closed_form_zero_queries(m):
+    """Q = 0: O[t] = mean(V[0..t]) and LSE[t] = ln(t+1), no oracle involved."""
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(5)
+    s, hq, hkv, d = 777, 8, 2, 128
+    q = torch.zeros((s, hq, d), device=dev, dtype=torch.bfloat16)
+    k, v = _randn((s, hkv, d), gen, dev), _randn((s, hkv, d), gen, dev)
+    out, lses, _, _ = run_explicit(m, q, k, v, [0, 333, 777], 0.088)
+    vf = v.double().cpu()
+    mean = torch.cumsum(vf, 0) / torch.arange(1, s + 1, dtype=torch.float64).view(s, 1, 1)
+    ref = mean.repeat_interleave(hq // hkv, dim=1)
+    err = (out.double().cpu() - ref).abs()
+    assert err.max() <= O_MAX_ABS and err.mean() <= 2e-3
+    lse = torch.cat([x.cpu() for x in lses], 1).double()
+    lref = torch.log(torch.arange(1, s + 1, dtype=torch.float64)).view(1, s).expand(hq, s)
+    assert (lse - lref).abs().max() <= LSE_MAX_ABS
+
+
+def test_closed_form_unit_values(m):
+    """V = 1: every output is 1 (up to bf16 rounding of the probabilities)."""
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(6)
+    s, hq, hkv, d = 600, 4, 4, 64
+    q, k = _randn((s, hq, d), gen, dev), _randn((s, hkv, d), gen, dev)
+    v = torch.ones((s, hkv, d), device=dev, dtype=torch.bfloat16)
+    out, _, _, _ = run_explicit(m, q, k, v, [0, 128, 600], 0.125)
+    assert (out.float() - 1.0).abs().max().item() <= 1e-2
+
+
+def test_cache_rows_past_prefix_never_read(m):
+    """NaN in cache rows >= prefix+len must not reach the output."""
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(8)
+    s, hq, hkv, d = 900, 8, 2, 128
+    q, k, v = _randn((s, hq, d), gen, dev), _randn((s, hkv, d), gen, dev), _randn((s, hkv, d), gen, dev)
+    bounds = [0, 300, 650, 900]
+    nan_k = torch.full((s, hkv, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    nan_v = nan_k.clone()
+    out_nan, l_nan, _, _ = run_explicit(m, q, k, v, bounds, 0.088, nan_k, nan_v)
+    out_zero, l_zero, _, _ = run_explicit(m, q, k, v, bounds, 0.088)
+    assert torch.equal(out_nan, out_zero)
+    for a, b in zip(l_nan, l_zero):
+        assert torch.equal(a, b)
+
+
+def test_chunked_matches_single_chunk_on_gpu(m):
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(9)
+    s, hq, hkv, d = 2048, 8, 2, 128
+    q, k, v = _randn((s, hq, d), gen, dev), _randn((s, hkv, d), gen, dev), _randn((s, hkv, d), gen, dev)
+    one, l1, _, _ = run_explicit(m, q, k, v, [0, s], 0.088)
+    many, lm, _, _ = run_explicit(m, q, k, v, P.boundaries(s, 5, 128), 0.088)
+    assert (one.float() - many.float()).abs().max().item() <= 1e-2
+    assert (torch.cat(lm, 1) - l1[0]).abs().max().item() <= 5e-4
+
+
+def test_varlen_equals_single_launches_bitwise(m):
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(10)
+    hq, hkv, d = 8, 2, 128
+    lens = [300, 1000, 129, 640]
+    cu = np.concatenate([[0], np.cumsum(lens)]).tolist()
+    t = cu[-1]
+    q, k, v = _randn((t, hq, d), gen, dev), _randn((t, hkv, d), gen, dev), _randn((t, hkv, d), gen, dev)
+    # chunk 0 = first 40 % of every request, chunk 1 = the rest
+    cut = [int(0.4 * n) for n in lens]
+    out_v = torch.zeros((t, hq, d), device=dev, dtype=torch.bfloat16)
+    lse_v = torch.zeros((hq, t), device=dev, dtype=torch.float32)
+    out_s = torch.zeros_like(out_v)
+    lse_s = torch.zeros_like(lse_v)
+    for step in range(2):
+        items = []
+        for r in range(len(lens)):
+            b0, b1 = (0, cut[r]) if step == 0 else (cut[r], lens[r])
+            items.append((cu[r] + b0, cu[r], b0, b1 - b0))
+        m.mocap_chunk_attn_varlen(q, k, v, items, out_v, lse_v, 0.088)
+        for (qr, kr, pre, ln) in items:
+            lse_tmp = torch.zeros((hq, ln), device=dev, dtype=torch.float32)
+            m.mocap_chunk_attn(q[qr:qr + ln], k[kr:kr + pre + ln], v[kr:kr + pre + ln], pre,
+                               out_s[qr:qr + ln], lse_tmp, 0.088)
+            lse_s[:, qr:qr + ln] = lse_tmp
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    assert torch.equal(out_v, out_s) and torch.equal(lse_v, lse_s)
+    # and against the oracle
+    for r in range(len(lens)):
+        a, b = cu[r], cu[r + 1]
+        o_ref, l_ref = A.causal_attention(f64(q[a:b]), f64(k[a:b]), f64(v[a:b]), 0.088)
+        assert_close(out_v[a:b].float().cpu().numpy(), lse_v[:, a:b].cpu().numpy(), o_ref, l_ref,
+                     f"request {r}")
+
+
+# ---------------------------------------------------------------- workloads --
+def _workload_parity(m, index, rows_fn, chunks=None):
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(index)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev)
+    assert pf.bounds[0] == P.boundaries(w.seq_lens[0], w.num_chunks[0], 128, w.mode)
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
+    return check_single_request(pf, q, k, v, rows_fn=rows_fn, chunks=chunks)
+
+
+def test_workload1_tiny_all_elements(m):
+    _workload_parity(m, 1, None)
+
+
+def test_workload2_8k_sampled(m):
+    _workload_parity(m, 2, lambda n, i: sample_rows(n, every=61, seed=i))
+
+
+def test_workload3_32k_lbcp_sampled(m):
+    _workload_parity(m, 3, lambda n, i: sample_rows(n, every=257, seed=i))
+
+
+def test_workload4_128k_lbcp_sampled(m):
+    # the first, a middle and the last three chunks, sparsely sampled
+    _workload_parity(m, 4, lambda n, i: sample_rows(n, every=1021, edge=2, seed=i)[::3],
+                     chunks=[0, 1, 15, 29, 30, 31])
+
+
+def test_workload5_varlen_sampled(m):
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(5)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev)
+    for r in range(len(w.seq_lens)):
+        assert pf.bounds[r] == P.boundaries(w.seq_lens[r], w.num_chunks[r], 128, 1)
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
+    lse = pf.lse_packed()
+    for r in range(len(w.seq_lens)):
+        a = pf.cu[r]
+        kf, vf = f64(k[a:a + w.seq_lens[r]]), f64(v[a:a + w.seq_lens[r]])
+        b = pf.bounds[r]
+        for i in (0, len(b) - 2):
+            rows = sample_rows(b[i + 1] - b[i], every=509, edge=2, seed=r)
+            idx = torch.as_tensor(rows + a + b[i], device=dev)
+            o_ref, l_ref = chunk_rows_oracle(f64(q[idx]), kf[:b[i + 1]], vf[:b[i + 1]], b[i], rows,
+                                             w.scale)
+            assert_close(pf.out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref,
+                         l_ref, f"request {r} chunk {i}")

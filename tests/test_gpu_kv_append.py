@@ -1,0 +1,55 @@
+"""GPU: mocap_kv_append writes exactly the chunk rows, bit for bit, and no
+other cache byte (sentinel bit patterns, NaN included, must survive)."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import attention as A
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def m():
+    import paper_2606_22968_gb300 as mod
+    mod._lib.load()
+    return mod
+
+
+@pytest.mark.parametrize("cap,offset,length,hkv,d", [
+    (1000, 0, 1000, 8, 128),
+    (1000, 3, 1, 8, 128),
+    (4099, 1234, 2047, 8, 128),
+    (513, 511, 2, 4, 64),
+    (300, 17, 250, 1, 8),
+    (70000, 65536, 4464, 8, 128),
+])
+def test_append_bitwise_with_sentinels(m, cap, offset, length, hkv, d):
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(cap + offset)
+    sentinel = torch.randint(-32768, 32767, (cap, hkv, d), generator=gen, device=dev,
+                             dtype=torch.int16)
+    sentinel[::7] = 0x7FC1  # NaN bit patterns among the sentinels
+    kc = sentinel.clone().view(torch.bfloat16)
+    vc = (sentinel ^ 0x5555).view(torch.bfloat16)
+    k = torch.randint(-32768, 32767, (length, hkv, d), generator=gen, device=dev,
+                      dtype=torch.int16).view(torch.bfloat16)
+    v = torch.randint(-32768, 32767, (length, hkv, d), generator=gen, device=dev,
+                      dtype=torch.int16).view(torch.bfloat16)
+    kc0 = kc.view(torch.int16).cpu().numpy()
+    vc0 = vc.view(torch.int16).cpu().numpy()
+    m.mocap_kv_append(k, v, kc, vc, offset)
+    torch.cuda.synchronize()
+    k_ref = A.kv_append(kc0, k.view(torch.int16).cpu().numpy(), offset)
+    v_ref = A.kv_append(vc0, v.view(torch.int16).cpu().numpy(), offset)
+    assert np.array_equal(kc.view(torch.int16).cpu().numpy(), k_ref)
+    assert np.array_equal(vc.view(torch.int16).cpu().numpy(), v_ref)
+
+
+def test_append_rejects_overflow(m):
+    dev = torch.device("cuda")
+    kc = torch.zeros((10, 8, 128), device=dev, dtype=torch.bfloat16)
+    k = torch.zeros((4, 8, 128), device=dev, dtype=torch.bfloat16)
+    with pytest.raises(m.MocapError):
+        m.mocap_kv_append(k, k, kc, kc.clone(), 7)
