@@ -45,6 +45,9 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-rows-per-chunk", type=int, default=2)
+    ap.add_argument("--case", default=None,
+                    help="profiling case 'prefix,len,Hq,Hkv,d': one chunk attention launch "
+                         "repeated warmup+steps times (no JSON metric line)")
     return ap.parse_args()
 
 
@@ -462,8 +465,40 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
             "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
 
+def profile_case(args):
+    """A single chunk_attn launch shape, repeated: the small case for ncu."""
+    import torch
+    import paper_2606_22968_gb300 as m
+    prefix, length, hq, hkv, d = (int(x) for x in args.case.split(","))
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(7)
+    q = torch.randn((length, hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    kc = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    vc = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    out = torch.empty_like(q)
+    lse = torch.empty((hq, length), device=dev, dtype=torch.float32)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    times = []
+    for i in range(args.warmup + args.steps):
+        ev[0].record()
+        m.mocap_chunk_attn(q, kc, vc, prefix, out, lse, 1.0 / math.sqrt(d))
+        ev[1].record()
+        torch.cuda.synchronize()
+        if i >= args.warmup:
+            times.append(ev[0].elapsed_time(ev[1]))
+    if m.mocap_last_device_status() != m.MOCAP_OK:
+        raise RuntimeError("device wait expired")
+    flops = 4 * hq * d * (length * prefix + length * (length + 1) // 2)
+    ms = statistics.median(times)
+    print(json.dumps({"case": args.case, "ms": ms, "tflops": flops / ms / 1e9,
+                      "kv_bytes": 2 * (prefix + length) * hkv * d * 2}), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
+    if args.case:
+        return profile_case(args)
     rank, world, local = init_dist(args)
     try:
         if args.impl == "reference":
