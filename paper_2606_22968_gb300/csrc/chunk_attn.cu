@@ -12,9 +12,8 @@
 //   warp 1        MMA issuer (one thread): S_s = Q_s K_j^T into TMEM, then
 //                 O_s += P_s V_j with P_s read from TMEM; tcgen05.commit
 //                 signals S ready / stage free / O final.
-//   warps 2-5     softmax for head slot 0, warps 6-9 for slot 1: a warp may
-//                 touch only TMEM lanes 32*(warp%4) .. +31, and any 4
-//                 consecutive warps cover all 128.  Thread r
+//   warps 4-7     softmax for head slot 0, warps 8-11 for slot 1 (a warp may
+//                 touch only TMEM lanes 32*(warp%4) .. +31).  Thread r
 //                 owns TMEM lane r = query row r, so row max / row sum are
 //                 thread-local (no shuffles).  Online softmax in fp32, log2
 //                 domain; O is rescaled in TMEM only when the running max grows
@@ -46,7 +45,17 @@ namespace {
 constexpr int kBlockM = 128;   // query rows per tile = TMEM lanes
 constexpr int kBlockN = 128;   // keys per K/V tile
 constexpr int kStages = 4;     // ring stages, each holds one K or one V tile
-constexpr int kThreads = 320;  // 10 warps: producer, MMA, 2 x 4 softmax
+constexpr int kThreads = 384;  // 3 warpgroups: {producer, MMA, 2 idle}, softmax 0, softmax 1
+// Register split (setmaxnreg): the kernel is built for 168 registers per
+// thread (384 x 168 = 64512 <= 65536); warpgroup 0 gives up to 56 and the two
+// softmax warpgroups grow to 224: 128*56 + 256*224 = 64512.  The host refuses
+// to launch if the compiled count differs, since an unbalanced split would
+// block in setmaxnreg.inc.
+constexpr int kLaunchRegs = 168;
+constexpr uint32_t kRegsControl = 56;
+constexpr uint32_t kRegsSoftmax = 224;
+static_assert(kThreads * kLaunchRegs <= 65536, "register file");
+static_assert(128 * kRegsControl + 256 * kRegsSoftmax <= kThreads * kLaunchRegs, "split");
 constexpr int kBoxCols = 64;   // bf16 per 128-byte swizzled row
 constexpr int kBoxBytes = kBlockM * kBoxCols * 2;  // 16 KB: one TMA box
 constexpr uint32_t kTmemCols = 512;
@@ -130,15 +139,255 @@ __device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint3
   }
 }
 
-template <int D>
-__device__ __forceinline__ void tmem_ld128(uint32_t taddr, float (&x)[128]) {
+// One row of S (128 fp32 columns) into registers, with the causal mask
+// applied when the tile crosses the diagonal (column c is key j*128 + c;
+// `lim` is the last column this row may see).
+__device__ __forceinline__ void load_scores(uint32_t taddr, bool masked, int lim, float (&x)[128]) {
+  uint32_t r[128];
+  tmem_ld128(taddr, r);
 #pragma unroll
-  for (int c = 0; c < 4; ++c) {
-    uint32_t r[32];
-    tmem_ld32(taddr + c * 32, r);
+  for (int c = 0; c < 128; ++c) x[c] = __uint_as_float(r[c]);
+  if (masked) {
 #pragma unroll
-    for (int e = 0; e < 32; ++e) x[c * 32 + e] = __uint_as_float(r[e]);
+    for (int c = 0; c < 128; ++c)
+      if (c > lim) x[c] = -INFINITY;
   }
+}
+
+// Row max as 8 independent chains of 3-input max, then a short tree.
+__device__ __forceinline__ float row_max(const float (&x)[128]) {
+  float m[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) m[i] = fmax3(x[i], x[8 + i], x[16 + i]);
+#pragma unroll
+  for (int c = 24; c < 128; c += 16) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) m[i] = fmax3(m[i], x[c + i], c + 8 + i < 128 ? x[c + 8 + i] : m[i]);
+  }
+  const float a = fmax3(m[0], m[1], m[2]);
+  const float b = fmax3(m[3], m[4], m[5]);
+  return fmax3(a, b, fmaxf(m[6], m[7]));
+}
+
+// Warpgroup 0: warp 0 is the TMA producer, warp 1 the MMA issuer (one lane
+// each); warps 2-3 only take part in the barriers.
+template <int D, int MAXI>
+__device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_t base,
+                                              uint32_t bars, uint32_t tmem, uint32_t warp,
+                                              uint32_t lane, int item, int g, int h0, int r0,
+                                              int nslots, int n_kv) {
+  using L = Layout<D>;
+  auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
+  if (warp == 0) {
+    // ===================== TMA producer =====================================
+    if (lane == 0) {
+      const CUtensorMap *mq = &p.tq[item];
+      const CUtensorMap *mk = &p.tk[item];
+      const CUtensorMap *mv = &p.tv[item];
+      prefetch_tmap(mq);
+      prefetch_tmap(mk);
+      prefetch_tmap(mv);
+      mbar_arrive_expect_tx(bar(L::kBarQ), nslots * L::kTileBytes);
+      for (int s = 0; s < nslots; ++s)
+        for (int c = 0; c < D / kBoxCols; ++c)
+          tma_load_3d(base + L::kQ + s * L::kTileBytes + c * kBoxBytes, mq, bar(L::kBarQ),
+                      c * kBoxCols, h0 + s, r0);
+      const int n_seq = 2 * n_kv;  // K_0, V_0, K_1, V_1, ...
+      bool ok = true;
+      int seq = 0;
+      for (; seq < n_seq; ++seq) {
+        const int st = seq % kStages;
+        if (seq >= kStages && !mbar_wait(bar(L::kBarEmpty + st), ((seq / kStages) - 1) & 1,
+                                         p.status, kWaitLimitNs, true, kHintProducer)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(bar(L::kBarFull + st), L::kTileBytes);
+        const CUtensorMap *m = (seq & 1) ? mv : mk;
+        const int key0 = (seq >> 1) * kBlockN;
+        for (int c = 0; c < D / kBoxCols; ++c)
+          tma_load_3d(base + L::kRing + st * L::kTileBytes + c * kBoxBytes, m,
+                      bar(L::kBarFull + st), c * kBoxCols, g, key0);
+      }
+      // Copies still in flight land before the CTA may exit.
+      mbar_wait(bar(L::kBarQ), 0, p.status, kDrainLimitNs, false);
+      for (int s2 = max(0, seq - kStages); s2 < seq; ++s2)
+        mbar_wait(bar(L::kBarFull + s2 % kStages), (s2 / kStages) & 1, p.status, kDrainLimitNs,
+                  false);
+      // Normal exit: the last stage releases (tcgen05.commit arrivals) landed.
+      if (ok)
+        for (int s2 = max(0, n_seq - kStages); s2 < n_seq; ++s2)
+          if (!mbar_wait(bar(L::kBarEmpty + s2 % kStages), (s2 / kStages) & 1, p.status)) break;
+    }
+  } else if (warp == 1) {
+    // ===================== MMA issuer =======================================
+    if (lane == 0) {
+      const uint32_t q_smem = base + L::kQ;
+      auto stage_smem = [&](int seq) -> uint32_t {
+        return base + L::kRing + (seq % kStages) * L::kTileBytes;
+      };
+      bool ok = mbar_wait(bar(L::kBarQ), 0, p.status, kWaitLimitNs, true, kHintMma) &&
+                mbar_wait(bar(L::kBarFull + 0), 0, p.status, kWaitLimitNs, true, kHintMma);
+      if (ok) {
+        tc_fence_after();
+        for (int s = 0; s < nslots; ++s) {
+          issue_qk<D>(tmem + s * kBlockN, q_smem + s * L::kTileBytes, stage_smem(0));
+          tc_commit(bar(L::kBarS + s));
+        }
+        tc_commit(bar(L::kBarEmpty + 0));
+        for (int j = 0; j < n_kv && ok; ++j) {
+          const int sv = 2 * j + 1;
+          const int sk = 2 * j + 2;
+          const bool has_next = j + 1 < n_kv;
+          ok = mbar_wait(bar(L::kBarFull + sv % kStages), (sv / kStages) & 1, p.status,
+                         kWaitLimitNs, true, kHintMma);
+          if (ok && has_next)
+            ok = mbar_wait(bar(L::kBarFull + sk % kStages), (sk / kStages) & 1, p.status,
+                           kWaitLimitNs, true, kHintMma);
+          if (!ok) break;
+          tc_fence_after();
+          for (int s = 0; s < nslots; ++s) {
+            ok = mbar_wait(bar(L::kBarP + s), j & 1, p.status, kWaitLimitNs, true, kHintMma);
+            if (!ok) break;
+            tc_fence_after();
+            issue_pv<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, stage_smem(sv), j > 0);
+            if (has_next) {
+              issue_qk<D>(tmem + s * kBlockN, q_smem + s * L::kTileBytes, stage_smem(sk));
+              tc_commit(bar(L::kBarS + s));
+            } else {
+              tc_commit(bar(L::kBarO + s));
+            }
+          }
+          if (!ok) break;
+          tc_commit(bar(L::kBarEmpty + sv % kStages));
+          if (has_next) tc_commit(bar(L::kBarEmpty + sk % kStages));
+        }
+      }
+      // Every issued MMA completes before TMEM is released.
+      tc_commit(bar(L::kBarDrain));
+      mbar_wait(bar(L::kBarDrain), 0, p.status, kDrainLimitNs, false);
+    }
+  }
+}
+
+// Warpgroups 1 and 2: online softmax for head slot (warp - 4) / 4, then the
+// epilogue (O / l -> bf16, LSE).
+template <int D, int MAXI>
+__device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t bars,
+                                             uint32_t tmem, uint32_t warp, uint32_t lane,
+                                             const ItemDesc &it, int h0, int r0, int nslots,
+                                             int n_kv, int qpos0, int n_unmasked) {
+  using L = Layout<D>;
+  auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
+  const int s = static_cast<int>(warp - 4) / 4;
+  if (s < nslots) {
+    const uint32_t quarter = warp & 3u;
+    const int row = static_cast<int>(quarter * 32 + lane);
+    const uint32_t lane_addr = tmem + ((quarter * 32u) << 16);
+    const uint32_t s_addr = lane_addr + s * kBlockN;
+    const uint32_t o_addr = lane_addr + 2 * kBlockN + s * D;
+    const int qpos = qpos0 + row;
+    const float sl2 = p.scale_log2;
+    float m = -INFINITY;  // running max of scale*log2(e)*s, possibly stale by < 2^8
+    float l = 0.f;        // running sum of fp32 probabilities
+    bool ok = true;
+    for (int j = 0; j < n_kv; ++j) {
+      if (!mbar_wait_warp(bar(L::kBarS + s), j & 1, p.status, kHintSoftmax)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float x[128];
+      const bool masked = j >= n_unmasked;
+      const int lim = qpos - j * kBlockN;  // last visible column of this row
+      load_scores(s_addr, masked, lim, x);
+      const float mt = row_max(x) * sl2;
+      if (j == 0) {
+        m = mt;  // key 0 is visible to every row: finite
+      } else if (__any_sync(0xffffffffu, mt > m + kMaxGrowthLog2)) {
+        // Rare: the running max grew by more than 2^8.  Rescale O and l,
+        // then re-read S so its registers are free during the rescale.
+        const float mn = fmaxf(m, mt);
+        const float f = ex2_approx(m - mn);
+        l *= f;
+        m = mn;
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(o_addr + c * 32, r);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * f);
+          tmem_st32(o_addr + c * 32, r);
+        }
+        tmem_st_wait();
+        load_scores(s_addr, masked, lim, x);
+      }
+      // p = 2^(s * scale * log2 e - m): packed FMA for the argument, MUFU
+      // for 2^x, packed adds into four independent partial sums.
+      const uint64_t sl2x2 = f2(sl2, sl2);
+      const uint64_t negm2 = f2(-m, -m);
+      uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const int c = cc * 32 + 2 * e;
+          float a, b;
+          f2_split(ffma2(f2(x[c], x[c + 1]), sl2x2, negm2), a, b);
+          a = ex2_approx(a);
+          b = ex2_approx(b);
+          acc[e & 3] = fadd2(acc[e & 3], f2(a, b));
+          pk[e] = pack_bf16(a, b);
+        }
+        tmem_st16(s_addr + cc * 16, pk);  // P columns 16cc .. 16cc+15 alias S
+      }
+      float sum0, sum1, sum2, sum3, sum4, sum5, sum6, sum7;
+      f2_split(acc[0], sum0, sum1);
+      f2_split(acc[1], sum2, sum3);
+      f2_split(acc[2], sum4, sum5);
+      f2_split(acc[3], sum6, sum7);
+      sum0 = (sum0 + sum1) + (sum2 + sum3);
+      sum1 = (sum4 + sum5) + (sum6 + sum7);
+      l += sum0 + sum1;
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(L::kBarP + s));
+    }
+    if (ok) ok = mbar_wait_warp(bar(L::kBarO + s), 0, p.status);
+    if (ok) {
+      tc_fence_after();
+      const float inv = 1.0f / l;
+      const bool valid = r0 + row < it.len;
+      const int64_t orow = it.q_row + r0 + row;
+      __nv_bfloat16 *dst = p.out + (orow * p.n_q_heads + h0 + s) * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(o_addr + c * 32, r);
+        uint32_t pk[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e)
+          pk[e] = pack_bf16(__uint_as_float(r[2 * e]) * inv, __uint_as_float(r[2 * e + 1]) * inv);
+        if (valid) {
+          uint4 *d4 = reinterpret_cast<uint4 *>(dst + c * 32);
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            d4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        }
+      }
+      if (valid)
+        p.lse[static_cast<int64_t>(h0 + s) * p.lse_stride + orow] =
+            (m + log2f(l)) * 0.69314718055994530942f;
+    }
+  }
+}
+
+// All 384 threads, reached from each warpgroup's own code path (the
+// non-aligned barrier form allows different call sites).
+__device__ __forceinline__ void cta_barrier() {
+  asm volatile("barrier.sync 1, %0;" ::"n"(kThreads) : "memory");
 }
 
 template <int D, int MAXI>
@@ -205,208 +454,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-
-  if (warp == 0) {
-    // ===================== TMA producer =====================================
-    if (lane == 0) {
-      const CUtensorMap *mq = &p.tq[item];
-      const CUtensorMap *mk = &p.tk[item];
-      const CUtensorMap *mv = &p.tv[item];
-      prefetch_tmap(mq);
-      prefetch_tmap(mk);
-      prefetch_tmap(mv);
-      mbar_arrive_expect_tx(bar(L::kBarQ), nslots * L::kTileBytes);
-      for (int s = 0; s < nslots; ++s)
-        for (int c = 0; c < D / kBoxCols; ++c)
-          tma_load_3d(base + L::kQ + s * L::kTileBytes + c * kBoxBytes, mq, bar(L::kBarQ),
-                      c * kBoxCols, h0 + s, r0);
-      const int n_seq = 2 * n_kv;  // K_0, V_0, K_1, V_1, ...
-      bool ok = true;
-      int seq = 0;
-      for (; seq < n_seq; ++seq) {
-        const int st = seq % kStages;
-        if (seq >= kStages &&
-            !mbar_wait(bar(L::kBarEmpty + st), ((seq / kStages) - 1) & 1, p.status)) {
-          ok = false;
-          break;
-        }
-        mbar_arrive_expect_tx(bar(L::kBarFull + st), L::kTileBytes);
-        const CUtensorMap *m = (seq & 1) ? mv : mk;
-        const int key0 = (seq >> 1) * kBlockN;
-        for (int c = 0; c < D / kBoxCols; ++c)
-          tma_load_3d(base + L::kRing + st * L::kTileBytes + c * kBoxBytes, m,
-                      bar(L::kBarFull + st), c * kBoxCols, g, key0);
-      }
-      // Copies still in flight land before the CTA may exit.
-      mbar_wait(bar(L::kBarQ), 0, p.status, kDrainLimitNs, false);
-      for (int s2 = max(0, seq - kStages); s2 < seq; ++s2)
-        mbar_wait(bar(L::kBarFull + s2 % kStages), (s2 / kStages) & 1, p.status, kDrainLimitNs,
-                  false);
-      // Normal exit: the last stage releases (tcgen05.commit arrivals) landed.
-      if (ok)
-        for (int s2 = max(0, n_seq - kStages); s2 < n_seq; ++s2)
-          if (!mbar_wait(bar(L::kBarEmpty + s2 % kStages), (s2 / kStages) & 1, p.status)) break;
-    }
-  } else if (warp == 1) {
-    // ===================== MMA issuer =======================================
-    if (lane == 0) {
-      const uint32_t q_smem = base + L::kQ;
-      auto stage_smem = [&](int seq) -> uint32_t {
-        return base + L::kRing + (seq % kStages) * L::kTileBytes;
-      };
-      bool ok = mbar_wait(bar(L::kBarQ), 0, p.status) &&
-                mbar_wait(bar(L::kBarFull + 0), 0, p.status);
-      if (ok) {
-        tc_fence_after();
-        for (int s = 0; s < nslots; ++s) {
-          issue_qk<D>(tmem + s * kBlockN, q_smem + s * L::kTileBytes, stage_smem(0));
-          tc_commit(bar(L::kBarS + s));
-        }
-        tc_commit(bar(L::kBarEmpty + 0));
-        for (int j = 0; j < n_kv && ok; ++j) {
-          const int sv = 2 * j + 1;
-          const int sk = 2 * j + 2;
-          const bool has_next = j + 1 < n_kv;
-          ok = mbar_wait(bar(L::kBarFull + sv % kStages), (sv / kStages) & 1, p.status);
-          if (ok && has_next)
-            ok = mbar_wait(bar(L::kBarFull + sk % kStages), (sk / kStages) & 1, p.status);
-          if (!ok) break;
-          tc_fence_after();
-          for (int s = 0; s < nslots; ++s) {
-            ok = mbar_wait(bar(L::kBarP + s), j & 1, p.status);
-            if (!ok) break;
-            tc_fence_after();
-            issue_pv<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, stage_smem(sv), j > 0);
-            if (has_next) {
-              issue_qk<D>(tmem + s * kBlockN, q_smem + s * L::kTileBytes, stage_smem(sk));
-              tc_commit(bar(L::kBarS + s));
-            } else {
-              tc_commit(bar(L::kBarO + s));
-            }
-          }
-          if (!ok) break;
-          tc_commit(bar(L::kBarEmpty + sv % kStages));
-          if (has_next) tc_commit(bar(L::kBarEmpty + sk % kStages));
-        }
-      }
-      // Every issued MMA completes before TMEM is released.
-      tc_commit(bar(L::kBarDrain));
-      mbar_wait(bar(L::kBarDrain), 0, p.status, kDrainLimitNs, false);
+  if (warp < 4) {
+    setmaxnreg_dec<kRegsControl>();
+    control_roles<D, MAXI>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, n_kv);
+    tc_fence_before();
+    cta_barrier();
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc(tmem, kTmemCols);
     }
   } else {
-    // ===================== softmax / epilogue ===============================
-    const int s = static_cast<int>(warp - 2) / 4;
-    if (s < nslots) {
-      const uint32_t quarter = warp & 3u;
-      const int row = static_cast<int>(quarter * 32 + lane);
-      const uint32_t lane_addr = tmem + ((quarter * 32u) << 16);
-      const uint32_t s_addr = lane_addr + s * kBlockN;
-      const uint32_t o_addr = lane_addr + 2 * kBlockN + s * D;
-      const int qpos = qpos0 + row;
-      const float sl2 = p.scale_log2;
-      float m = -INFINITY;  // running max of scale*log2(e)*s, possibly stale by < 2^8
-      float l = 0.f;        // running sum of fp32 probabilities
-      bool ok = true;
-      for (int j = 0; j < n_kv; ++j) {
-        if (!mbar_wait_warp(bar(L::kBarS + s), j & 1, p.status)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        float x[128];
-        tmem_ld128<D>(s_addr, x);
-        if (j >= n_unmasked) {
-          const int lim = qpos - j * kBlockN;  // last visible column of this row
-#pragma unroll
-          for (int c = 0; c < 128; ++c)
-            if (c > lim) x[c] = -INFINITY;
-        }
-        float tmax = x[0];
-#pragma unroll
-        for (int c = 1; c < 128; ++c) tmax = fmaxf(tmax, x[c]);
-        const float mt = tmax * sl2;
-        if (j == 0) {
-          m = mt;  // key 0 is visible to every row: finite
-        } else if (__any_sync(0xffffffffu, mt > m + kMaxGrowthLog2)) {
-          // Rare: the running max grew by more than 2^8.  Rescale O and l,
-          // then re-read S so its registers are free during the rescale.
-          const float mn = fmaxf(m, mt);
-          const float f = ex2_approx(m - mn);
-          l *= f;
-          m = mn;
-#pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t r[32];
-            tmem_ld32(o_addr + c * 32, r);
-#pragma unroll
-            for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * f);
-            tmem_st32(o_addr + c * 32, r);
-          }
-          tmem_st_wait();
-          tmem_ld128<D>(s_addr, x);
-          if (j >= n_unmasked) {
-            const int lim = qpos - j * kBlockN;
-#pragma unroll
-            for (int c = 0; c < 128; ++c)
-              if (c > lim) x[c] = -INFINITY;
-          }
-        }
-        const float neg_m = -m;
-        float sum0 = 0.f, sum1 = 0.f;
-#pragma unroll
-        for (int cc = 0; cc < 4; ++cc) {
-          uint32_t pk[16];
-#pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            const float a = ex2_approx(fmaf(x[cc * 32 + 2 * e], sl2, neg_m));
-            const float b = ex2_approx(fmaf(x[cc * 32 + 2 * e + 1], sl2, neg_m));
-            sum0 += a;
-            sum1 += b;
-            pk[e] = pack_bf16(a, b);
-          }
-          tmem_st16(s_addr + cc * 16, pk);  // P columns 16cc .. 16cc+15 alias S
-        }
-        l += sum0 + sum1;
-        tmem_st_wait();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(L::kBarP + s));
-      }
-      if (ok) ok = mbar_wait_warp(bar(L::kBarO + s), 0, p.status);
-      if (ok) {
-        tc_fence_after();
-        const float inv = 1.0f / l;
-        const bool valid = r0 + row < it.len;
-        const int64_t orow = it.q_row + r0 + row;
-        __nv_bfloat16 *dst = p.out + (orow * p.n_q_heads + h0 + s) * D;
-#pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(o_addr + c * 32, r);
-          uint32_t pk[16];
-#pragma unroll
-          for (int e = 0; e < 16; ++e)
-            pk[e] = pack_bf16(__uint_as_float(r[2 * e]) * inv, __uint_as_float(r[2 * e + 1]) * inv);
-          if (valid) {
-            uint4 *d4 = reinterpret_cast<uint4 *>(dst + c * 32);
-#pragma unroll
-            for (int v = 0; v < 4; ++v)
-              d4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
-          }
-        }
-        if (valid)
-          p.lse[static_cast<int64_t>(h0 + s) * p.lse_stride + orow] =
-              (m + log2f(l)) * 0.69314718055994530942f;
-      }
-    }
-  }
-
-  // ---- teardown -------------------------------------------------------------
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    setmaxnreg_inc<kRegsSoftmax>();
+    softmax_role<D, MAXI>(p, bar(0), tmem, warp, lane, it, h0, r0, nslots, n_kv, qpos0,
+                          n_unmasked);
+    tc_fence_before();
+    cta_barrier();
   }
 }
 
@@ -508,6 +570,9 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
   if (!attr_done[dev]) {
+    cudaFuncAttributes fa{};
+    if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) return MOCAP_ECUDA;
+    if (fa.numRegs != kLaunchRegs) return MOCAP_EUNSUPPORTED;  // split would not balance
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes) !=
         cudaSuccess)
       return MOCAP_ECUDA;
