@@ -114,27 +114,29 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 }
 
 // S = Q K^T for one head slot: M=128, N=128, K=D; both operands K-major.
+// q_desc / k_desc describe the tiles' first 16-column step; step kk starts
+// (kk / 4) boxes and (kk % 4) * 32 bytes further (descriptor units of 16 B).
 template <int D>
-__device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint32_t q_smem, uint32_t k_smem) {
+__device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint64_t q_desc, uint64_t k_desc) {
   constexpr uint32_t idesc = idesc_bf16_f32(kBlockM, kBlockN, false, false);
 #pragma unroll
   for (int kk = 0; kk < D / 16; ++kk) {
-    const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;  // 16 bf16 = 32 bytes
-    mma_ss(s_tmem, sdesc_sw128(q_smem + off, 16, 1024), sdesc_sw128(k_smem + off, 16, 1024),
-           idesc, kk > 0 ? 1u : 0u);
+    const uint64_t off = static_cast<uint64_t>(((kk / 4) * kBoxBytes + (kk % 4) * 32) >> 4);
+    mma_ss(s_tmem, q_desc + off, k_desc + off, idesc, kk > 0 ? 1u : 0u);
   }
 }
 
 // O += P V for one head slot: M=128, N=D, K=128 keys.  P (A operand) lives in
 // TMEM, 2 bf16 per column; V (B operand) is MN-major: d is contiguous, two
-// 64-wide d halves 16 KB apart (LBO), 8-key groups 1024 bytes apart (SBO).
+// 64-wide d halves 16 KB apart (leading byte offset), 8-key groups 1024
+// bytes apart (stride byte offset); step kk starts 16 keys = 2048 B further.
 template <int D>
-__device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint32_t v_smem,
+__device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint64_t v_desc,
                                          bool accumulate) {
   constexpr uint32_t idesc = idesc_bf16_f32(kBlockM, D, false, true);
 #pragma unroll
   for (int kk = 0; kk < kBlockN / 16; ++kk) {
-    mma_ts(o_tmem, p_tmem + kk * 8, sdesc_sw128(v_smem + kk * 16 * 128, kBoxBytes, 1024), idesc,
+    mma_ts(o_tmem, p_tmem + kk * 8, v_desc + static_cast<uint64_t>((kk * 2048) >> 4), idesc,
            (accumulate || kk > 0) ? 1u : 0u);
   }
 }
@@ -221,52 +223,69 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
     }
   } else if (warp == 1) {
     // ===================== MMA issuer =======================================
-    if (lane == 0) {
-      const uint32_t q_smem = base + L::kQ;
-      auto stage_smem = [&](int seq) -> uint32_t {
-        return base + L::kRing + (seq % kStages) * L::kTileBytes;
-      };
-      bool ok = mbar_wait(bar(L::kBarQ), 0, p.status, kWaitLimitNs, true, kHintMma) &&
-                mbar_wait(bar(L::kBarFull + 0), 0, p.status, kWaitLimitNs, true, kHintMma);
-      if (ok) {
-        tc_fence_after();
+    // The whole warp runs the loop (descriptors stay warp-uniform); one
+    // elected lane issues the MMAs and their commits.
+    const bool leader = elect_one();
+    auto wait = [&](int b, int parity) {
+      return mbar_wait_warp(bar(b), parity & 1, p.status, kHintMma);
+    };
+    // Descriptors of Q slot 0 and ring stage 0; other tiles are whole
+    // multiples of kTileBytes further (descriptor start field in 16 B units).
+    const uint64_t q_desc0 = sdesc_sw128(base + L::kQ, 16, 1024);
+    const uint64_t k_desc0 = sdesc_sw128(base + L::kRing, 16, 1024);
+    const uint64_t v_desc0 = sdesc_sw128(base + L::kRing, kBoxBytes, 1024);
+    constexpr uint64_t kTileStep = static_cast<uint64_t>(L::kTileBytes >> 4);
+    auto q_desc = [&](int s) { return q_desc0 + static_cast<uint64_t>(s) * kTileStep; };
+    auto k_desc = [&](int st) { return k_desc0 + static_cast<uint64_t>(st) * kTileStep; };
+    auto v_desc = [&](int st) { return v_desc0 + static_cast<uint64_t>(st) * kTileStep; };
+    bool ok = wait(L::kBarQ, 0) && wait(L::kBarFull + 0, 0);
+    if (ok) {
+      tc_fence_after();
+      if (leader) {
         for (int s = 0; s < nslots; ++s) {
-          issue_qk<D>(tmem + s * kBlockN, q_smem + s * L::kTileBytes, stage_smem(0));
+          issue_qk<D>(tmem + s * kBlockN, q_desc(s), k_desc(0));
           tc_commit(bar(L::kBarS + s));
         }
         tc_commit(bar(L::kBarEmpty + 0));
-        for (int j = 0; j < n_kv && ok; ++j) {
-          const int sv = 2 * j + 1;
-          const int sk = 2 * j + 2;
-          const bool has_next = j + 1 < n_kv;
-          ok = mbar_wait(bar(L::kBarFull + sv % kStages), (sv / kStages) & 1, p.status,
-                         kWaitLimitNs, true, kHintMma);
-          if (ok && has_next)
-            ok = mbar_wait(bar(L::kBarFull + sk % kStages), (sk / kStages) & 1, p.status,
-                           kWaitLimitNs, true, kHintMma);
+      }
+      __syncwarp();
+      for (int j = 0; j < n_kv && ok; ++j) {
+        const int sv = 2 * j + 1;
+        const int sk = 2 * j + 2;
+        const bool has_next = j + 1 < n_kv;
+        ok = wait(L::kBarFull + sv % kStages, sv / kStages);
+        if (ok && has_next) ok = wait(L::kBarFull + sk % kStages, sk / kStages);
+        if (!ok) break;
+        for (int s = 0; s < nslots; ++s) {
+          ok = wait(L::kBarP + s, j);
           if (!ok) break;
           tc_fence_after();
-          for (int s = 0; s < nslots; ++s) {
-            ok = mbar_wait(bar(L::kBarP + s), j & 1, p.status, kWaitLimitNs, true, kHintMma);
-            if (!ok) break;
-            tc_fence_after();
-            issue_pv<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, stage_smem(sv), j > 0);
+          if (leader) {
+            issue_pv<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
+                        j > 0);
             if (has_next) {
-              issue_qk<D>(tmem + s * kBlockN, q_smem + s * L::kTileBytes, stage_smem(sk));
+              issue_qk<D>(tmem + s * kBlockN, q_desc(s), k_desc(sk % kStages));
               tc_commit(bar(L::kBarS + s));
             } else {
               tc_commit(bar(L::kBarO + s));
             }
           }
-          if (!ok) break;
+          __syncwarp();
+        }
+        if (!ok) break;
+        if (leader) {
           tc_commit(bar(L::kBarEmpty + sv % kStages));
           if (has_next) tc_commit(bar(L::kBarEmpty + sk % kStages));
         }
+        __syncwarp();
       }
-      // Every issued MMA completes before TMEM is released.
+    }
+    // Every issued MMA completes before TMEM is released.
+    if (leader) {
       tc_commit(bar(L::kBarDrain));
       mbar_wait(bar(L::kBarDrain), 0, p.status, kDrainLimitNs, false);
     }
+    __syncwarp();
   }
 }
 

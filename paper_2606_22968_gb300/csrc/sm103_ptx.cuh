@@ -21,7 +21,7 @@ constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per wait
 #define MOCAP_HINT_PRODUCER 100000u
 #endif
 #ifndef MOCAP_HINT_MMA
-#define MOCAP_HINT_MMA 100000u
+#define MOCAP_HINT_MMA 0u
 #endif
 #ifndef MOCAP_HINT_SOFTMAX
 #define MOCAP_HINT_SOFTMAX 100000u
@@ -110,6 +110,17 @@ __device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity, ui
                                                uint32_t hint_ns = 0) {
   const bool ok = mbar_wait(bar, parity, status, kWaitLimitNs, true, hint_ns);
   return __all_sync(0xffffffffu, ok);
+}
+
+// One lane of the (converged) warp returns true.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "elect.sync _|p, 0xffffffff;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(pred));
+  return pred != 0;
 }
 
 // Register budget per thread of the calling warpgroup (all 4 warps execute it).
@@ -321,6 +332,20 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float d;
   asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
   return d;
+}
+
+// 16-byte shared-memory store (generic proxy).
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                             uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+               "r"(d)
+               : "memory");
+}
+
+// Make this thread's generic-proxy shared-memory writes visible to the async
+// proxy (tensor core / TMA reads) once the following synchronisation is seen.
+__device__ __forceinline__ void fence_proxy_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // 2^x on the special-function unit (PTX ex2.approx.ftz.f32); ex2(-inf) = +0.
