@@ -18,7 +18,9 @@
 //                 thread-local (no shuffles).  Online softmax in fp32, log2
 //                 domain; O is rescaled in TMEM only when the running max grows
 //                 by more than 2^8 (exact: the final 1/l uses the same max).
-//                 P is written back to TMEM as packed bf16 (aliasing S).
+//                 P is written back to TMEM as packed bf16 (aliasing S), in
+//                 two halves of 64 keys, each signalled on its own barrier
+//                 so the first half of P V overlaps the second half's exps.
 //   TMEM (512 columns): S0 [0,128) S1 [128,256) O0 [256,256+D) O1 [256+D, ..).
 // The two slots share every K/V tile (two heads of one GQA group), so the
 // tensor core alternates between them while the other slot's softmax runs.
@@ -99,10 +101,11 @@ struct Layout {
   static constexpr int kBarFull = 1;               // kStages
   static constexpr int kBarEmpty = 1 + kStages;    // kStages
   static constexpr int kBarS = 1 + 2 * kStages;    // 2
-  static constexpr int kBarP = 3 + 2 * kStages;    // 2
+  static constexpr int kBarP = 3 + 2 * kStages;    // 2: keys 0..63 of P written
   static constexpr int kBarO = 5 + 2 * kStages;    // 2
   static constexpr int kBarDrain = 7 + 2 * kStages;
-  static constexpr int kNumBars = 8 + 2 * kStages;
+  static constexpr int kBarPHi = 8 + 2 * kStages;  // 2: keys 64..127 of P written
+  static constexpr int kNumBars = 10 + 2 * kStages;
   static constexpr int kTmemSlot = kBars + 8 * kNumBars;
   static constexpr int kFlag = kTmemSlot + 4;
   static constexpr int kBytes = kFlag + 4 + 1024;  // + slack for 1024-byte alignment
@@ -126,18 +129,20 @@ __device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint64_t q_desc, uint6
   }
 }
 
-// O += P V for one head slot: M=128, N=D, K=128 keys.  P (A operand) lives in
-// TMEM, 2 bf16 per column; V (B operand) is MN-major: d is contiguous, two
-// 64-wide d halves 16 KB apart (leading byte offset), 8-key groups 1024
-// bytes apart (stride byte offset); step kk starts 16 keys = 2048 B further.
+// Half h of O += P V for one head slot: M=128, N=D, keys 64h .. 64h+63 (four
+// K=16 steps).  P (A operand) lives in TMEM, 2 bf16 per column; V (B operand)
+// is MN-major: d is contiguous, two 64-wide d halves 16 KB apart (leading byte
+// offset), 8-key groups 1024 bytes apart (stride byte offset); step kk starts
+// 16 keys = 2048 B further.
 template <int D>
-__device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint64_t v_desc,
-                                         bool accumulate) {
+__device__ __forceinline__ void issue_pv_half(uint32_t o_tmem, uint32_t p_tmem, uint64_t v_desc,
+                                              bool accumulate, int h) {
   constexpr uint32_t idesc = idesc_bf16_f32(kBlockM, D, false, true);
 #pragma unroll
-  for (int kk = 0; kk < kBlockN / 16; ++kk) {
+  for (int k = 0; k < 4; ++k) {
+    const int kk = 4 * h + k;
     mma_ts(o_tmem, p_tmem + kk * 8, v_desc + static_cast<uint64_t>((kk * 2048) >> 4), idesc,
-           (accumulate || kk > 0) ? 1u : 0u);
+           (accumulate || k > 0) ? 1u : 0u);
   }
 }
 
@@ -257,12 +262,21 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
         if (ok && has_next) ok = wait(L::kBarFull + sk % kStages, sk / kStages);
         if (!ok) break;
         for (int s = 0; s < nslots; ++s) {
+          // P arrives in two halves (keys 0..63 on kBarP, 64..127 on kBarPHi),
+          // each barrier completing once per tile.
           ok = wait(L::kBarP + s, j);
           if (!ok) break;
           tc_fence_after();
+          if (leader)
+            issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
+                             j > 0, 0);
+          __syncwarp();
+          ok = wait(L::kBarPHi + s, j);
+          if (!ok) break;
+          tc_fence_after();
           if (leader) {
-            issue_pv<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
-                        j > 0);
+            issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
+                             true, 1);
             if (has_next) {
               issue_qk<D>(tmem + s * kBlockN, q_desc(s), k_desc(sk % kStages));
               tc_commit(bar(L::kBarS + s));
@@ -360,6 +374,12 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
           pk[e] = pack_bf16(a, b);
         }
         tmem_st16(s_addr + cc * 16, pk);  // P columns 16cc .. 16cc+15 alias S
+        if (cc == 1) {  // keys 0..63 of P are in TMEM: the first half of P V may start
+          tmem_st_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(L::kBarP + s));
+        }
       }
       float sum0, sum1, sum2, sum3, sum4, sum5, sum6, sum7;
       f2_split(acc[0], sum0, sum1);
@@ -372,7 +392,7 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(bar(L::kBarP + s));
+      if (lane == 0) mbar_arrive(bar(L::kBarPHi + s));
     }
     if (ok) ok = mbar_wait_warp(bar(L::kBarO + s), 0, p.status);
     if (ok) {
@@ -467,6 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(L::kBarO + s), 1);
     }
     mbar_init(bar(L::kBarDrain), 1);
+    for (int s = 0; s < 2; ++s) mbar_init(bar(L::kBarPHi + s), 4);
     fence_mbar_init();
   }
   tc_fence_before();

@@ -58,13 +58,24 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
                : "memory");
 }
 
-// Test for completion of the phase with the given parity.  A thread whose
-// phase is still open may be suspended by the hardware: for a system-defined
-// time (hint_ns == 0) or up to hint_ns nanoseconds.
+// Test for completion of the phase with the given parity.  hint_ns selects
+// the form: kSpin = non-blocking test_wait (the caller spins); 0 = try_wait,
+// which may suspend the thread for a system-defined time; otherwise try_wait
+// with that suspend limit in ns.  Suspended threads resume when the phase
+// completes.
+constexpr uint32_t kSpin = 1u;
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity,
                                               uint32_t hint_ns = 0) {
   uint32_t ok;
-  if (hint_ns == 0) {
+  if (hint_ns == kSpin) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+  } else if (hint_ns == 0) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
