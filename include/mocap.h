@@ -29,7 +29,7 @@
  *     call returns without synchronising.  No hidden host<->device traffic.
  *   - Arguments are validated before any launch; on MOCAP_EINVAL or
  *     MOCAP_EUNSUPPORTED nothing was enqueued.  MOCAP_ECUDA reports a failed
- *     launch (the CUDA error is left for cudaGetLastError()).
+ *     CUDA call or launch (the launch error is consumed).
  */
 #ifndef MOCAP_H_
 #define MOCAP_H_
@@ -119,9 +119,12 @@ mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk,
  *   v_cache   are never read (their contents may be anything, NaN included)
  *   out       bf16 [len, n_q_heads, head_dim]
  *   lse       fp32 [n_q_heads, len]
- *   workspace, workspace_bytes: caller-owned device scratch of at least
- *             mocap_chunk_attn_workspace_size(...) bytes (may be NULL when
- *             that size is 0).
+ *   workspace, workspace_bytes: optional caller-owned device scratch
+ *             (16-byte aligned).  With at least
+ *             mocap_chunk_attn_workspace_size(...) bytes the key range may
+ *             be split (same results up to fp32 rounding order); with less,
+ *             or NULL, the single-pass kernel runs.  Contents on entry are
+ *             ignored; it must not be used by overlapping work.
  *
  * Requirements: head_dim in {64, 128} (else MOCAP_EUNSUPPORTED); n_q_heads a
  * multiple of n_kv_heads; scale > 0 and finite; prefix >= 0; len >= 0
@@ -136,10 +139,26 @@ mocap_status mocap_chunk_attn(const void *q, const void *k_cache, const void *v_
                               void *workspace, size_t workspace_bytes,
                               mocap_stream_t stream);
 
-/* Bytes of device scratch mocap_chunk_attn needs for this shape (0 today:
- * the single-pass kernel keeps all intermediates on chip). */
-size_t mocap_chunk_attn_workspace_size(int64_t prefix, int64_t len,
-                                       int32_t n_q_heads, int32_t head_dim);
+/*
+ * mocap_chunk_attn_workspace_size -- bytes of caller-owned device scratch that
+ * let mocap_chunk_attn split the chunk's key range (split-KV) for this shape.
+ *
+ * Late chunks of a long prompt have few 128-row query blocks but long
+ * prefixes, so their CTAs are few and long and the last wave leaves SMs idle
+ * (wave quantisation).  With enough workspace the kernel splits each query
+ * block's key tiles into 2..4 contiguous ranges, writes per-range fp32
+ * partials (O / l and the range's LSE) to the workspace, and a second kernel
+ * merges them: O = sum_k exp(LSE_k - LSE) O_k, LSE = ln sum_k exp(LSE_k).
+ * The split count is chosen on the host by a list-scheduling estimate over
+ * the device's SM count; 0 means no split helps (or invalid arguments).
+ * Environment: MOCAP_SPLIT_KV=0 disables splitting, MOCAP_SPLIT_KV=1..4
+ * forces that split count (capped so the first 128-row block keeps at least
+ * one key tile per split); it is read on every call.
+ * Layout: o_part [splits, len, Hq, d] fp32, then (256-byte aligned)
+ * lse_part [splits, Hq, len] fp32.
+ */
+size_t mocap_chunk_attn_workspace_size(int64_t prefix, int64_t len, int32_t n_q_heads,
+                                       int32_t n_kv_heads, int32_t head_dim);
 
 /*
  * One (request, chunk) item of a varlen launch.  All offsets are in rows.

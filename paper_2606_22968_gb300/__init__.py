@@ -69,8 +69,11 @@ def mocap_kv_append(k_chunk, v_chunk, k_cache, v_cache, offset: int, stream=None
                                        _stream(stream)), "mocap_kv_append")
 
 
-def mocap_chunk_attn_workspace_size(prefix: int, length: int, n_q_heads: int, head_dim: int) -> int:
-    return int(_lib.load().mocap_chunk_attn_workspace_size(prefix, length, n_q_heads, head_dim))
+def mocap_chunk_attn_workspace_size(prefix: int, length: int, n_q_heads: int, n_kv_heads: int,
+                                    head_dim: int) -> int:
+    """Bytes of scratch that let mocap_chunk_attn split the key range (0 = no split)."""
+    return int(_lib.load().mocap_chunk_attn_workspace_size(prefix, length, n_q_heads, n_kv_heads,
+                                                           head_dim))
 
 
 def mocap_chunk_attn(q, k_cache, v_cache, prefix: int, out, lse, scale: float,
@@ -82,6 +85,8 @@ def mocap_chunk_attn(q, k_cache, v_cache, prefix: int, out, lse, scale: float,
     length, n_q, d = q.shape
     n_kv = k_cache.shape[1]
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    if workspace is not None and not workspace.is_contiguous():
+        raise ValueError("workspace must be contiguous")
     _check(_lib.load().mocap_chunk_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), prefix, length,
                                         n_q, n_kv, d, scale, _ptr(out), _ptr(lse),
                                         _ptr(workspace), ws_bytes, _stream(stream)),

@@ -34,6 +34,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -88,6 +89,13 @@ struct AttnParams {
   int32_t heads_per_group;
   int32_t pairs_per_group;
   float scale_log2;  // scale * log2(e)
+  // Split-KV: when splits > 1 (single item only), CTA (unit, k) covers key
+  // tiles [k n / splits, (k+1) n / splits) of its unit and writes fp32
+  // partials instead of the final output: o_part [splits, len, Hq, D]
+  // (normalised by its own row sum) and lse_part [splits, Hq, len].
+  float *o_part;
+  float *lse_part;
+  int32_t splits;
 };
 
 template <int D>
@@ -182,7 +190,7 @@ template <int D, int MAXI>
 __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_t base,
                                               uint32_t bars, uint32_t tmem, uint32_t warp,
                                               uint32_t lane, int item, int g, int h0, int r0,
-                                              int nslots, int n_kv) {
+                                              int nslots, int t0, int n_kv) {
   using L = Layout<D>;
   auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
   if (warp == 0) {
@@ -211,7 +219,7 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
         }
         mbar_arrive_expect_tx(bar(L::kBarFull + st), L::kTileBytes);
         const CUtensorMap *m = (seq & 1) ? mv : mk;
-        const int key0 = (seq >> 1) * kBlockN;
+        const int key0 = (t0 + (seq >> 1)) * kBlockN;
         for (int c = 0; c < D / kBoxCols; ++c)
           tma_load_3d(base + L::kRing + st * L::kTileBytes + c * kBoxBytes, m,
                       bar(L::kBarFull + st), c * kBoxCols, g, key0);
@@ -309,7 +317,8 @@ template <int D, int MAXI>
 __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t bars,
                                              uint32_t tmem, uint32_t warp, uint32_t lane,
                                              const ItemDesc &it, int h0, int r0, int nslots,
-                                             int n_kv, int qpos0, int n_unmasked) {
+                                             int split, int t0, int n_kv, int qpos0,
+                                             int n_unmasked) {
   using L = Layout<D>;
   auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
   const int s = static_cast<int>(warp - 4) / 4;
@@ -331,12 +340,13 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
       }
       tc_fence_after();
       float x[128];
-      const bool masked = j >= n_unmasked;
-      const int lim = qpos - j * kBlockN;  // last visible column of this row
+      const int kt = t0 + j;  // key tile index
+      const bool masked = kt >= n_unmasked;
+      const int lim = qpos - kt * kBlockN;  // last visible column of this row
       load_scores(s_addr, masked, lim, x);
       const float mt = row_max(x) * sl2;
       if (j == 0) {
-        m = mt;  // key 0 is visible to every row: finite
+        m = mt;  // -inf only if this row sees no key of a split's first tile
       } else if (__any_sync(0xffffffffu, mt > m + kMaxGrowthLog2)) {
         // Rare: the running max grew by more than 2^8.  Rescale O and l,
         // then re-read S so its registers are free during the rescale.
@@ -358,7 +368,8 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
       // p = 2^(s * scale * log2 e - m): packed FMA for the argument, MUFU
       // for 2^x, packed adds into four independent partial sums.
       const uint64_t sl2x2 = f2(sl2, sl2);
-      const uint64_t negm2 = f2(-m, -m);
+      const float neg_m = m > -INFINITY ? -m : 0.0f;  // rows with no key yet: p = 0
+      const uint64_t negm2 = f2(neg_m, neg_m);
       uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
       for (int cc = 0; cc < 4; ++cc) {
@@ -395,7 +406,32 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
       if (lane == 0) mbar_arrive(bar(L::kBarPHi + s));
     }
     if (ok) ok = mbar_wait_warp(bar(L::kBarO + s), 0, p.status);
-    if (ok) {
+    if (ok && p.splits > 1) {
+      // Split-KV partial: O / l in fp32 and this range's natural-log LSE;
+      // a row that saw no key in the range gets weight 0 (LSE = -inf).
+      tc_fence_after();
+      const bool valid = r0 + row < it.len;
+      const bool any = l > 0.0f;
+      const float inv = any ? 1.0f / l : 0.0f;
+      const int64_t prow = static_cast<int64_t>(split) * it.len + r0 + row;
+      float *dst = p.o_part + (prow * p.n_q_heads + h0 + s) * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(o_addr + c * 32, r);
+        if (valid) {
+          float4 *d4 = reinterpret_cast<float4 *>(dst + c * 32);
+#pragma unroll
+          for (int v = 0; v < 8; ++v)
+            d4[v] = make_float4(__uint_as_float(r[4 * v]) * inv, __uint_as_float(r[4 * v + 1]) * inv,
+                                __uint_as_float(r[4 * v + 2]) * inv,
+                                __uint_as_float(r[4 * v + 3]) * inv);
+        }
+      }
+      if (valid)
+        p.lse_part[(static_cast<int64_t>(split) * p.n_q_heads + h0 + s) * it.len + r0 + row] =
+            any ? (m + log2f(l)) * 0.69314718055994530942f : -INFINITY;
+    } else if (ok) {
       tc_fence_after();
       const float inv = 1.0f / l;
       const bool valid = r0 + row < it.len;
@@ -460,6 +496,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   w /= p.pairs_per_group;
   const int g = w % p.n_kv_heads;
   w /= p.n_kv_heads;
+  const int split = w % p.splits;
+  w /= p.splits;
   const int qblock = it.q_blocks - 1 - w;  // heaviest (latest) row blocks first
   const int r0 = qblock * kBlockM;
   const int h0 = g * p.heads_per_group + 2 * pair;
@@ -467,8 +505,29 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int qpos0 = it.prefix + r0;
   const int kv_len = it.prefix + it.len;
   const int kv_end = min(qpos0 + kBlockM, kv_len);
-  const int n_kv = (kv_end + kBlockN - 1) / kBlockN;
+  const int n_tiles = (kv_end + kBlockN - 1) / kBlockN;
   const int n_unmasked = (qpos0 + 1) / kBlockN;  // tiles wholly at or below the diagonal
+  // this CTA's key tiles: [t0, t0 + n_kv), split `split` of `splits`
+  const int t0 = static_cast<int>(static_cast<int64_t>(split) * n_tiles / p.splits);
+  const int n_kv =
+      static_cast<int>(static_cast<int64_t>(split + 1) * n_tiles / p.splits) - t0;
+
+  if (n_kv <= 0) {
+    // No key tile in this split (the host never schedules one): an empty
+    // partial, weight 0 in the combine.
+    if (p.splits > 1 && warp >= 4) {
+      const int sl = static_cast<int>(warp - 4) / 4;
+      const int row = static_cast<int>((warp & 3u) * 32 + lane);
+      if (sl < nslots && r0 + row < it.len) {
+        const int64_t prow = static_cast<int64_t>(split) * it.len + r0 + row;
+        float *dst = p.o_part + (prow * p.n_q_heads + h0 + sl) * D;
+        for (int c = 0; c < D; ++c) dst[c] = 0.0f;
+        p.lse_part[(static_cast<int64_t>(split) * p.n_q_heads + h0 + sl) * it.len + r0 + row] =
+            -INFINITY;
+      }
+    }
+    return;
+  }
 
   // ---- setup --------------------------------------------------------------
   if (warp == 1) {
@@ -496,7 +555,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   if (warp < 4) {
     setmaxnreg_dec<kRegsControl>();
-    control_roles<D, MAXI>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, n_kv);
+    control_roles<D, MAXI>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, t0,
+                           n_kv);
     tc_fence_before();
     cta_barrier();
     if (warp == 1) {
@@ -505,11 +565,63 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     setmaxnreg_inc<kRegsSoftmax>();
-    softmax_role<D, MAXI>(p, bar(0), tmem, warp, lane, it, h0, r0, nslots, n_kv, qpos0,
+    softmax_role<D, MAXI>(p, bar(0), tmem, warp, lane, it, h0, r0, nslots, split, t0, n_kv, qpos0,
                           n_unmasked);
     tc_fence_before();
     cta_barrier();
   }
+}
+
+// Split-KV combine: the softmax over the union of disjoint key ranges weighs
+// each range's normalised output by exp(LSE_k - LSE), LSE = ln sum_k exp(LSE_k).
+// One warp per (row, head); each lane owns D/32 consecutive columns.
+template <int D>
+__global__ void __launch_bounds__(256) attn_combine_kernel(
+    const float *__restrict__ o_part, const float *__restrict__ lse_part, int splits,
+    int64_t len, int n_q_heads, __nv_bfloat16 *__restrict__ out, float *__restrict__ lse,
+    int64_t lse_stride) {
+  constexpr int kPer = D / 32;
+  const int64_t idx = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (idx >= len * n_q_heads) return;
+  const int lane = threadIdx.x & 31;
+  const int64_t row = idx / n_q_heads;
+  const int h = static_cast<int>(idx % n_q_heads);
+  float lk[8];
+  float mx = -INFINITY;
+  for (int k = 0; k < splits; ++k) {
+    lk[k] = lse_part[(static_cast<int64_t>(k) * n_q_heads + h) * len + row];
+    mx = fmaxf(mx, lk[k]);
+  }
+  float wsum = 0.0f;
+  for (int k = 0; k < splits; ++k) {
+    lk[k] = lk[k] > -INFINITY ? expf(lk[k] - mx) : 0.0f;
+    wsum += lk[k];
+  }
+  const float inv = 1.0f / wsum;
+  float acc[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) acc[e] = 0.0f;
+  for (int k = 0; k < splits; ++k) {
+    const float wk = lk[k] * inv;
+    const float *src = o_part + ((static_cast<int64_t>(k) * len + row) * n_q_heads + h) * D + lane * kPer;
+    if (kPer == 4) {
+      const float4 v = *reinterpret_cast<const float4 *>(src);
+      acc[0] += wk * v.x;
+      acc[1] += wk * v.y;
+      acc[2] += wk * v.z;
+      acc[3] += wk * v.w;
+    } else {
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) acc[e] += wk * src[e];
+    }
+  }
+  __nv_bfloat16 *dst = out + (row * n_q_heads + h) * D + lane * kPer;
+#pragma unroll
+  for (int e = 0; e < kPer; e += 2) {
+    __nv_bfloat162 v2 = __floats2bfloat162_rn(acc[e], acc[e + 1]);
+    *reinterpret_cast<__nv_bfloat162 *>(dst + e) = v2;
+  }
+  if (lane == 0) lse[static_cast<int64_t>(h) * lse_stride + row] = mx + logf(wsum);
 }
 
 // ------------------------------------------------------------------ host --
@@ -558,10 +670,82 @@ struct HostItem {
   int64_t q_row, kv_row, prefix, len;
 };
 
+// Split-KV scratch (single item): o_part [splits, len, Hq, D] fp32 followed by
+// lse_part [splits, Hq, len] fp32, the latter 256-byte aligned.
+struct SplitPlan {
+  int splits = 1;
+  size_t o_bytes = 0, lse_off = 0, bytes = 0;
+};
+
+SplitPlan split_layout(int splits, int64_t len, int n_q_heads, int head_dim) {
+  SplitPlan sp;
+  sp.splits = splits;
+  if (splits <= 1) return sp;
+  sp.o_bytes = static_cast<size_t>(splits) * len * n_q_heads * head_dim * sizeof(float);
+  sp.lse_off = (sp.o_bytes + 255) / 256 * 256;
+  sp.bytes = sp.lse_off + static_cast<size_t>(splits) * n_q_heads * len * sizeof(float);
+  return sp;
+}
+
+int sm_count_cached() {
+  static int cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+// Split count for one chunk: list-schedule the CTAs (heaviest first, one per
+// SM at a time) for 1..4 key-range splits and keep the fastest estimate.
+// Cost units: one 128-key tile of a head pair ~ 1.4 us; a CTA's fixed cost
+// ~ 4 us; the combine reads splits x (4D + 4) and writes 2D + 4 bytes per
+// (row, head) at ~5 TB/s, plus ~3 us for its launch.
+int choose_splits(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads, int head_dim,
+                  int sms) {
+  const int group = n_q_heads / n_kv_heads;
+  const int64_t pairs = (group + 1) / 2;
+  const int64_t q_blocks = (len + kBlockM - 1) / kBlockM;
+  const int64_t units = q_blocks * n_kv_heads * pairs;
+  if (units <= 0 || units >= 8LL * sms) return 1;  // many waves: little to gain
+  const int64_t min_tiles = (std::min<int64_t>(prefix + kBlockM, prefix + len) + kBlockN - 1) / kBlockN;
+  const double tile_us = 1.4 * (head_dim / 128.0), cta_us = 4.0;
+  double best_t = 0.0;
+  int best = 1;
+  std::vector<double> sm(static_cast<size_t>(sms));
+  for (int sp = 1; sp <= 4 && sp <= min_tiles; ++sp) {
+    std::fill(sm.begin(), sm.end(), 0.0);
+    for (int64_t qb = q_blocks - 1; qb >= 0; --qb) {
+      const int64_t kv_end = std::min<int64_t>(prefix + qb * kBlockM + kBlockM, prefix + len);
+      const int64_t tiles = (kv_end + kBlockN - 1) / kBlockN;
+      for (int64_t u = 0; u < n_kv_heads * pairs; ++u)
+        for (int k = 0; k < sp; ++k) {
+          const int64_t nk = (k + 1) * tiles / sp - k * tiles / sp;
+          auto it = std::min_element(sm.begin(), sm.end());
+          *it += cta_us + tile_us * static_cast<double>(nk);
+        }
+    }
+    double t = *std::max_element(sm.begin(), sm.end());
+    if (sp > 1)
+      t += 3.0 + static_cast<double>(len) * n_q_heads *
+                     (sp * (4.0 * head_dim + 4.0) + 2.0 * head_dim + 4.0) / 5e6;
+    if (sp == 1 || t < best_t) {
+      best_t = t;
+      best = sp;
+    }
+  }
+  return best;
+}
+
 template <int D, int MAXI>
 mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
                     const std::vector<HostItem> &items, int64_t lse_stride, const Shape &sh,
-                    float scale, void *out, float *lse, cudaStream_t stream) {
+                    float scale, void *out, float *lse, cudaStream_t stream,
+                    const SplitPlan &sp = SplitPlan(), void *workspace = nullptr) {
   using L = Layout<D>;
   static AttnParams<MAXI> prm;  // large: build in static storage, guarded below
   static std::mutex mu;
@@ -589,7 +773,7 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     d.len = static_cast<int32_t>(h.len);
     d.q_blocks = static_cast<int32_t>((h.len + kBlockM - 1) / kBlockM);
     d.cta_begin = static_cast<int32_t>(ctas);
-    ctas += static_cast<int64_t>(d.q_blocks) * sh.n_kv_heads * pairs;
+    ctas += static_cast<int64_t>(d.q_blocks) * sh.n_kv_heads * pairs * sp.splits;
     ++n;
   }
   if (n == 0) return MOCAP_OK;
@@ -604,6 +788,12 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
   prm.heads_per_group = group;
   prm.pairs_per_group = pairs;
   prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
+  prm.splits = sp.splits;
+  if (sp.splits > 1) {
+    if (n != 1 || workspace == nullptr) return MOCAP_EINVAL;
+    prm.o_part = static_cast<float *>(workspace);
+    prm.lse_part = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + sp.lse_off);
+  }
 
   auto kern = chunk_attn_kernel<D, MAXI>;
   static bool attr_done[64] = {};
@@ -619,16 +809,27 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     attr_done[dev] = true;
   }
   kern<<<static_cast<unsigned>(ctas), kThreads, L::kBytes, stream>>>(prm);
-  return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+  if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
+  if (sp.splits > 1) {
+    const int64_t len = items[0].len;
+    const int64_t warps = len * sh.n_q_heads;
+    attn_combine_kernel<D><<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
+        prm.o_part, prm.lse_part, sp.splits, len, sh.n_q_heads, prm.out, lse, lse_stride);
+    if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
+  }
+  return MOCAP_OK;
 }
 
 template <int MAXI>
 mocap_status dispatch(const void *q, const void *k_cache, const void *v_cache,
                       const std::vector<HostItem> &items, int64_t lse_stride, const Shape &sh,
-                      float scale, void *out, float *lse, cudaStream_t stream) {
+                      float scale, void *out, float *lse, cudaStream_t stream,
+                      const SplitPlan &sp = SplitPlan(), void *workspace = nullptr) {
   if (sh.head_dim == 128)
-    return launch<128, MAXI>(q, k_cache, v_cache, items, lse_stride, sh, scale, out, lse, stream);
-  return launch<64, MAXI>(q, k_cache, v_cache, items, lse_stride, sh, scale, out, lse, stream);
+    return launch<128, MAXI>(q, k_cache, v_cache, items, lse_stride, sh, scale, out, lse, stream,
+                             sp, workspace);
+  return launch<64, MAXI>(q, k_cache, v_cache, items, lse_stride, sh, scale, out, lse, stream, sp,
+                          workspace);
 }
 
 bool pointers_ok(const void *q, const void *k, const void *v, const void *out, const float *lse) {
@@ -644,24 +845,53 @@ constexpr int64_t kMaxRows = 0x7fffffffLL;
 
 using mocap::HostItem;
 
-extern "C" size_t mocap_chunk_attn_workspace_size(int64_t, int64_t, int32_t, int32_t) { return 0; }
+namespace {
+// The split the library uses for this shape when given enough workspace.
+mocap::SplitPlan plan_for(int64_t prefix, int64_t len, int32_t n_q_heads, int32_t n_kv_heads,
+                          int32_t head_dim) {
+  const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
+  if (mocap::check_shape(sh, 1.0f) != MOCAP_OK || prefix < 0 || len <= 0 ||
+      prefix > mocap::kMaxRows - len)
+    return mocap::SplitPlan();
+  int splits =
+      mocap::choose_splits(prefix, len, n_q_heads, n_kv_heads, head_dim, mocap::sm_count_cached());
+  // MOCAP_SPLIT_KV: 0 never splits; 1..4 forces that count (tests, tuning),
+  // capped so the first row block still has a key tile per split.
+  if (const char *env = std::getenv("MOCAP_SPLIT_KV")) {
+    const int forced = std::atoi(env);
+    if (forced >= 0 && forced <= 4) {
+      const int64_t min_tiles = (std::min<int64_t>(prefix + mocap::kBlockM, prefix + len) +
+                                 mocap::kBlockN - 1) / mocap::kBlockN;
+      splits = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(forced, min_tiles)));
+    }
+  }
+  return mocap::split_layout(splits, len, n_q_heads, head_dim);
+}
+}  // namespace
+
+extern "C" size_t mocap_chunk_attn_workspace_size(int64_t prefix, int64_t len, int32_t n_q_heads,
+                                                  int32_t n_kv_heads, int32_t head_dim) {
+  return plan_for(prefix, len, n_q_heads, n_kv_heads, head_dim).bytes;
+}
 
 extern "C" mocap_status mocap_chunk_attn(const void *q, const void *k_cache, const void *v_cache,
                                          int64_t prefix, int64_t len, int32_t n_q_heads,
                                          int32_t n_kv_heads, int32_t head_dim, float scale,
                                          void *out, float *lse, void *workspace,
                                          size_t workspace_bytes, mocap_stream_t stream) {
-  (void)workspace;
-  (void)workspace_bytes;
   const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
   const mocap_status st = mocap::check_shape(sh, scale);
   if (st != MOCAP_OK) return st;
   if (prefix < 0 || len < 0 || prefix > mocap::kMaxRows - len) return MOCAP_EINVAL;
   if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
+  if (workspace != nullptr && !mocap::aligned16(workspace)) return MOCAP_EINVAL;
   if (len == 0) return MOCAP_OK;
+  // Split the key range only when the caller's scratch holds the partials.
+  mocap::SplitPlan sp = plan_for(prefix, len, n_q_heads, n_kv_heads, head_dim);
+  if (sp.splits > 1 && (workspace == nullptr || workspace_bytes < sp.bytes)) sp = mocap::SplitPlan();
   std::vector<HostItem> items{{0, 0, prefix, len}};
   return mocap::dispatch<1>(q, k_cache, v_cache, items, len, sh, scale, out, lse,
-                            reinterpret_cast<cudaStream_t>(stream));
+                            reinterpret_cast<cudaStream_t>(stream), sp, workspace);
 }
 
 extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache,

@@ -14,7 +14,7 @@ from typing import List, Optional
 import torch
 
 from . import (MOCAP_PART_LBCP, MOCAP_PART_UNIFORM, mocap_chunk_attn, mocap_chunk_attn_varlen,
-               mocap_kv_append, mocap_lbcp_partition)
+               mocap_chunk_attn_workspace_size, mocap_kv_append, mocap_lbcp_partition)
 from .workloads import GRANULARITY, Workload, request_offsets
 
 
@@ -28,7 +28,7 @@ class ChunkedPrefill:
     ``[Hq, T]`` array over the packed rows.
     """
 
-    def __init__(self, w: Workload, device, mode: Optional[int] = None):
+    def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True):
         self.w = w
         self.device = torch.device(device)
         self.mode = w.mode if mode is None else mode
@@ -42,6 +42,15 @@ class ChunkedPrefill:
         self.out = torch.empty((total, w.n_q_heads, w.head_dim), **kw)
         self.lse = torch.empty((w.n_q_heads * total,), device=self.device, dtype=torch.float32)
         self.single = len(w.seq_lens) == 1
+        # Split-KV scratch for the single-request path: the largest any chunk uses.
+        self.workspace = None
+        if self.single and split_kv:
+            b = self.bounds[0]
+            need = max(mocap_chunk_attn_workspace_size(b[i], b[i + 1] - b[i], w.n_q_heads,
+                                                       w.n_kv_heads, w.head_dim)
+                       for i in range(len(b) - 1))
+            if need > 0:
+                self.workspace = torch.empty((need,), device=self.device, dtype=torch.uint8)
 
     def partition(self):
         """Chunk boundaries of every request (host call into the library)."""
@@ -87,7 +96,8 @@ class ChunkedPrefill:
             (_, c), = step
             b0, b1 = self.bounds[0][c], self.bounds[0][c + 1]
             mocap_chunk_attn(q[b0:b1], self.k_cache, self.v_cache, b0, self.out[b0:b1],
-                             self.chunk_lse(c), w.scale, stream=stream)
+                             self.chunk_lse(c), w.scale, workspace=self.workspace,
+                             stream=stream)
         else:
             items = []
             for r, c in step:

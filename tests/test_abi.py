@@ -154,3 +154,22 @@ def test_varlen_rejects_bad_items_before_launch(lib):
     assert call([(0, 0, 0, 10)], n=-1) == 1
     assert call([]) == 0
     assert call([(0, 0, 5, 0)]) == 0                     # empty item: no-op
+
+
+def test_workspace_size_split_plan(lib):
+    # many row blocks: no split; few long row blocks: a split and its layout
+    assert lib.mocap_chunk_attn_workspace_size(0, 23168, 64, 8, 128) == 0
+    ws = lib.mocap_chunk_attn_workspace_size(129024, 2048, 64, 8, 128)
+    if ws:
+        splits = None
+        for s in (2, 3, 4):
+            o = s * 2048 * 64 * 128 * 4
+            if ws == (o + 255) // 256 * 256 + s * 64 * 2048 * 4:
+                splits = s
+        assert splits is not None, ws
+    # tiny: one 8-unit chunk with a long prefix always splits
+    assert lib.mocap_chunk_attn_workspace_size(100000, 256, 8, 2, 128) > 0
+    # invalid shapes report 0
+    assert lib.mocap_chunk_attn_workspace_size(0, 100, 6, 4, 128) == 0
+    assert lib.mocap_chunk_attn_workspace_size(0, 100, 8, 2, 96) == 0
+    assert lib.mocap_chunk_attn_workspace_size(-1, 100, 8, 2, 128) == 0

@@ -249,3 +249,48 @@ def test_workload5_varlen_sampled(m):
                                              w.scale)
             assert_close(pf.out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref,
                          l_ref, f"request {r} chunk {i}")
+
+
+SPLIT_CASES = [
+    # (prefix, len, Hq, Hkv, d, forced splits or None for the library's choice)
+    (100000, 256, 8, 2, 128, None),   # few row blocks, long prefix: the heuristic splits
+    (4096, 500, 8, 2, 128, None),
+    (100, 300, 8, 2, 128, 2),         # row block 0's 2nd split sees no key for rows 0..27
+    (200, 2000, 8, 2, 128, 3),
+    (1000, 130, 4, 4, 64, 4),
+    (6000, 1, 6, 2, 128, 4),
+    (129024 - 2 * 128 + 77, 2048, 64, 8, 128, 2),  # late chunk of the 128k shape, unaligned
+]
+
+
+@pytest.mark.parametrize("prefix,length,hq,hkv,d,forced", SPLIT_CASES)
+def test_split_kv_matches_oracle_and_single_pass(m, monkeypatch, prefix, length, hq, hkv, d,
+                                                 forced):
+    if forced is not None:
+        monkeypatch.setenv("MOCAP_SPLIT_KV", str(forced))
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(prefix + length)
+    s = prefix + length
+    q = _randn((length, hq, d), gen, dev)
+    k, v = _randn((s, hkv, d), gen, dev), _randn((s, hkv, d), gen, dev)
+    scale = 1.0 / math.sqrt(d)
+    ws_bytes = m.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d)
+    assert ws_bytes > 0, "shape chosen to exercise the split path"
+    ws = torch.full((ws_bytes,), 0xFF, device=dev, dtype=torch.uint8)  # NaN garbage
+    out_s = torch.empty((length, hq, d), device=dev, dtype=torch.bfloat16)
+    lse_s = torch.empty((hq, length), device=dev, dtype=torch.float32)
+    m.mocap_chunk_attn(q, k, v, prefix, out_s, lse_s, scale, workspace=ws)
+    out_1 = torch.empty_like(out_s)
+    lse_1 = torch.empty_like(lse_s)
+    m.mocap_chunk_attn(q, k, v, prefix, out_1, lse_1, scale)  # no workspace: single pass
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    rows = np.arange(length) if length <= 512 else sample_rows(length, every=37)
+    idx = torch.as_tensor(rows, device=dev)
+    o_ref, l_ref = chunk_rows_oracle(f64(q[idx]), f64(k), f64(v), prefix, rows, scale)
+    assert_close(out_s[idx].float().cpu().numpy(), lse_s[:, idx].cpu().numpy(), o_ref, l_ref,
+                 "split")
+    assert_close(out_1[idx].float().cpu().numpy(), lse_1[:, idx].cpu().numpy(), o_ref, l_ref,
+                 "single")
+    assert (out_s.float() - out_1.float()).abs().max().item() <= 1e-2
+    assert (lse_s - lse_1).abs().max().item() <= 1e-4
