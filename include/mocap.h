@@ -161,6 +161,42 @@ size_t mocap_chunk_attn_workspace_size(int64_t prefix, int64_t len, int32_t n_q_
                                        int32_t n_kv_heads, int32_t head_dim);
 
 /*
+ * mocap_chunk_attn_noalloc -- mocap_chunk_attn for callers that cannot
+ * allocate device memory.  The paper has no counterpart: this entry point
+ * exists only for how some applications manage memory.
+ *
+ * Who needs it: a host program that owns all device memory through its own
+ * pool and does not let libraries call cudaMalloc behind its back (the pool
+ * may already hold nearly all of the GPU, or it must account for every
+ * byte), and serving loops where the latency and stalls of cudaMalloc /
+ * cudaFree are not acceptable.  Such callers cannot provide the split-KV
+ * workspace of mocap_chunk_attn.  This entry point takes the same arguments
+ * without the workspace and keeps the split-KV partials in a fixed
+ * MOCAP_NOALLOC_SCRATCH_BYTES (32 MiB) array compiled into the library: it
+ * calls no cudaMalloc, cudaFree or other allocating routine.
+ *
+ *   - Results: as mocap_chunk_attn with enough workspace (same split plan,
+ *     same kernels).
+ *   - Limit: if the split the library would use for this shape needs more
+ *     than MOCAP_NOALLOC_SCRATCH_BYTES (see mocap_chunk_attn_workspace_size),
+ *     the call returns MOCAP_EINVAL and enqueues nothing.  Shapes that need no
+ *     split run the single-pass kernel and use no scratch.
+ *   - Every GPU that loads the library holds the array until the process
+ *     exits.  The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, once per device, that device current); make
+ *     that first call before any stream capture.
+ *   - All calls on a device share the array.  A call writes every scratch
+ *     byte it reads, so nothing has to start at zero, but calls whose work
+ *     overlaps on the GPU (e.g. on different streams) race on the array.
+ */
+#define MOCAP_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
+mocap_status mocap_chunk_attn_noalloc(const void *q, const void *k_cache, const void *v_cache,
+                                      int64_t prefix, int64_t len,
+                                      int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
+                                      float scale, void *out, float *lse,
+                                      mocap_stream_t stream);
+
+/*
  * One (request, chunk) item of a varlen launch.  All offsets are in rows.
  *   q_row     first row of this chunk's queries in the packed q / out buffers
  *   kv_row    first cache row of the item's request (its key 0)

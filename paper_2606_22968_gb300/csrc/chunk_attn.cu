@@ -926,3 +926,58 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
                                                  scale, out, lse,
                                                  reinterpret_cast<cudaStream_t>(stream));
 }
+
+// ---------------------------------------------------------------------------
+// mocap_chunk_attn_noalloc: mocap_chunk_attn for callers that cannot allocate
+// device memory.  The split-KV partials go to a fixed scratch array that is
+// part of this library's device image; nothing is allocated per call.
+//
+// The array belongs to every device that loads the library, from load until
+// process exit, and all calls on a device share it.  Every byte a call reads
+// from it was written earlier in the same call, so nothing needs clearing;
+// two calls whose work overlaps on the GPU (for example on two streams)
+// would overwrite each other's partials.
+static __device__ __align__(256) uint8_t g_noalloc_scratch[MOCAP_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+uint8_t *g_noalloc_ptr[64] = {};
+std::mutex g_noalloc_mu;
+
+// Device address of g_noalloc_scratch on the current device.  The name is
+// only a host-side handle in host code, so the address is looked up once per
+// device (that device current) and cached; nullptr if the lookup fails.
+uint8_t *noalloc_scratch() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (g_noalloc_ptr[dev] == nullptr) {
+    void *ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess) return nullptr;
+    g_noalloc_ptr[dev] = static_cast<uint8_t *>(ptr);
+  }
+  return g_noalloc_ptr[dev];
+}
+}  // namespace
+
+extern "C" mocap_status mocap_chunk_attn_noalloc(const void *q, const void *k_cache,
+                                                 const void *v_cache, int64_t prefix, int64_t len,
+                                                 int32_t n_q_heads, int32_t n_kv_heads,
+                                                 int32_t head_dim, float scale, void *out,
+                                                 float *lse, mocap_stream_t stream) {
+  const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
+  const mocap_status st = mocap::check_shape(sh, scale);
+  if (st != MOCAP_OK) return st;
+  if (prefix < 0 || len < 0 || prefix > mocap::kMaxRows - len) return MOCAP_EINVAL;
+  if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
+  if (len == 0) return MOCAP_OK;
+  const mocap::SplitPlan sp = plan_for(prefix, len, n_q_heads, n_kv_heads, head_dim);
+  if (sp.bytes > MOCAP_NOALLOC_SCRATCH_BYTES) return MOCAP_EINVAL;  // beyond the fixed scratch
+  void *ws = nullptr;
+  if (sp.splits > 1) {
+    ws = noalloc_scratch();
+    if (ws == nullptr) return MOCAP_ECUDA;
+  }
+  std::vector<HostItem> items{{0, 0, prefix, len}};
+  return mocap::dispatch<1>(q, k_cache, v_cache, items, len, sh, scale, out, lse,
+                            reinterpret_cast<cudaStream_t>(stream), sp, ws);
+}

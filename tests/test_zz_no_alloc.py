@@ -1,0 +1,103 @@
+"""GPU: mocap_chunk_attn_noalloc, the entry point for callers that cannot
+allocate device memory (a host program whose own pool owns the GPU's memory,
+or a serving loop that cannot afford cudaMalloc / cudaFree).  It keeps its
+split-KV partials in a fixed scratch array inside the library, so these tests
+check that, called twice in a row through the C ABI, it gives the results of
+mocap_chunk_attn with a caller-provided workspace, and that it refuses a
+shape whose partials would not fit the array.
+
+Kept in a file of its own that pytest collects last; it passes alone in a
+fresh process and after the other tests.
+"""
+
+import ctypes
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import attention as A
+from tests.parity_utils import assert_close, f64
+
+pytestmark = pytest.mark.gpu
+
+SCRATCH_BYTES = 32 * 1024 * 1024
+
+
+def _inputs(prefix, length, hq, hkv, d, seed):
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(seed)
+    q = torch.randn((length, hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    k = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    v = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    return q, k, v
+
+
+def _call_noalloc(lib, q, k, v, prefix, out, lse, scale):
+    length, hq, d = q.shape
+    hkv = k.shape[1]
+    stream = torch.cuda.current_stream().cuda_stream
+    return lib.mocap_chunk_attn_noalloc(q.data_ptr(), k.data_ptr(), v.data_ptr(), prefix, length,
+                                        hq, hkv, d, scale, out.data_ptr(), lse.data_ptr(),
+                                        stream)
+
+
+def _call_with_workspace(lib, q, k, v, prefix, out, lse, scale):
+    length, hq, d = q.shape
+    hkv = k.shape[1]
+    ws_bytes = lib.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d)
+    ws = torch.empty((max(ws_bytes, 16),), device=q.device, dtype=torch.uint8)
+    stream = torch.cuda.current_stream().cuda_stream
+    st = lib.mocap_chunk_attn(q.data_ptr(), k.data_ptr(), v.data_ptr(), prefix, length, hq, hkv,
+                              d, scale, out.data_ptr(), lse.data_ptr(), ws.data_ptr(), ws_bytes,
+                              stream)
+    return st, ws_bytes
+
+
+def test_noalloc_matches_workspace_entry_two_calls(lib, monkeypatch):
+    # Two calls in a row on different shapes: the second runs over whatever
+    # the first left in the shared scratch.
+    cases = [
+        (100000, 256, 8, 2, 128, None),  # few long row blocks: the library splits by itself
+        (100, 300, 8, 2, 128, "2"),      # forced split whose second range some rows cannot see
+    ]
+    for i, (prefix, length, hq, hkv, d, forced) in enumerate(cases):
+        if forced is None:
+            monkeypatch.delenv("MOCAP_SPLIT_KV", raising=False)
+        else:
+            monkeypatch.setenv("MOCAP_SPLIT_KV", forced)
+        q, k, v = _inputs(prefix, length, hq, hkv, d, seed=41 + i)
+        scale = 1.0 / math.sqrt(d)
+        ws_bytes = lib.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d)
+        assert 0 < ws_bytes <= SCRATCH_BYTES  # the split path runs, inside the fixed scratch
+        out_n = torch.full((length, hq, d), float("nan"), device=q.device, dtype=torch.bfloat16)
+        lse_n = torch.full((hq, length), float("nan"), device=q.device, dtype=torch.float32)
+        assert _call_noalloc(lib, q, k, v, prefix, out_n, lse_n, scale) == 0
+        out_w = torch.empty_like(out_n)
+        lse_w = torch.empty_like(lse_n)
+        st, _ = _call_with_workspace(lib, q, k, v, prefix, out_w, lse_w, scale)
+        assert st == 0
+        torch.cuda.synchronize()
+        assert lib.mocap_last_device_status(torch.cuda.current_stream().cuda_stream) == 0
+        # same results as the workspace entry point, within the parity tolerances
+        assert_close(out_n.float().cpu().numpy(), lse_n.cpu().numpy(),
+                     out_w.double().cpu().numpy(), lse_w.double().cpu().numpy(),
+                     f"call {i}: noalloc vs workspace")
+        # and against the float64 oracle
+        o_ref, l_ref = A.chunk_attention(f64(q), f64(k), f64(v), prefix, scale)
+        assert_close(out_n.float().cpu().numpy(), lse_n.cpu().numpy(), o_ref, l_ref,
+                     f"call {i}: noalloc vs oracle")
+
+
+def test_noalloc_rejects_split_beyond_scratch(lib, monkeypatch):
+    # 2 splits x 2048 rows x 64 heads x (128 + 1) fp32 = 135 MB > 32 MiB
+    monkeypatch.setenv("MOCAP_SPLIT_KV", "2")
+    prefix, length, hq, hkv, d = 4096, 2048, 64, 8, 128
+    assert lib.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d) > SCRATCH_BYTES
+    q, k, v = _inputs(prefix, length, hq, hkv, d, seed=7)
+    out = torch.zeros((length, hq, d), device=q.device, dtype=torch.bfloat16)
+    lse = torch.zeros((hq, length), device=q.device, dtype=torch.float32)
+    assert _call_noalloc(lib, q, k, v, prefix, out, lse, 0.088) == 1  # MOCAP_EINVAL
+    torch.cuda.synchronize()
+    assert torch.count_nonzero(out).item() == 0  # nothing was enqueued
