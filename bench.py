@@ -271,6 +271,12 @@ def max_over_ranks(x, world, device):
     return float(t.item())
 
 
+def replica_throughput(units_per_rank, ms_per_step_max, world):
+    """Whole-job rate of N independent replicas: every rank processed the same
+    units per step; the slowest rank's step time bounds the job."""
+    return world * units_per_rank / (ms_per_step_max * 1e-3)
+
+
 def reference_arm(args, rank, world):
     """The float64 oracle, timed on the host cores on a bounded sample."""
     import torch
@@ -371,8 +377,8 @@ def ours_arm(args, rank, world, local):
                  for c in range(n_chunks)]
     cv = statistics.pstdev(per_chunk) / statistics.mean(per_chunk) if n_chunks > 1 else 0.0
 
-    value = world * total_flops / (ms_step * 1e-3) / 1e12
-    tokens_per_s = world * w.total_tokens / (ms_step * 1e-3)
+    value = replica_throughput(total_flops, ms_step, world) / 1e12
+    tokens_per_s = replica_throughput(w.total_tokens, ms_step, world)
     peaks, peak_src = load_peaks()
     peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAK_TFLOPS))
     attn_avg_ms = statistics.mean(attn_step_ms)

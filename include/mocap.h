@@ -15,6 +15,7 @@
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
  *   mocap_last_device_status  bounded-wait timeouts reported by the kernels
+ *   mocap_selftest_bounded_wait  drives that timeout path on purpose (tests)
  *   mocap_status_string       text for a status code
  *
  * Conventions for every entry point:
@@ -242,6 +243,19 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
  * MOCAP_ECUDA if the synchronisation itself failed.
  */
 mocap_status mocap_last_device_status(mocap_stream_t stream);
+
+/*
+ * mocap_selftest_bounded_wait -- exercises the kernels' failure path without
+ * a fault.  Every wait in this library's kernels is bounded: past its limit
+ * it records MOCAP_ETIMEOUT in the device status word and the kernel unwinds
+ * (no trap, no hang).  This launches a one-thread kernel that waits, with
+ * the same bounded wait, on a barrier nothing ever completes, for limit_us
+ * microseconds (1 .. 1000000, else MOCAP_EINVAL).  Afterwards
+ * mocap_last_device_status() reports MOCAP_ETIMEOUT, and until it is read
+ * every attention launch returns without doing work.  No counterpart in the
+ * paper: failure detection for shared GPUs.
+ */
+mocap_status mocap_selftest_bounded_wait(uint32_t limit_us, mocap_stream_t stream);
 
 /* Static, NUL-terminated name of a status code. */
 const char *mocap_status_string(mocap_status status);

@@ -111,5 +111,11 @@ def mocap_last_device_status(stream=None) -> int:
     return int(_lib.load().mocap_last_device_status(_stream(stream)))
 
 
+def mocap_selftest_bounded_wait(limit_us: int, stream=None):
+    """Launch a kernel whose bounded wait expires after limit_us (failure-path test)."""
+    _check(_lib.load().mocap_selftest_bounded_wait(limit_us, _stream(stream)),
+           "mocap_selftest_bounded_wait")
+
+
 def mocap_status_string(status: int) -> str:
     return _lib.load().mocap_status_string(status).decode()

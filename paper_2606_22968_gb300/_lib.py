@@ -30,6 +30,7 @@ SIGNATURES = {
                                         c_i64, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp, c_vp,
                                         c_vp]),
     "mocap_last_device_status": (c_i32, [c_vp]),
+    "mocap_selftest_bounded_wait": (c_i32, [ctypes.c_uint32, c_vp]),
     "mocap_status_string": (ctypes.c_char_p, [c_i32]),
 }
 

@@ -2,6 +2,7 @@
 #include <mutex>
 
 #include "internal.h"
+#include "sm103_ptx.cuh"
 
 namespace {
 __device__ uint32_t g_device_status;  // 0 = OK, MOCAP_ETIMEOUT after an expired wait
@@ -48,4 +49,27 @@ extern "C" const char *mocap_status_string(mocap_status status) {
     case MOCAP_ETIMEOUT: return "MOCAP_ETIMEOUT: device wait expired";
   }
   return "MOCAP_UNKNOWN";
+}
+
+namespace {
+// One thread waits, through the same bounded wait the attention kernel uses,
+// on an mbarrier that nothing ever arrives on.
+__global__ void bounded_wait_selftest_kernel(uint32_t *status, uint64_t limit_ns) {
+  __shared__ alignas(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    const uint32_t b = mocap::smem_u32(&bar);
+    mocap::mbar_init(b, 1);
+    mocap::fence_mbar_init();
+    mocap::mbar_wait(b, 0, status, limit_ns, false);
+  }
+}
+}  // namespace
+
+extern "C" mocap_status mocap_selftest_bounded_wait(uint32_t limit_us, mocap_stream_t stream) {
+  if (limit_us == 0 || limit_us > 1000000u) return MOCAP_EINVAL;
+  uint32_t *status = mocap::device_status_ptr();
+  if (status == nullptr) return MOCAP_ECUDA;
+  bounded_wait_selftest_kernel<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      status, static_cast<uint64_t>(limit_us) * 1000u);
+  return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
 }

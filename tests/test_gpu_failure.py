@@ -1,0 +1,65 @@
+"""GPU failure detection without a GPU fault: a bounded wait that expires
+records MOCAP_ETIMEOUT, the host reads (and clears) it, launches made while
+it is set do nothing, and the context stays usable."""
+
+import math
+import time
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import attention as A
+from tests.parity_utils import assert_close, f64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def m():
+    import paper_2606_22968_gb300 as mod
+    mod._lib.load()
+    return mod
+
+
+def _small(dev, seed=3):
+    gen = torch.Generator(device=dev).manual_seed(seed)
+    q = torch.randn((300, 8, 128), generator=gen, device=dev, dtype=torch.bfloat16)
+    k = torch.randn((300, 2, 128), generator=gen, device=dev, dtype=torch.bfloat16)
+    v = torch.randn((300, 2, 128), generator=gen, device=dev, dtype=torch.bfloat16)
+    return q, k, v
+
+
+def test_expired_wait_is_reported_and_cleared(m):
+    assert m.mocap_last_device_status() == m.MOCAP_OK
+    t0 = time.perf_counter()
+    m.mocap_selftest_bounded_wait(50000)  # 50 ms
+    st = m.mocap_last_device_status()     # synchronises the stream
+    elapsed = time.perf_counter() - t0
+    assert st == m.MOCAP_ETIMEOUT
+    assert elapsed >= 0.045
+    assert m.mocap_last_device_status() == m.MOCAP_OK  # read clears it
+
+
+def test_launch_after_expired_wait_does_nothing_then_recovers(m):
+    dev = torch.device("cuda")
+    q, k, v = _small(dev)
+    out = torch.full_like(q, float("nan"))
+    lse = torch.full((8, 300), float("nan"), device=dev, dtype=torch.float32)
+    m.mocap_selftest_bounded_wait(20000)
+    m.mocap_chunk_attn(q, k, v, 0, out, lse, 0.088)   # queued behind the expired wait
+    torch.cuda.synchronize()
+    assert torch.isnan(out.float()).all() and torch.isnan(lse).all()
+    assert m.mocap_last_device_status() == m.MOCAP_ETIMEOUT
+    # the context is usable: the same launch now computes the right answer
+    m.mocap_chunk_attn(q, k, v, 0, out, lse, 0.088)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == m.MOCAP_OK
+    o_ref, l_ref = A.causal_attention(f64(q), f64(k), f64(v), 0.088)
+    assert_close(out.float().cpu().numpy(), lse.cpu().numpy(), o_ref, l_ref)
+
+
+def test_selftest_rejects_bad_limits(m):
+    for bad in (0, 1000001):
+        with pytest.raises(m.MocapError):
+            m.mocap_selftest_bounded_wait(bad)
