@@ -6,7 +6,8 @@
 // balances.  The kernel computes, for query head h (KV head h / group) and
 // global row t, O_t = softmax_{j<=t}(scale q_t.k_j) V and LSE_t = ln sum exp.
 //
-// Design (one CTA = 128 query rows x up to two query heads of one KV group):
+// Design (one CTA = 128 query rows x up to two query heads of one KV group;
+// CTAs are ordered KV-group-major, heaviest row block first within a group):
 //   warp 0        TMA producer: Q tiles once, then K_j, V_j tiles (128 keys)
 //                 through a 4-deep ring of 128-byte-swizzled smem stages.
 //   warp 1        MMA issuer (one thread): S_s = Q_s K_j^T into TMEM, then
@@ -492,13 +493,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   while (item + 1 < p.n_items && cta >= p.items[item + 1].cta_begin) ++item;
   const ItemDesc it = p.items[item];
   int w = cta - it.cta_begin;
+  // CTA order: head pair fastest, then split, then row block (heaviest
+  // first), then KV group slowest, so the CTAs resident at once mostly
+  // stream the same group's K/V through L2 (less DRAM traffic and power).
   const int pair = w % p.pairs_per_group;
   w /= p.pairs_per_group;
-  const int g = w % p.n_kv_heads;
-  w /= p.n_kv_heads;
   const int split = w % p.splits;
   w /= p.splits;
-  const int qblock = it.q_blocks - 1 - w;  // heaviest (latest) row blocks first
+  const int qblock = it.q_blocks - 1 - w % it.q_blocks;
+  const int g = w / it.q_blocks;
   const int r0 = qblock * kBlockM;
   const int h0 = g * p.heads_per_group + 2 * pair;
   const int nslots = min(2, p.heads_per_group - 2 * pair);
