@@ -434,8 +434,8 @@ def ours_arm(args, rank, world, local):
 
 def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
     """The same metric through the public API with host buffers: each step
-    copies Q/K/V from pinned host memory, runs the hot path and copies O and
-    LSE back."""
+    runs ChunkedPrefill.run_from_host, which copies every chunk's Q/K/V from
+    pinned host memory and its O and LSE back, overlapped with compute."""
     import torch
     hq, hk, hv = (t.cpu().pin_memory() for t in (q, k, v))
     ho = torch.empty(pf.out.shape, dtype=pf.out.dtype).pin_memory()
@@ -445,13 +445,8 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
     d2h = ho.numel() * ho.element_size() + hl.numel() * hl.element_size()
 
     def step():
-        dq.copy_(hq, non_blocking=True)
-        dk.copy_(hk, non_blocking=True)
-        dv.copy_(hv, non_blocking=True)
         pf.partition()
-        pf.run(dq, dk, dv, stream)
-        ho.copy_(pf.out, non_blocking=True)
-        hl.copy_(pf.lse, non_blocking=True)
+        pf.run_from_host(hq, hk, hv, ho, hl, dq, dk, dv)
 
     step()
     torch.cuda.synchronize(dev)
@@ -465,40 +460,11 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
     torch.cuda.synchronize(dev)
     barrier(world)
     ms = max_over_ranks(t0.elapsed_time(t1) / args.e2e_steps, world, dev)
-    if not torch.equal(ho.to(dev), pf.out):
-        raise RuntimeError("e2e: host copy of O differs")
-    return {"value": world * total_flops / (ms * 1e-3) / 1e12, "unit": "TFLOP/s",
-            "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
-
-
-def profile_case(args):
-    """A single chunk_attn launch shape, repeated: the small case for ncu."""
-    import torch
-    import paper_2606_22968_gb300 as m
-    prefix, length, hq, hkv, d = (int(x) for x in args.case.split(","))
-    dev = torch.device("cuda")
-    gen = torch.Generator(device=dev).manual_seed(7)
-    q = torch.randn((length, hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
-    kc = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
-    vc = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
-    out = torch.empty_like(q)
-    lse = torch.empty((hq, length), device=dev, dtype=torch.float32)
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-    times = []
-    for i in range(args.warmup + args.steps):
-        ev[0].record()
-        m.mocap_chunk_attn(q, kc, vc, prefix, out, lse, 1.0 / math.sqrt(d))
-        ev[1].record()
-        torch.cuda.synchronize()
-        if i >= args.warmup:
-            times.append(ev[0].elapsed_time(ev[1]))
-    if m.mocap_last_device_status() != m.MOCAP_OK:
-        raise RuntimeError("device wait expired")
-    flops = 4 * hq * d * (length * prefix + length * (length + 1) // 2)
-    ms = statistics.median(times)
-    print(json.dumps({"case": args.case, "ms": ms, "tflops": flops / ms / 1e9,
-                      "kv_bytes": 2 * (prefix + length) * hkv * d * 2}), flush=True)
-    return 0
+    if not torch.equal(ho.to(dev), pf.out) or not torch.equal(hl.to(dev), pf.lse):
+        raise RuntimeError("e2e: host copies of O / LSE differ from the device results")
+    return {"value": replica_throughput(total_flops, ms, world) / 1e12, "unit": "TFLOP/s",
+            "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "overlap": "per-chunk H2D / compute / D2H on three streams"}
 
 
 def main():

@@ -114,3 +114,56 @@ class ChunkedPrefill:
         for i, step in enumerate(self.steps()):
             self.run_step(q, k, v, step, stream,
                           None if chunk_events is None else chunk_events[i])
+
+    # -- from host memory ------------------------------------------------------------
+    def _rows(self, r, c):
+        b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
+        return slice(self.cu[r] + b0, self.cu[r] + b1), b0, b1
+
+    def run_from_host(self, host_q, host_k, host_v, host_out, host_lse, q, k, v):
+        """The whole prompt from (pinned) host memory, overlapping transfers
+        with compute.
+
+        Every chunk's Q/K/V rows are copied into the device buffers ``q, k, v``
+        on a copy stream, in chunk order; the compute stream starts chunk i as
+        soon as its rows have landed, and a third stream copies chunk i's O
+        and LSE back to ``host_out`` / ``host_lse`` (shaped like ``self.out``
+        and ``self.lse``) as soon as its attention is done.  The caller's
+        current stream waits for everything before this returns."""
+        compute = torch.cuda.current_stream(self.device)
+        h2d = torch.cuda.Stream(self.device)
+        d2h = torch.cuda.Stream(self.device)
+        steps = self.steps()
+        hq = self.w.n_q_heads
+        landed = []
+        h2d.wait_stream(compute)  # device buffers are free of earlier work
+        with torch.cuda.stream(h2d):
+            for step in steps:
+                for r, c in step:
+                    rows, _, _ = self._rows(r, c)
+                    q[rows].copy_(host_q[rows], non_blocking=True)
+                    k[rows].copy_(host_k[rows], non_blocking=True)
+                    v[rows].copy_(host_v[rows], non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(h2d)
+                landed.append(ev)
+        d2h.wait_stream(compute)
+        lse2d = None if self.single else self.lse_packed()
+        host_lse2d = None if self.single else host_lse.view(hq, self.w.total_tokens)
+        for i, step in enumerate(steps):
+            compute.wait_event(landed[i])
+            self.run_step(q, k, v, step, compute)
+            done = torch.cuda.Event()
+            done.record(compute)
+            d2h.wait_event(done)
+            with torch.cuda.stream(d2h):
+                for r, c in step:
+                    rows, b0, b1 = self._rows(r, c)
+                    host_out[rows].copy_(self.out[rows], non_blocking=True)
+                    if self.single:
+                        host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
+                                                        non_blocking=True)
+                    else:
+                        host_lse2d[:, rows].copy_(lse2d[:, rows], non_blocking=True)
+        compute.wait_stream(d2h)
+        compute.wait_stream(h2d)

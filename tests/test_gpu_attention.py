@@ -294,3 +294,28 @@ def test_split_kv_matches_oracle_and_single_pass(m, monkeypatch, prefix, length,
                  "single")
     assert (out_s.float() - out_1.float()).abs().max().item() <= 1e-2
     assert (lse_s - lse_1).abs().max().item() <= 1e-4
+
+
+@pytest.mark.parametrize("index", [3, 5])
+def test_run_from_host_matches_device_run(m, index):
+    """Streaming the prompt from pinned host memory (overlapped copies) gives
+    exactly the device-resident results."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(index)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev)
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    out_ref, lse_ref = pf.out.clone(), pf.lse.clone()
+    pf.out.fill_(float("nan"))
+    pf.lse.fill_(float("nan"))
+    hq, hk, hv = (t.cpu().pin_memory() for t in (q, k, v))
+    ho = torch.full(pf.out.shape, float("nan"), dtype=pf.out.dtype).pin_memory()
+    hl = torch.full(pf.lse.shape, float("nan"), dtype=pf.lse.dtype).pin_memory()
+    dq, dk, dv = (torch.full_like(t, float("nan")) for t in (q, k, v))
+    pf.run_from_host(hq, hk, hv, ho, hl, dq, dk, dv)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    assert torch.equal(ho, out_ref.cpu()) and torch.equal(hl, lse_ref.cpu())
