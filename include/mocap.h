@@ -11,6 +11,7 @@
  * balance that cost.  The library exposes:
  *
  *   mocap_lbcp_partition      chunk boundaries (host, exact integers)
+ *   mocap_lbcp_partition_dp   boundaries from Algorithm 1's stage-1 DP (host)
  *   mocap_kv_append           chunk K/V -> contiguous bf16 KV cache (device)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
@@ -83,6 +84,39 @@ typedef enum {
 mocap_status mocap_lbcp_partition(int64_t seq_len, int32_t num_chunks,
                                   int32_t granularity, mocap_part_mode mode,
                                   int64_t *boundaries);
+
+typedef enum {
+  MOCAP_COST_CAUSAL = 0,   /* chunk cost c (p + c/2): causal (query, key) pairs */
+  MOCAP_COST_EQ1 = 1       /* chunk cost c (p + c): Eq. 1 as printed            */
+} mocap_cost_model;
+
+/*
+ * mocap_lbcp_partition_dp -- chunk boundaries from the dynamic program of
+ * Algorithm 1, stage 1 (Sec. 4.2): the compute-balanced initialisation that
+ * minimises t_sum + (N - 1) t_max for an N-stage chunked pipeline.
+ *
+ * Positions and sizes are counted in units of `granularity` (U = seq_len /
+ * g; the last chunk absorbs seq_len % g).  EvaluateChunk(k, s), the cost of a
+ * chunk of k units starting at unit s, is k (2 s + k) (MOCAP_COST_CAUSAL,
+ * twice c (p + c/2)) or 2 k (s + k) (MOCAP_COST_EQ1, twice Eq. 1's c (p + c)),
+ * plus gemm_weight * k for the GEMM term of Eq. 1.  The loops run as in the
+ * algorithm: chunk index m from M down to 1, start s from U-1 down to 0,
+ * size k upward; state (m, s) keeps the first k that gives the smallest
+ * t_sum + (N - 1) max(t, t_max) over its suffix.  Exact integer arithmetic:
+ * bit-exact on every platform.  The stage-2 simulated annealing of
+ * Algorithm 1 needs the paper's multi-stage execution model and is not
+ * provided.
+ *
+ *   num_stages   N >= 1 pipeline stages
+ *   gemm_weight  >= 0, weight of the linear term (same doubled units)
+ *   boundaries   HOST array of num_chunks + 1 int64, written on success
+ * MOCAP_EINVAL for bad arguments; MOCAP_EUNSUPPORTED when M * U^2 > 4e9 (the
+ * O(M U^2) host work would be too long; use a coarser granularity).
+ */
+mocap_status mocap_lbcp_partition_dp(int64_t seq_len, int32_t num_chunks,
+                                     int32_t granularity, int32_t num_stages,
+                                     mocap_cost_model model, int64_t gemm_weight,
+                                     int64_t *boundaries);
 
 /*
  * mocap_kv_append -- write a chunk's K and V into the KV cache.

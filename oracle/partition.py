@@ -116,3 +116,72 @@ def causal_pairs(bounds: List[int]) -> List[int]:
         c = bounds[i + 1] - bounds[i]
         out.append(c * p + c * (c + 1) // 2)
     return out
+
+
+# ---------------------------------------------------------------------------
+# Algorithm 1, stage 1 (Sec. 4.2): the compute-balanced DP initialisation.
+#
+# Positions and chunk sizes are counted in units of the granularity g
+# (U = S // g units; the last chunk absorbs S % g tokens).  EvaluateChunk(k, s)
+# is the compute cost of a chunk of k units starting at unit s, doubled so it
+# stays an integer:
+#   COST_CAUSAL: 2 * k (s + k/2) = k (2 s + k)      (c_i (p_i + c_i / 2))
+#   COST_EQ1:    2 * k (s + k)                       (Eq. 1 as printed)
+# plus gemm_weight * k for the GEMM term of Eq. 1 (cost proportional to c_i).
+# Suffix states (m, s) keep one (t_max, t_sum) pair: the one minimising
+# t_sum + (N - 1) t_max over the chunk sizes k tried in increasing order
+# (strict improvement, so the smallest k wins ties).
+
+COST_CAUSAL = 0
+COST_EQ1 = 1
+
+
+def evaluate_chunk(k: int, s: int, model: int, gemm_weight: int) -> int:
+    if model == COST_CAUSAL:
+        attn = k * (2 * s + k)
+    elif model == COST_EQ1:
+        attn = 2 * k * (s + k)
+    else:
+        raise ValueError("unknown cost model")
+    return attn + gemm_weight * k
+
+
+def dp_boundaries(seq_len: int, num_chunks: int, granularity: int, num_stages: int,
+                  model: int = COST_CAUSAL, gemm_weight: int = 0) -> List[int]:
+    """Chunk boundaries from stage 1 of Algorithm 1 (exact integers)."""
+    units = _check(seq_len, num_chunks, granularity)
+    if num_stages < 1 or gemm_weight < 0:
+        raise ValueError("num_stages >= 1 and gemm_weight >= 0 required")
+    M, S, N = num_chunks, units, num_stages
+    t_max = {(M + 1, S): 0}
+    t_sum = {(M + 1, S): 0}
+    ss = {}
+    for m in range(M, 0, -1):                      # chunk index, last first
+        for s in range(S - 1, -1, -1):             # start position, right to left
+            for k in range(1, S - s - (M - m) + 1):  # candidate chunk size
+                nxt = (m + 1, s + k)
+                if nxt not in t_max:
+                    continue
+                t = evaluate_chunk(k, s, model, gemm_weight)
+                tmax_new = max(t_max[nxt], t)
+                tsum_new = t_sum[nxt] + t
+                cur = (m, s)
+                if cur not in t_max or \
+                        tsum_new + (N - 1) * tmax_new < t_sum[cur] + (N - 1) * t_max[cur]:
+                    t_max[cur], t_sum[cur], ss[cur] = tmax_new, tsum_new, k
+    out, s = [0], 0
+    for m in range(1, M + 1):
+        s += ss[(m, s)]
+        out.append(granularity * s)
+    out[-1] = seq_len
+    return out
+
+
+def dp_objective(bounds: List[int], granularity: int, num_stages: int,
+                 model: int = COST_CAUSAL, gemm_weight: int = 0) -> int:
+    """t_sum + (N - 1) t_max of a partition whose interior boundaries are
+    multiples of the granularity (units as in dp_boundaries)."""
+    units = [b // granularity for b in bounds[:-1]] + [bounds[-1] // granularity]
+    costs = [evaluate_chunk(units[i + 1] - units[i], units[i], model, gemm_weight)
+             for i in range(len(units) - 1)]
+    return sum(costs) + (num_stages - 1) * max(costs)

@@ -61,6 +61,20 @@ def mocap_lbcp_partition(seq_len: int, num_chunks: int, granularity: int = 128,
     return list(out)
 
 
+MOCAP_COST_CAUSAL, MOCAP_COST_EQ1 = 0, 1
+
+
+def mocap_lbcp_partition_dp(seq_len: int, num_chunks: int, granularity: int = 128,
+                            num_stages: int = 16, model: int = MOCAP_COST_CAUSAL,
+                            gemm_weight: int = 0) -> List[int]:
+    """Boundaries from the stage-1 dynamic program of Algorithm 1."""
+    out = (ctypes.c_int64 * (num_chunks + 1))()
+    _check(_lib.load().mocap_lbcp_partition_dp(seq_len, num_chunks, granularity, num_stages,
+                                               model, gemm_weight, out),
+           "mocap_lbcp_partition_dp")
+    return list(out)
+
+
 def mocap_kv_append(k_chunk, v_chunk, k_cache, v_cache, offset: int, stream=None):
     """Copy chunk K/V ([len, Hkv, d] bf16) into cache rows [offset, offset+len)."""
     length, n_kv, d = k_chunk.shape

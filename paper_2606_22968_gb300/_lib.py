@@ -20,6 +20,8 @@ class VarlenItem(ctypes.Structure):
 
 SIGNATURES = {
     "mocap_lbcp_partition": (c_i32, [c_i64, c_i32, c_i32, c_i32, ctypes.POINTER(c_i64)]),
+    "mocap_lbcp_partition_dp": (c_i32, [c_i64, c_i32, c_i32, c_i32, c_i32, c_i64,
+                                        ctypes.POINTER(c_i64)]),
     "mocap_kv_append": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32, c_i32, c_vp]),
     "mocap_chunk_attn": (c_i32, [c_vp, c_vp, c_vp, c_i64, c_i64, c_i32, c_i32, c_i32, c_f32,
                                  c_vp, c_vp, c_vp, c_sz, c_vp]),

@@ -11,6 +11,7 @@
 //   b_i = min(max(g n_i, b_{i-1} + g), g (U - (M - i))),  b_0 = 0, b_M = S.
 // Uniform mode: n_i = round_half_up(i U / M) = floor((2 i U + M) / (2 M)).
 #include <cstdint>
+#include <vector>
 
 #include "internal.h"
 
@@ -65,5 +66,64 @@ extern "C" mocap_status mocap_lbcp_partition(int64_t seq_len, int32_t num_chunks
     boundaries[i] = b;
   }
   boundaries[m] = seq_len;
+  return MOCAP_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Stage 1 of Algorithm 1 (Sec. 4.2): dynamic programming over (chunk index m,
+// start position s, chunk size k), all counted in units of the granularity.
+// Suffix state (m, s) keeps the (t_max, t_sum) of the chunk sizes tried so far
+// that minimises t_sum + (N - 1) t_max; k is tried in increasing order and
+// only a strict improvement replaces the kept choice.  EvaluateChunk is the
+// chunk's compute cost, doubled to stay integral: k (2 s + k) for the causal
+// count c (p + c/2), 2 k (s + k) for Eq. 1 as printed, plus gemm_weight * k.
+extern "C" mocap_status mocap_lbcp_partition_dp(int64_t seq_len, int32_t num_chunks,
+                                                int32_t granularity, int32_t num_stages,
+                                                mocap_cost_model model, int64_t gemm_weight,
+                                                int64_t *boundaries) {
+  if (boundaries == nullptr || seq_len <= 0 || num_chunks < 1 || granularity < 1 ||
+      num_stages < 1 || gemm_weight < 0)
+    return MOCAP_EINVAL;
+  if (model != MOCAP_COST_CAUSAL && model != MOCAP_COST_EQ1) return MOCAP_EINVAL;
+  if (static_cast<int64_t>(num_chunks) * granularity > seq_len) return MOCAP_EINVAL;
+  const int64_t U = seq_len / granularity;
+  const int64_t M = num_chunks;
+  if (static_cast<double>(M) * static_cast<double>(U) * static_cast<double>(U) > 4e9)
+    return MOCAP_EUNSUPPORTED;  // O(M U^2) host work; use a coarser granularity
+  if (gemm_weight > (int64_t(1) << 40)) return MOCAP_EINVAL;
+  const int64_t nm1 = num_stages - 1;
+  const size_t W = static_cast<size_t>(U + 1);
+  auto at = [&](int64_t m, int64_t s) { return static_cast<size_t>(m) * W + static_cast<size_t>(s); };
+  std::vector<int64_t> t_max(static_cast<size_t>(M + 2) * W, 0), t_sum(t_max.size(), 0);
+  std::vector<uint8_t> set(t_max.size(), 0);
+  std::vector<int32_t> ss(t_max.size(), 0);
+  set[at(M + 1, U)] = 1;
+  for (int64_t m = M; m >= 1; --m) {
+    for (int64_t s = U - 1; s >= 0; --s) {
+      const size_t cur = at(m, s);
+      for (int64_t k = 1; k <= U - s - (M - m); ++k) {
+        const size_t nxt = at(m + 1, s + k);
+        if (!set[nxt]) continue;
+        const int64_t attn = model == MOCAP_COST_CAUSAL ? k * (2 * s + k) : 2 * k * (s + k);
+        const int64_t t = attn + gemm_weight * k;
+        const int64_t tmax_new = t_max[nxt] > t ? t_max[nxt] : t;
+        const int64_t tsum_new = t_sum[nxt] + t;
+        if (!set[cur] || tsum_new + nm1 * tmax_new < t_sum[cur] + nm1 * t_max[cur]) {
+          t_max[cur] = tmax_new;
+          t_sum[cur] = tsum_new;
+          ss[cur] = static_cast<int32_t>(k);
+          set[cur] = 1;
+        }
+      }
+    }
+  }
+  if (!set[at(1, 0)]) return MOCAP_EINVAL;
+  boundaries[0] = 0;
+  int64_t s = 0;
+  for (int64_t m = 1; m <= M; ++m) {
+    s += ss[at(m, s)];
+    boundaries[m] = granularity * s;
+  }
+  boundaries[M] = seq_len;
   return MOCAP_OK;
 }

@@ -173,3 +173,28 @@ def test_workspace_size_split_plan(lib):
     assert lib.mocap_chunk_attn_workspace_size(0, 100, 6, 4, 128) == 0
     assert lib.mocap_chunk_attn_workspace_size(0, 100, 8, 2, 96) == 0
     assert lib.mocap_chunk_attn_workspace_size(-1, 100, 8, 2, 128) == 0
+
+
+def test_dp_partition_bit_exact_vs_oracle(lib):
+    rnd = random.Random(9)
+    for _ in range(60):
+        g = rnd.choice([64, 128, 256])
+        units = rnd.randint(1, 160)
+        m = rnd.randint(1, min(units, 12))
+        s = units * g + rnd.choice([0, 0, 1, 63])
+        n = rnd.choice([1, 2, 4, 16, 1000])
+        model = rnd.randint(0, 1)
+        gemm = rnd.choice([0, 5, 1000])
+        out = (ctypes.c_int64 * (m + 1))()
+        assert lib.mocap_lbcp_partition_dp(s, m, g, n, model, gemm, out) == 0
+        assert list(out) == P.dp_boundaries(s, m, g, n, model, gemm), (s, m, g, n, model, gemm)
+
+
+def test_dp_partition_invalid_and_limits(lib):
+    out = (ctypes.c_int64 * 40)()
+    assert lib.mocap_lbcp_partition_dp(1024, 2, 128, 0, 0, 0, out) == 1      # N < 1
+    assert lib.mocap_lbcp_partition_dp(1024, 2, 128, 4, 5, 0, out) == 1      # model
+    assert lib.mocap_lbcp_partition_dp(1024, 2, 128, 4, 0, -1, out) == 1     # weight
+    assert lib.mocap_lbcp_partition_dp(1024, 9, 128, 4, 0, 0, out) == 1      # M g > S
+    assert lib.mocap_lbcp_partition_dp(1 << 30, 32, 1, 4, 0, 0, out) == 3    # too large
+    assert lib.mocap_lbcp_partition_dp(131072, 32, 128, 16, 0, 0, out) == 0

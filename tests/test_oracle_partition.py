@@ -6,6 +6,7 @@ cost model by its algebra and by brute-force pair counting, the clamps by
 invariants, and the closed form at the boundaries where sqrt(i/M) is rational.
 """
 
+import functools
 import math
 import os
 import random
@@ -173,3 +174,96 @@ def test_golden_boundaries():
     assert len(rows) >= 8
     for (s, m, g, mode), b in rows:
         assert P.boundaries(s, m, g, mode) == b
+
+
+# ---------------------------------------------------------------- Algorithm 1 DP --
+def _compositions(total, parts):
+    """All ways to write `total` units as `parts` positive sizes."""
+    if parts == 1:
+        yield (total,)
+        return
+    for first in range(1, total - parts + 2):
+        for rest in _compositions(total - first, parts - 1):
+            yield (first,) + rest
+
+
+@functools.lru_cache(maxsize=None)
+def _brute_cost(k, s, model, gemm):
+    """Chunk cost from counted (query, key) pairs, independent of the oracle.
+
+    Causal: twice c (p + c/2) = twice the causal pair count minus c (the
+    pair count is c p + c (c + 1) / 2).  Eq. 1: twice c (p + c), every key up
+    to the chunk end for every query of the chunk.  Plus gemm * c."""
+    queries = range(s, s + k)
+    if model == P.COST_CAUSAL:
+        pairs = sum(1 for t in queries for j in range(s + k) if j <= t)
+        attn = 2 * pairs - k
+    else:
+        attn = 2 * sum(1 for t in queries for j in range(s + k))
+    return attn + gemm * k
+
+
+def _chunk_costs(sizes, model, gemm):
+    s, out = 0, []
+    for k in sizes:
+        out.append(_brute_cost(k, s, model, gemm))
+        s += k
+    return out
+
+
+@pytest.mark.parametrize("model", [P.COST_CAUSAL, P.COST_EQ1])
+def test_evaluate_chunk_counts_pairs(model):
+    for k in range(1, 9):
+        for s in range(0, 9):
+            for gemm in (0, 5):
+                assert P.evaluate_chunk(k, s, model, gemm) == _brute_cost(k, s, model, gemm)
+
+
+@pytest.mark.parametrize("model", [P.COST_CAUSAL, P.COST_EQ1])
+@pytest.mark.parametrize("gemm", [0, 3, 40])
+def test_dp_single_stage_minimises_total_cost(model, gemm):
+    # N = 1: the objective is t_sum alone, which decomposes over chunks, so the
+    # suffix recursion is exact: the DP total equals the brute-force minimum.
+    for units in range(1, 11):
+        for m in range(1, min(units, 5) + 1):
+            b = P.dp_boundaries(units * 128, m, 128, 1, model, gemm)
+            sizes = [(b[i + 1] - b[i]) // 128 for i in range(m)]
+            best = min(sum(_chunk_costs(c, model, gemm)) for c in _compositions(units, m))
+            assert sum(_chunk_costs(sizes, model, gemm)) == best
+
+
+@pytest.mark.parametrize("model", [P.COST_CAUSAL, P.COST_EQ1])
+@pytest.mark.parametrize("gemm", [0, 7])
+def test_dp_many_stages_reaches_the_minimax_chunk(model, gemm):
+    # (N - 1) larger than any possible t_sum: comparisons are lexicographic in
+    # (t_max, t_sum), every kept suffix has the least t_max, and max(t, .) is
+    # monotone, so the DP's largest chunk cost is the brute-force minimax.
+    for units in range(1, 12):
+        for m in range(1, min(units, 5) + 1):
+            n_stages = 10 ** 9
+            b = P.dp_boundaries(units * 128, m, 128, n_stages, model, gemm)
+            sizes = [(b[i + 1] - b[i]) // 128 for i in range(m)]
+            best = min(max(_chunk_costs(c, model, gemm)) for c in _compositions(units, m))
+            assert max(_chunk_costs(sizes, model, gemm)) == best
+
+
+def test_dp_invariants_and_remainder():
+    for s, m, n in [(1000, 3, 4), (32768, 16, 16), (640, 5, 2), (100000, 9, 16)]:
+        b = P.dp_boundaries(s, m, 128 if s != 100000 else 64, n)
+        g = 128 if s != 100000 else 64
+        _check_invariants(b, s, m, g)
+
+
+def test_dp_causal_cost_telescopes():
+    # with the causal model and no GEMM term every partition has t_sum = U^2
+    for units, m in [(7, 3), (12, 4), (20, 6)]:
+        b = P.dp_boundaries(units * 128, m, 128, 8)
+        sizes = [(b[i + 1] - b[i]) // 128 for i in range(m)]
+        assert sum(_chunk_costs(sizes, P.COST_CAUSAL, 0)) == units * units
+
+
+def test_dp_beats_closed_form_objective_on_workload_shapes():
+    for s, m in [(32768, 16), (8192, 8)]:
+        dp = P.dp_boundaries(s, m, 128, 16)
+        cf = P.boundaries(s, m, 128)
+        assert P.dp_objective(dp, 128, 16) <= P.dp_objective(cf, 128, 16)
