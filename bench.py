@@ -44,6 +44,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-uniform", action="store_true",
+                    help="skip the uniform-boundary per-chunk latency comparison")
     ap.add_argument("--cpu-rows-per-chunk", type=int, default=2)
     ap.add_argument("--case", default=None,
                     help="profiling case 'prefix,len,Hq,Hkv,d': one chunk attention launch "
@@ -416,6 +418,8 @@ def ours_arm(args, rank, world, local):
         "gpu_launches": args.steps * sum(1 + len(st) for st in steps_plan),
     }
 
+    if pf.mode == workloads.MODE_LBCP and pf.single and not args.no_uniform:
+        line["uniform_boundaries"] = measure_uniform(w, q, k, v, dev, stream)
     if not args.no_e2e:
         line["e2e"] = measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -430,6 +434,28 @@ def ours_arm(args, rank, world, local):
     if rank == 0:
         print(json.dumps(line), flush=True)
     return 0
+
+
+def measure_uniform(w, q, k, v, dev, stream, reps=3):
+    """Per-chunk attention latency with uniform boundaries (outside the timed
+    region): without latency-balanced chunks the late chunks dominate."""
+    import torch
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    from paper_2606_22968_gb300 import workloads
+    pu = ChunkedPrefill(w, dev, mode=workloads.MODE_UNIFORM)
+    n = len(pu.steps())
+    times = []
+    for _ in range(reps):
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n)]
+        pu.run(q, k, v, stream, ev)
+        torch.cuda.synchronize(dev)
+        times.append([ev[c][1].elapsed_time(ev[c][2]) for c in range(n)])
+    per_chunk = [statistics.median(t[c] for t in times) for c in range(n)]
+    del pu
+    return {"per_chunk_attn_ms": {"min": min(per_chunk), "max": max(per_chunk),
+                                  "max_over_min": max(per_chunk) / min(per_chunk),
+                                  "cv": statistics.pstdev(per_chunk) / statistics.mean(per_chunk)},
+            "attn_ms_per_step": sum(per_chunk)}
 
 
 def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):

@@ -12,7 +12,8 @@
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kUnroll = 4;
+constexpr int kUnroll = 4;        // 16-byte vectors in flight per thread
+constexpr int kCtasPerSm = 32;    // grid cap; the loop strides over the rest
 
 __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
   uint4 v;
@@ -82,7 +83,7 @@ extern "C" mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk
   const int64_t n = len * row_elems / 8;  // 16-byte vectors per tensor
   const int64_t dst_off = offset * row_elems / 8;
   const int64_t want = (2 * n + kThreads * kUnroll - 1) / (kThreads * kUnroll);
-  const int64_t cap = static_cast<int64_t>(sm_count()) * 8;
+  const int64_t cap = static_cast<int64_t>(sm_count()) * kCtasPerSm;
   const int blocks = static_cast<int>(std::max<int64_t>(1, std::min(want, cap)));
   kv_append_kernel<<<blocks, kThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
       static_cast<const uint4 *>(k_chunk), static_cast<const uint4 *>(v_chunk),
