@@ -44,6 +44,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-graph", action="store_true",
+                    help="skip the CUDA-graph replay measurement")
     ap.add_argument("--no-uniform", action="store_true",
                     help="skip the uniform-boundary per-chunk latency comparison")
     ap.add_argument("--cpu-rows-per-chunk", type=int, default=2)
@@ -418,6 +420,9 @@ def ours_arm(args, rank, world, local):
         "gpu_launches": args.steps * sum(1 + len(st) for st in steps_plan),
     }
 
+    if not args.no_graph:
+        line["graph_replay"] = measure_graph(args, pf, q, k, v, dev, stream, total_flops,
+                                             w.total_tokens, world)
     if pf.mode == workloads.MODE_LBCP and pf.single and not args.no_uniform:
         line["uniform_boundaries"] = measure_uniform(w, q, k, v, dev, stream)
     if not args.no_e2e:
@@ -434,6 +439,32 @@ def ours_arm(args, rank, world, local):
     if rank == 0:
         print(json.dumps(line), flush=True)
     return 0
+
+
+def measure_graph(args, pf, q, k, v, dev, stream, total_flops, tokens, world):
+    """The same step replayed as one captured CUDA graph (every append,
+    attention launch and combine of the prompt): no per-launch host work and
+    no gaps between launches.  Timed like the main region, after it."""
+    import torch
+    graph = pf.capture(q, k, v)
+    for _ in range(args.warmup):
+        pf.partition()
+        graph.replay()
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        pf.partition()
+        graph.replay()
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world, dev)
+    del graph
+    return {"ms_per_step": ms, "value": replica_throughput(total_flops, ms, world) / 1e12,
+            "unit": "TFLOP/s", "prefill_tokens_per_s": replica_throughput(tokens, ms, world)}
 
 
 def measure_uniform(w, q, k, v, dev, stream, reps=3):

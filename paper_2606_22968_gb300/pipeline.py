@@ -167,3 +167,20 @@ class ChunkedPrefill:
                         host_lse2d[:, rows].copy_(lse2d[:, rows], non_blocking=True)
         compute.wait_stream(d2h)
         compute.wait_stream(h2d)
+
+    # -- CUDA graph ------------------------------------------------------------------
+    def capture(self, q, k, v, stream=None):
+        """Record the whole prompt's launch sequence (every append, attention
+        launch and split-KV combine) into one CUDA graph.  Replaying it runs
+        the same kernels on the same buffers without per-launch host work or
+        gaps between launches.  Call ``run`` once first so one-time set-up
+        (device attributes, symbol lookups) happens outside the capture; the
+        graph holds the current boundaries and buffer addresses."""
+        graph = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream(self.device) if stream is None else stream
+        side.wait_stream(torch.cuda.current_stream(self.device))
+        with torch.cuda.stream(side):
+            with torch.cuda.graph(graph, stream=side):
+                self.run(q, k, v, side)
+        torch.cuda.current_stream(self.device).wait_stream(side)
+        return graph

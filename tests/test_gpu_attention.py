@@ -319,3 +319,28 @@ def test_run_from_host_matches_device_run(m, index):
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == 0
     assert torch.equal(ho, out_ref.cpu()) and torch.equal(hl, lse_ref.cpu())
+
+
+@pytest.mark.parametrize("index", [1, 3, 5])
+def test_graph_replay_matches_eager_run(m, index):
+    """The whole prompt captured in one CUDA graph gives bitwise the eager results."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(index)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev)
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    out_ref, lse_ref = pf.out.clone(), pf.lse.clone()
+    graph = pf.capture(q, k, v)
+    for _ in range(2):
+        pf.out.fill_(float("nan"))
+        pf.lse.fill_(float("nan"))
+        pf.k_cache.fill_(float("nan"))
+        pf.v_cache.fill_(float("nan"))
+        graph.replay()
+        torch.cuda.synchronize()
+        assert m.mocap_last_device_status() == 0
+        assert torch.equal(pf.out, out_ref) and torch.equal(pf.lse, lse_ref)
+        assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
