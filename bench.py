@@ -46,6 +46,10 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-graph", action="store_true",
                     help="skip the CUDA-graph replay measurement")
+    ap.add_argument("--no-projection", action="store_true",
+                    help="skip the QKV projection + RoPE + append measurement")
+    ap.add_argument("--hidden", type=int, default=8192,
+                    help="hidden size for the projection measurement (Llama-3-70B: 8192)")
     ap.add_argument("--no-uniform", action="store_true",
                     help="skip the uniform-boundary per-chunk latency comparison")
     ap.add_argument("--cpu-rows-per-chunk", type=int, default=2)
@@ -423,6 +427,9 @@ def ours_arm(args, rank, world, local):
     if not args.no_graph:
         line["graph_replay"] = measure_graph(args, pf, q, k, v, dev, stream, total_flops,
                                              w.total_tokens, world)
+    if pf.single and not args.no_projection:
+        line["qkv_projection"] = measure_projection(args, m, w, pf, q, dev, stream, total_flops,
+                                                    peak)
     if pf.mode == workloads.MODE_LBCP and pf.single and not args.no_uniform:
         line["uniform_boundaries"] = measure_uniform(w, q, k, v, dev, stream)
     if not args.no_e2e:
@@ -465,6 +472,55 @@ def measure_graph(args, pf, q, k, v, dev, stream, total_flops, tokens, world):
     del graph
     return {"ms_per_step": ms, "value": replica_throughput(total_flops, ms, world) / 1e12,
             "unit": "TFLOP/s", "prefill_tokens_per_s": replica_throughput(tokens, ms, world)}
+
+
+def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
+    """Eq. 1's GEMM term for the same chunks: per chunk, the QKV projection of
+    its hidden states (random-init weights of the model's shape) with RoPE and
+    the KV append fused; then the whole chunk stage (projection, attention).
+    Timed outside the main region, CUDA events, K steps after W warm-ups."""
+    import torch
+    hidden = args.hidden
+    n_out = (w.n_q_heads + 2 * w.n_kv_heads) * w.head_dim
+    gen = torch.Generator(device=dev).manual_seed(w.seed + 1000)
+    x = torch.randn((w.total_tokens, hidden), generator=gen, device=dev, dtype=torch.bfloat16)
+    wq = (torch.randn((n_out, hidden), generator=gen, device=dev) / hidden ** 0.5).bfloat16()
+    qbuf = torch.empty_like(q)
+    b = pf.bounds[0]
+    gemm_flops = 2 * w.total_tokens * hidden * n_out
+
+    def project(c):
+        m.mocap_qkv_rope_append(x[b[c]:b[c + 1]], wq, qbuf[b[c]:b[c + 1]], pf.k_cache,
+                                pf.v_cache, b[c], stream=stream)
+
+    def attend(c):
+        m.mocap_chunk_attn(qbuf[b[c]:b[c + 1]], pf.k_cache, pf.v_cache, b[c],
+                           pf.out[b[c]:b[c + 1]], pf.chunk_lse(c), w.scale,
+                           workspace=pf.workspace, stream=stream)
+
+    def timed(fn):
+        for _ in range(args.warmup):
+            fn()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / args.steps
+
+    n = len(b) - 1
+    ms_gemm = timed(lambda: [project(c) for c in range(n)])
+    ms_stage = timed(lambda: [(project(c), attend(c)) for c in range(n)])
+    if m.mocap_last_device_status() != m.MOCAP_OK:
+        raise RuntimeError("device wait expired in the projection measurement")
+    gemm_tf = gemm_flops / (ms_gemm * 1e-3) / 1e12
+    return {"hidden": hidden, "n_out": n_out, "flop_per_step": gemm_flops,
+            "ms_per_step": ms_gemm, "tflops": gemm_tf, "frac_of_peak": gemm_tf / peak,
+            "stage_ms_per_step": ms_stage,
+            "stage_tflops": (gemm_flops + attn_flops) / (ms_stage * 1e-3) / 1e12,
+            "stage_tokens_per_s": w.total_tokens / (ms_stage * 1e-3)}
 
 
 def measure_uniform(w, q, k, v, dev, stream, reps=3):

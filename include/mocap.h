@@ -13,6 +13,7 @@
  *   mocap_lbcp_partition      chunk boundaries (host, exact integers)
  *   mocap_lbcp_partition_dp   boundaries from Algorithm 1's stage-1 DP (host)
  *   mocap_kv_append           chunk K/V -> contiguous bf16 KV cache (device)
+ *   mocap_qkv_rope_append     QKV projection + RoPE + KV append (device GEMM)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
  *   mocap_last_device_status  bounded-wait timeouts reported by the kernels
@@ -136,6 +137,34 @@ mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk,
                              int64_t cache_capacity, int64_t offset, int64_t len,
                              int32_t n_kv_heads, int32_t head_dim,
                              mocap_stream_t stream);
+
+/*
+ * mocap_qkv_rope_append -- a chunk's QKV projection, rotary embedding and KV
+ * append in one kernel.
+ *
+ * Sec. 3.2 / Eq. 1: each chunk also pays GEMM work that grows with its
+ * length alone; the QKV projection is the one attention depends on.  For the
+ * chunk's hidden states X (bf16 [len, hidden]) and the packed weights W (bf16
+ * [(Hq + 2 Hkv) d, hidden]; rows 0 .. Hq d - 1 produce Q, the next Hkv d
+ * produce K, the last Hkv d produce V):
+ *   [Q | K | V] = X W^T                                   (fp32 accumulate)
+ *   Q and K rotated at positions offset + r (rotate-half RoPE: dims j and
+ *   j + d/2 of each head turn by (offset + r) * rope_theta^(-2j/d))
+ *   q_out[r]                 <- Q (bf16 [len, Hq, d])
+ *   k_cache[offset + r], v_cache[offset + r] <- K, V (bf16 [capacity, Hkv, d])
+ * so the attention of the same chunk can run right after it.  Cache rows
+ * outside [offset, offset + len) are not touched.
+ *
+ * Requirements: head_dim in {64, 128} and (Hq + 2 Hkv) * head_dim a multiple
+ * of 256 (else MOCAP_EUNSUPPORTED); hidden a multiple of 8; rope_theta > 1;
+ * 16-byte aligned pointers; offset + len <= cache_capacity.  len == 0 is a
+ * no-op.  Persistent tcgen05 GEMM: 128 x 256 output tiles, K steps of 64.
+ */
+mocap_status mocap_qkv_rope_append(const void *x, const void *w_qkv, void *q_out,
+                                   void *k_cache, void *v_cache, int64_t cache_capacity,
+                                   int64_t offset, int64_t len, int32_t hidden,
+                                   int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
+                                   float rope_theta, mocap_stream_t stream);
 
 /*
  * mocap_chunk_attn -- attention of one chunk against its KV prefix.

@@ -16,9 +16,11 @@ Contents
                earlier chunks plus itself), the KV-append definition
                (Sec. 2.2 / 3.1: KV of earlier chunks stays live) and the
                split-KV log-sum-exp combine.
+``projection`` The QKV projection of a chunk (Sec. 3.2 / Eq. 1's GEMM term)
+               with the rotary position embedding applied to Q and K.
 
 Every function is pinned by ``tests/test_oracle_*.py`` against brute force,
 closed forms and invariants (nothing in this package is "parity unpinned").
 """
 
-from . import attention, partition  # noqa: F401
+from . import attention, partition, projection  # noqa: F401

@@ -83,6 +83,20 @@ def mocap_kv_append(k_chunk, v_chunk, k_cache, v_cache, offset: int, stream=None
                                        _stream(stream)), "mocap_kv_append")
 
 
+def mocap_qkv_rope_append(x, w_qkv, q_out, k_cache, v_cache, offset: int,
+                          rope_theta: float = 500000.0, stream=None):
+    """[Q|K|V] = x w_qkv^T, RoPE on Q/K at positions offset + r, Q -> q_out,
+    K/V -> cache rows [offset, offset + len).  x [len, hidden], w_qkv
+    [(Hq + 2 Hkv) d, hidden], q_out [len, Hq, d], caches [cap, Hkv, d] (bf16)."""
+    length, hidden = x.shape
+    _, n_q, d = q_out.shape
+    n_kv = k_cache.shape[1]
+    _check(_lib.load().mocap_qkv_rope_append(_ptr(x), _ptr(w_qkv), _ptr(q_out), _ptr(k_cache),
+                                             _ptr(v_cache), k_cache.shape[0], offset, length,
+                                             hidden, n_q, n_kv, d, rope_theta, _stream(stream)),
+           "mocap_qkv_rope_append")
+
+
 def mocap_chunk_attn_workspace_size(prefix: int, length: int, n_q_heads: int, n_kv_heads: int,
                                     head_dim: int) -> int:
     """Bytes of scratch that let mocap_chunk_attn split the key range (0 = no split)."""

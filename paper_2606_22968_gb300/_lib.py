@@ -23,6 +23,8 @@ SIGNATURES = {
     "mocap_lbcp_partition_dp": (c_i32, [c_i64, c_i32, c_i32, c_i32, c_i32, c_i64,
                                         ctypes.POINTER(c_i64)]),
     "mocap_kv_append": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32, c_i32, c_vp]),
+    "mocap_qkv_rope_append": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32,
+                                      c_i32, c_i32, c_i32, c_f32, c_vp]),
     "mocap_chunk_attn": (c_i32, [c_vp, c_vp, c_vp, c_i64, c_i64, c_i32, c_i32, c_i32, c_f32,
                                  c_vp, c_vp, c_vp, c_sz, c_vp]),
     "mocap_chunk_attn_workspace_size": (c_sz, [c_i64, c_i64, c_i32, c_i32, c_i32]),

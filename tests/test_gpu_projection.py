@@ -1,0 +1,78 @@
+"""GPU parity of the fused QKV projection + RoPE + KV append against the
+float64 oracle (every element), with cache rows outside the chunk kept."""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import projection as R
+from tests.parity_utils import f64
+
+pytestmark = pytest.mark.gpu
+
+TOL_MAX, TOL_MEAN = 2e-2, 2e-3
+
+
+@pytest.fixture(scope="module")
+def m():
+    import paper_2606_22968_gb300 as mod
+    mod._lib.load()
+    return mod
+
+
+CASES = [
+    # (len, hidden, Hq, Hkv, d, offset, theta)
+    (300, 1024, 4, 2, 128, 0, 500000.0),
+    (1, 256, 4, 2, 128, 77, 500000.0),
+    (129, 200, 8, 8, 64, 1000, 10000.0),      # hidden not a multiple of 64
+    (1000, 512, 2, 1, 128, 130000, 500000.0),  # large positions
+    (512, 2048, 16, 2, 128, 4096, 500000.0),   # GQA 8:1, several n tiles
+]
+
+
+@pytest.mark.parametrize("length,hidden,hq,hkv,d,offset,theta", CASES)
+def test_qkv_rope_append_matches_oracle(m, length, hidden, hq, hkv, d, offset, theta):
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(length + hidden + offset)
+    x = torch.randn((length, hidden), generator=gen, device=dev).bfloat16()
+    n_out = (hq + 2 * hkv) * d
+    w = (torch.randn((n_out, hidden), generator=gen, device=dev) / math.sqrt(hidden)).bfloat16()
+    cap = offset + length + 5
+    sentinel = torch.randint(-30000, 30000, (cap, hkv, d), generator=gen, device=dev,
+                             dtype=torch.int16)
+    kc = sentinel.clone().view(torch.bfloat16)
+    vc = (sentinel ^ 0x1234).view(torch.bfloat16)
+    k0, v0 = kc.clone(), vc.clone()
+    q = torch.full((length, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    m.mocap_qkv_rope_append(x, w, q, kc, vc, offset, rope_theta=theta)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    q_ref, k_ref, v_ref = R.qkv_rope(f64(x), f64(w), hq, hkv, d, offset, theta)
+    for got, ref, name in [(q, q_ref, "Q"), (kc[offset:offset + length], k_ref, "K"),
+                           (vc[offset:offset + length], v_ref, "V")]:
+        err = np.abs(got.float().cpu().numpy() - ref)
+        assert err.max() <= TOL_MAX and err.mean() <= TOL_MEAN, (name, err.max(), err.mean())
+    # rows outside the chunk keep their bytes (compared as bit patterns: the
+    # sentinels include NaN encodings)
+    bits = lambda t: t.view(torch.int16)  # noqa: E731
+    for got, ref in [(kc, k0), (vc, v0)]:
+        assert torch.equal(bits(got[:offset]), bits(ref[:offset]))
+        assert torch.equal(bits(got[offset + length:]), bits(ref[offset + length:]))
+
+
+def test_qkv_rope_rejects_bad_shapes(m):
+    dev = torch.device("cuda")
+    x = torch.zeros((10, 128), device=dev, dtype=torch.bfloat16)
+    w = torch.zeros((3 * 64 * 2, 128), device=dev, dtype=torch.bfloat16)  # (2+2*2)*64=384: not /256
+    q = torch.zeros((10, 2, 64), device=dev, dtype=torch.bfloat16)
+    kc = torch.zeros((20, 2, 64), device=dev, dtype=torch.bfloat16)
+    with pytest.raises(m.MocapError):
+        m.mocap_qkv_rope_append(x, w, q, kc, kc.clone(), 0)
+    x2 = torch.zeros((10, 128), device=dev, dtype=torch.bfloat16)
+    w2 = torch.zeros((4 * 128, 128), device=dev, dtype=torch.bfloat16)
+    q2 = torch.zeros((10, 2, 128), device=dev, dtype=torch.bfloat16)
+    kc2 = torch.zeros((12, 1, 128), device=dev, dtype=torch.bfloat16)
+    with pytest.raises(m.MocapError):   # offset + len past the cache
+        m.mocap_qkv_rope_append(x2, w2, q2, kc2, kc2.clone(), 5)
