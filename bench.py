@@ -50,6 +50,8 @@ def parse_args():
                     help="skip the QKV projection + RoPE + append measurement")
     ap.add_argument("--hidden", type=int, default=8192,
                     help="hidden size for the projection measurement (Llama-3-70B: 8192)")
+    ap.add_argument("--no-last-row", action="store_true",
+                    help="skip the last-row-only attention measurement")
     ap.add_argument("--no-uniform", action="store_true",
                     help="skip the uniform-boundary per-chunk latency comparison")
     ap.add_argument("--cpu-rows-per-chunk", type=int, default=2)
@@ -430,6 +432,8 @@ def ours_arm(args, rank, world, local):
     if pf.single and not args.no_projection:
         line["qkv_projection"] = measure_projection(args, m, w, pf, q, dev, stream, total_flops,
                                                     peak)
+    if not args.no_last_row:
+        line["last_row"] = measure_last_row(args, m, w, pf, q, dev, stream, hbm)
     if pf.mode == workloads.MODE_LBCP and pf.single and not args.no_uniform:
         line["uniform_boundaries"] = measure_uniform(w, q, k, v, dev, stream)
     if not args.no_e2e:
@@ -521,6 +525,42 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
             "stage_ms_per_step": ms_stage,
             "stage_tflops": (gemm_flops + attn_flops) / (ms_stage * 1e-3) / 1e12,
             "stage_tokens_per_s": w.total_tokens / (ms_stage * 1e-3)}
+
+
+def measure_last_row(args, m, w, pf, q, dev, stream, hbm):
+    """The one output token of a prefill-only request needs the final layer's
+    attention for the last prompt row only: each request's last row against
+    all its keys (memory-bound; roofline = HBM).  Uses the caches the timed
+    run filled."""
+    import torch
+    n = len(w.seq_lens)
+    rows = [pf.cu[r] for r in range(n)]
+    lens = list(w.seq_lens)
+    q_last = torch.stack([q[pf.cu[r] + lens[r] - 1] for r in range(n)]).contiguous()
+    out = torch.empty_like(q_last)
+    lse = torch.empty((w.n_q_heads, n), device=dev, dtype=torch.float32)
+    ws = torch.empty((max(16, m.mocap_last_row_attn_workspace_size(lens, w.n_q_heads,
+                                                                   w.head_dim)),),
+                     device=dev, dtype=torch.uint8)
+    for _ in range(args.warmup):
+        m.mocap_last_row_attn(q_last, pf.k_cache, pf.v_cache, rows, lens, out, lse, w.scale,
+                              workspace=ws, stream=stream)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 20
+    e0.record(stream)
+    for _ in range(reps):
+        m.mocap_last_row_attn(q_last, pf.k_cache, pf.v_cache, rows, lens, out, lse, w.scale,
+                              workspace=ws, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    if m.mocap_last_device_status() != m.MOCAP_OK:
+        raise RuntimeError("device wait expired in the last-row measurement")
+    us = e0.elapsed_time(e1) / reps * 1e3
+    kv_bytes = sum(lens) * w.n_kv_heads * w.head_dim * 2 * 2
+    gbs = kv_bytes / (us * 1e-6) / 1e9
+    return {"us_per_call": us, "kv_bytes": kv_bytes, "gb_per_s": gbs, "frac_of_hbm": gbs / hbm,
+            "requests": n, "note": "back-to-back calls; K/V may be partly L2-resident"}
 
 
 def measure_uniform(w, q, k, v, dev, stream, reps=3):

@@ -16,6 +16,7 @@
  *   mocap_qkv_rope_append     QKV projection + RoPE + KV append (device GEMM)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
+ *   mocap_last_row_attn       each request's last row only (prefill-only output)
  *   mocap_last_device_status  bounded-wait timeouts reported by the kernels
  *   mocap_selftest_bounded_wait  drives that timeout path on purpose (tests)
  *   mocap_status_string       text for a status code
@@ -298,6 +299,34 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
                                      int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
                                      float scale, void *out, float *lse,
                                      mocap_stream_t stream);
+
+/*
+ * mocap_last_row_attn -- attention of each request's last prompt row only.
+ *
+ * Sec. 2.1: a prefill-only request emits a single token, so its final layer
+ * needs the attention output of the last row alone: for request r and query
+ * head h, the row at position kv_len[r] - 1 attends to every key of the
+ * request (keys 0 .. kv_len[r] - 1), with the same definition as
+ * mocap_chunk_attn.  This is memory-bound (each K/V byte serves only the
+ * n_q_heads / n_kv_heads heads of its group), so a dedicated kernel streams
+ * K/V through TMA and splits each request's keys into ranges of 2048 whose
+ * fp32 partials are merged like split-KV.
+ *
+ *   q_last    bf16 [n_req, Hq, d]: the last row's queries of each request
+ *   k_cache,  bf16 [kv_rows_total, Hkv, d]: request r's keys are rows
+ *   v_cache   kv_row[r] .. kv_row[r] + kv_len[r] - 1 (rows past them unread)
+ *   kv_row, kv_len  HOST arrays of n_req int64 (kv_len[r] >= 1)
+ *   out       bf16 [n_req, Hq, d];  lse fp32 [Hq, n_req]
+ *   workspace at least mocap_last_row_attn_workspace_size(...) bytes
+ * 1 <= n_req <= 64; Hq / Hkv <= 16; head_dim in {64, 128}.
+ */
+size_t mocap_last_row_attn_workspace_size(const int64_t *kv_len, int32_t n_req,
+                                          int32_t n_q_heads, int32_t head_dim);
+mocap_status mocap_last_row_attn(const void *q_last, const void *k_cache, const void *v_cache,
+                                 const int64_t *kv_row, const int64_t *kv_len, int32_t n_req,
+                                 int64_t kv_rows_total, int32_t n_q_heads, int32_t n_kv_heads,
+                                 int32_t head_dim, float scale, void *out, float *lse,
+                                 void *workspace, size_t workspace_bytes, mocap_stream_t stream);
 
 /*
  * mocap_last_device_status -- synchronises `stream`, then reads and clears

@@ -135,6 +135,32 @@ def mocap_chunk_attn_varlen(q, k_cache, v_cache, items: Sequence[tuple], out, ls
            "mocap_chunk_attn_varlen")
 
 
+def mocap_last_row_attn_workspace_size(kv_len, n_q_heads: int, head_dim: int) -> int:
+    arr = (ctypes.c_int64 * len(kv_len))(*kv_len)
+    return int(_lib.load().mocap_last_row_attn_workspace_size(arr, len(kv_len), n_q_heads,
+                                                              head_dim))
+
+
+def mocap_last_row_attn(q_last, k_cache, v_cache, kv_row, kv_len, out, lse, scale: float,
+                        workspace=None, stream=None):
+    """Each request's last row against all its keys.  q_last/out [n_req, Hq, d],
+    caches [rows, Hkv, d], lse [Hq, n_req]; kv_row/kv_len: host sequences."""
+    import torch
+    n_req, n_q, d = q_last.shape
+    n_kv = k_cache.shape[1]
+    rows = (ctypes.c_int64 * n_req)(*kv_row)
+    lens = (ctypes.c_int64 * n_req)(*kv_len)
+    need = mocap_last_row_attn_workspace_size(kv_len, n_q, d)
+    if workspace is None:
+        workspace = torch.empty((max(need, 16),), device=q_last.device, dtype=torch.uint8)
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(_lib.load().mocap_last_row_attn(_ptr(q_last), _ptr(k_cache), _ptr(v_cache), rows, lens,
+                                           n_req, k_cache.shape[0], n_q, n_kv, d, scale,
+                                           _ptr(out), _ptr(lse), _ptr(workspace), ws_bytes,
+                                           _stream(stream)),
+           "mocap_last_row_attn")
+
+
 def mocap_last_device_status(stream=None) -> int:
     return int(_lib.load().mocap_last_device_status(_stream(stream)))
 

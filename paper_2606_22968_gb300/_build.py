@@ -19,7 +19,8 @@ INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmocap.so")
 
-SOURCES = ["lbcp.cpp", "status.cu", "kv_append.cu", "chunk_attn.cu", "qkv_rope.cu"]
+SOURCES = ["lbcp.cpp", "status.cu", "kv_append.cu", "chunk_attn.cu", "qkv_rope.cu",
+           "last_row_attn.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr",
          "-I" + INCLUDE, "-I" + CSRC]

@@ -33,6 +33,10 @@ SIGNATURES = {
     "mocap_chunk_attn_varlen": (c_i32, [c_vp, c_vp, c_vp, ctypes.POINTER(VarlenItem), c_i32,
                                         c_i64, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp, c_vp,
                                         c_vp]),
+    "mocap_last_row_attn_workspace_size": (c_sz, [ctypes.POINTER(c_i64), c_i32, c_i32, c_i32]),
+    "mocap_last_row_attn": (c_i32, [c_vp, c_vp, c_vp, ctypes.POINTER(c_i64), ctypes.POINTER(c_i64),
+                                    c_i32, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp, c_vp, c_vp,
+                                    c_sz, c_vp]),
     "mocap_last_device_status": (c_i32, [c_vp]),
     "mocap_selftest_bounded_wait": (c_i32, [ctypes.c_uint32, c_vp]),
     "mocap_status_string": (ctypes.c_char_p, [c_i32]),

@@ -844,6 +844,23 @@ bool pointers_ok(const void *q, const void *k, const void *v, const void *out, c
 constexpr int64_t kMaxRows = 0x7fffffffLL;
 
 }  // namespace
+
+// Merge split partials (o_part [splits, len, Hq, d], lse_part [splits, Hq,
+// len]) into bf16 out [len, Hq, d] and fp32 lse [Hq, lse_stride].
+mocap_status launch_attn_combine(const float *o_part, const float *lse_part, int splits,
+                                 int64_t len, int n_q_heads, int head_dim, void *out, float *lse,
+                                 int64_t lse_stride, cudaStream_t stream) {
+  const int64_t warps = len * n_q_heads;
+  const unsigned blocks = static_cast<unsigned>((warps + 7) / 8);
+  auto *o = static_cast<__nv_bfloat16 *>(out);
+  if (head_dim == 128)
+    attn_combine_kernel<128><<<blocks, 256, 0, stream>>>(o_part, lse_part, splits, len, n_q_heads,
+                                                         o, lse, lse_stride);
+  else
+    attn_combine_kernel<64><<<blocks, 256, 0, stream>>>(o_part, lse_part, splits, len, n_q_heads,
+                                                        o, lse, lse_stride);
+  return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+}
 }  // namespace mocap
 
 using mocap::HostItem;
