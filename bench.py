@@ -540,7 +540,7 @@ def measure_last_row(args, m, w, pf, q, dev, stream, hbm):
     out = torch.empty_like(q_last)
     lse = torch.empty((w.n_q_heads, n), device=dev, dtype=torch.float32)
     ws = torch.empty((max(16, m.mocap_last_row_attn_workspace_size(lens, w.n_q_heads,
-                                                                   w.head_dim)),),
+                                                                   w.n_kv_heads, w.head_dim)),),
                      device=dev, dtype=torch.uint8)
     for _ in range(args.warmup):
         m.mocap_last_row_attn(q_last, pf.k_cache, pf.v_cache, rows, lens, out, lse, w.scale,

@@ -309,8 +309,10 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
  * request (keys 0 .. kv_len[r] - 1), with the same definition as
  * mocap_chunk_attn.  This is memory-bound (each K/V byte serves only the
  * n_q_heads / n_kv_heads heads of its group), so a dedicated kernel streams
- * K/V through TMA and splits each request's keys into ranges of 2048 whose
- * fp32 partials are merged like split-KV.
+ * K/V tiles through TMA, lets the tensor core form the small products in
+ * transposed form (keys, then dimensions, on the 128 TMEM lanes), and splits
+ * the requests' keys into ranges (about two CTAs per SM in total) whose fp32
+ * partials are merged like split-KV.
  *
  *   q_last    bf16 [n_req, Hq, d]: the last row's queries of each request
  *   k_cache,  bf16 [kv_rows_total, Hkv, d]: request r's keys are rows
@@ -321,7 +323,8 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
  * 1 <= n_req <= 64; Hq / Hkv <= 16; head_dim in {64, 128}.
  */
 size_t mocap_last_row_attn_workspace_size(const int64_t *kv_len, int32_t n_req,
-                                          int32_t n_q_heads, int32_t head_dim);
+                                          int32_t n_q_heads, int32_t n_kv_heads,
+                                          int32_t head_dim);
 mocap_status mocap_last_row_attn(const void *q_last, const void *k_cache, const void *v_cache,
                                  const int64_t *kv_row, const int64_t *kv_len, int32_t n_req,
                                  int64_t kv_rows_total, int32_t n_q_heads, int32_t n_kv_heads,

@@ -135,10 +135,11 @@ def mocap_chunk_attn_varlen(q, k_cache, v_cache, items: Sequence[tuple], out, ls
            "mocap_chunk_attn_varlen")
 
 
-def mocap_last_row_attn_workspace_size(kv_len, n_q_heads: int, head_dim: int) -> int:
+def mocap_last_row_attn_workspace_size(kv_len, n_q_heads: int, n_kv_heads: int,
+                                       head_dim: int) -> int:
     arr = (ctypes.c_int64 * len(kv_len))(*kv_len)
     return int(_lib.load().mocap_last_row_attn_workspace_size(arr, len(kv_len), n_q_heads,
-                                                              head_dim))
+                                                              n_kv_heads, head_dim))
 
 
 def mocap_last_row_attn(q_last, k_cache, v_cache, kv_row, kv_len, out, lse, scale: float,
@@ -150,7 +151,7 @@ def mocap_last_row_attn(q_last, k_cache, v_cache, kv_row, kv_len, out, lse, scal
     n_kv = k_cache.shape[1]
     rows = (ctypes.c_int64 * n_req)(*kv_row)
     lens = (ctypes.c_int64 * n_req)(*kv_len)
-    need = mocap_last_row_attn_workspace_size(kv_len, n_q, d)
+    need = mocap_last_row_attn_workspace_size(kv_len, n_q, n_kv, d)
     if workspace is None:
         workspace = torch.empty((max(need, 16),), device=q_last.device, dtype=torch.uint8)
     ws_bytes = workspace.numel() * workspace.element_size()

@@ -2,17 +2,18 @@
 //
 // Sec. 2.1: a prefill-only request produces one output token, so the final
 // layer needs the attention output of the last prompt row alone: one query
-// row per q-head against every key of the request.  That is memory-bound
-// (each K/V byte is used by the Hq/Hkv query heads of its group only), so
-// this kernel streams K/V at HBM speed instead of running the 128-row tensor
-// core tiles of the chunk kernel:
-//   grid  = (key-range split, request, KV group); 128 threads per CTA
-//   TMA   K and V tiles of 128 keys through a 3-stage ring (bounded waits)
-//   S     thread t owns key t: s_h = scale * q_h . k_t for the group's heads
-//   soft  per-head online softmax in fp32 (block reductions, log2 domain)
-//   P.V   thread t owns dimension t: o_h[t] += sum_keys p_h[key] v[key][t]
-// Each CTA writes an fp32 partial (O / l, LSE) for its key range; the
-// split-KV combine kernel merges them.
+// row per q-head against every key of the request.  Each K/V byte serves
+// only the Hq/Hkv query heads of its group, so the work is memory-bound; the
+// kernel streams K/V tiles through TMA and lets the tensor core do the small
+// products in transposed form, so the 128 keys (or 128 dims) of a tile sit on
+// the 128 TMEM lanes:
+//   S^T[key, h]   = K[key, :] . q_h          (M=128 keys, N=16 padded heads)
+//   O_t^T[dim, h] = sum_key V[key, dim] p_h[key]   (M=128 dims, A = V^T MN-major)
+// Thread t owns key t for the softmax (per-head max / sum by block
+// reductions, fp32, log2 domain) and dimension t for the output accumulator
+// (registers, rescaled per tile).  grid = (key-range split, request, KV
+// group); each CTA writes an fp32 partial (O / l, LSE) that the split-KV
+// combine kernel merges.
 #include <cmath>
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -35,73 +36,117 @@ mocap_status launch_attn_combine(const float *o_part, const float *lse_part, int
 
 namespace {
 
-constexpr int kKeys = 128;        // keys per tile
-constexpr int kStages = 3;
+constexpr int kKeys = 128;     // keys per tile = TMEM lanes of S^T
+// One K+V tile in flight per CTA; several CTAs per SM (76 KB of shared
+// memory each) overlap each other's loads and small MMAs.  Measured on
+// GB300 against 2 stages x 2 CTAs/SM: 4.1 vs 3.5 TB/s (131072 keys).
+constexpr int kStages = 1;
+constexpr int kCtasPerSm = 3;
 constexpr int kThreads = 128;
-constexpr int kMaxGroup = 16;     // q-heads per KV head
+constexpr int kMaxGroup = 16;  // q-heads per KV head (MMA N = 16)
+constexpr int kN = 16;
 constexpr int kMaxReq = 64;
-constexpr int kTilesPerSplit = 16;  // 2048 keys per CTA at most
+constexpr uint32_t kTmemCols = 32;  // S^T [0, 16), O^T tile [16, 32)
 
 struct LastRowParams {
   CUtensorMap tk[kMaxReq];  // K of request r: [kv_len_r, Hkv, D], box {64, 1, 128}, 128B swizzle
-  CUtensorMap tv[kMaxReq];  // V of request r: same box, no swizzle
+  CUtensorMap tv[kMaxReq];  // V of request r: same
   const __nv_bfloat16 *q;   // [n_req, Hq, D]
   float *o_part;            // [splits, n_req, Hq, D]
   float *lse_part;          // [splits, Hq, n_req]
   uint32_t *status;
   int32_t kv_len[kMaxReq];
-  int32_t n_req, n_q_heads, n_kv_heads, group, splits;
+  int32_t n_req, n_q_heads, n_kv_heads, group, splits, tiles_per_cta;
   float scale_log2;
 };
 
 template <int D>
 struct LrLayout {
-  static constexpr int kTile = kKeys * D * 2;          // one K or V tile (bf16)
-  static constexpr int kStage = 2 * kTile;             // K + V
+  static constexpr int kTile = kKeys * D * 2;     // one K or V tile (bf16)
+  static constexpr int kStage = 2 * kTile;        // K + V
   static constexpr int kRing = 0;
-  static constexpr int kQ = kStages * kStage;          // fp32 [G][D]
-  static constexpr int kP = kQ + kMaxGroup * D * 4;    // fp32 [G][128]
-  static constexpr int kRed = kP + kMaxGroup * kKeys * 4;  // fp32 [4 warps][G]
-  static constexpr int kBars = kRed + 4 * kMaxGroup * 4;
-  static constexpr int kBytes = kBars + 8 * 2 * kStages + 1024;  // + alignment slack
+  static constexpr int kQ = kStages * kStage;     // Q_g: [16 heads x D] K-major, swizzled
+  static constexpr int kP = kQ + kN * D * 2;      // P:   [16 heads x 128 keys] K-major
+  static constexpr int kRed = kP + kN * kKeys * 2;  // fp32 [4 warps][16]
+  static constexpr int kBars = kRed + 4 * kN * 4;   // full[kStages], mma
+  static constexpr int kTmemSlot = kBars + 8 * (kStages + 1);
+  static constexpr int kBytes = kTmemSlot + 8 + 1024;  // + alignment slack
 };
 static_assert(LrLayout<128>::kBytes <= 232448, "shared memory");
+
+// Byte offset of element (row, col) in a K-major bf16 operand of `rows`
+// rows stored as 64-column boxes with the 128-byte swizzle.
+__device__ __forceinline__ uint32_t sw_off(int row, int col, int rows) {
+  const int box = col >> 6, c = col & 63;
+  return box * rows * 128 + row * 128 + ((((c >> 3) ^ (row & 7)) << 4) | ((c & 7) << 1));
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+}
 
 template <int D>
 __global__ void __launch_bounds__(kThreads) last_row_kernel(const __grid_constant__ LastRowParams p) {
   using L = LrLayout<D>;
   extern __shared__ uint8_t sm_raw[];
-  // 1024-byte aligned base: swizzled TMA tiles start on a swizzle period
   uint8_t *sm = sm_raw + ((1024u - (smem_u32(sm_raw) & 1023u)) & 1023u);
   const int split = blockIdx.x, r = blockIdx.y, g = blockIdx.z;
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int G = p.group;
   const int kv_len = p.kv_len[r];
   const int tiles = (kv_len + kKeys - 1) / kKeys;
-  const int per = (tiles + p.splits - 1) / p.splits;
-  const int t0 = min(tiles, split * per), t1 = min(tiles, t0 + per);
-  float *q_s = reinterpret_cast<float *>(sm + L::kQ);
-  float *p_s = reinterpret_cast<float *>(sm + L::kP);
-  float *red = reinterpret_cast<float *>(sm + L::kRed);
+  const int t0 = min(tiles, split * p.tiles_per_cta), t1 = min(tiles, t0 + p.tiles_per_cta);
+  const int n = t1 - t0;
   const uint32_t base = smem_u32(sm);
+  float *red = reinterpret_cast<float *>(sm + L::kRed);
   auto full = [&](int s) { return base + L::kBars + 8u * s; };
+  const uint32_t mma_bar = base + L::kBars + 8u * kStages;
+  const int64_t prow = static_cast<int64_t>(split) * p.n_req + r;
 
   __shared__ uint32_t abort_flag;
   if (t == 0) abort_flag = *reinterpret_cast<volatile uint32_t *>(p.status);
   __syncthreads();
   if (abort_flag != 0u) return;
+  if (n <= 0) {  // no key in this split: an empty partial (weight 0 in the merge)
+    for (int h = 0; h < G; ++h) {
+      if (t < D) p.o_part[(prow * p.n_q_heads + g * G + h) * D + t] = 0.0f;
+      if (t == 0) p.lse_part[(static_cast<int64_t>(split) * p.n_q_heads + g * G + h) * p.n_req + r] = -INFINITY;
+    }
+    return;
+  }
 
-  // the group's query rows, fp32, pre-scaled by scale * log2(e)
-  for (int i = t; i < G * D; i += kThreads) {
+  // Q_g (unscaled bf16) and a zeroed P tile, in the MMA's swizzled layout.
+  for (int i = t; i < kN * D; i += kThreads) {
     const int h = i / D, c = i % D;
-    q_s[i] = __bfloat162float(p.q[(static_cast<int64_t>(r) * p.n_q_heads + g * G + h) * D + c]) *
-             p.scale_log2;
+    const __nv_bfloat16 v = h < G ? p.q[(static_cast<int64_t>(r) * p.n_q_heads + g * G + h) * D + c]
+                                  : __float2bfloat16(0.0f);
+    *reinterpret_cast<__nv_bfloat16 *>(sm + L::kQ + sw_off(h, c, kN)) = v;
+  }
+  for (int i = t; i < kN * kKeys / 8; i += kThreads)
+    reinterpret_cast<uint4 *>(sm + L::kP)[i] = make_uint4(0, 0, 0, 0);
+  if (warp == 0) {
+    tmem_alloc(base + L::kTmemSlot, kTmemCols);
+    tmem_relinquish();
   }
   if (t == 0) {
     for (int s = 0; s < kStages; ++s) mbar_init(full(s), 1);
+    mbar_init(mma_bar, 1);
     fence_mbar_init();
   }
+  fence_proxy_async_shared();
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(sm + L::kTmemSlot);
+  const uint32_t lane_addr = tmem + ((static_cast<uint32_t>(warp) * 32u) << 16);
 
   const CUtensorMap *mk = &p.tk[r];
   const CUtensorMap *mv = &p.tv[r];
@@ -113,11 +158,18 @@ __global__ void __launch_bounds__(kThreads) last_row_kernel(const __grid_constan
       tma_load_3d(dst + L::kTile + c * (kKeys * 128), mv, full(s), c * 64, g, tile * kKeys);
     }
   };
-  const int n = t1 - t0;
-  int issued = 0;  // tiles whose loads were started (thread 0)
+  int issued = 0;
   if (t == 0)
     for (; issued < min(n, kStages); ++issued) issue(t0 + issued, issued);
 
+  // V^T as the M=128 A operand: dims 64..127 are the tile's second 64-dim
+  // box (16 KB on).  With D = 64 there is no second box, so it aliases the
+  // first (leading offset 0): those lanes of O^T are never read, and every
+  // operand read stays inside this stage's V tile.
+  constexpr uint32_t kVAtomStride = D == 128 ? kKeys * 128 : 0;
+  constexpr uint32_t idesc_s = idesc_bf16_f32(128, kN, false, false);
+  constexpr uint32_t idesc_o = idesc_bf16_f32(128, kN, true, false);
+  const float sl2 = p.scale_log2;
   float m[kMaxGroup], lsum[kMaxGroup], o[kMaxGroup];
 #pragma unroll
   for (int h = 0; h < kMaxGroup; ++h) {
@@ -126,125 +178,128 @@ __global__ void __launch_bounds__(kThreads) last_row_kernel(const __grid_constan
     o[h] = 0.0f;
   }
   bool ok = true;
+  int mma_phase = 0;
   for (int j = 0; j < n; ++j) {
     const int s = j % kStages;
-    const bool landed = mbar_wait(full(s), (j / kStages) & 1, p.status);
-    if (!__syncthreads_and(landed)) {  // the whole CTA agrees before unwinding
+    const uint32_t kt = base + L::kRing + s * L::kStage, vt = kt + L::kTile;
+    if (!__syncthreads_and(mbar_wait(full(s), (j / kStages) & 1, p.status))) {
       ok = false;
       break;
     }
-    const uint8_t *kt = sm + L::kRing + s * L::kStage;  // box c: [128 keys][64 dims]
-    const uint8_t *vt = kt + L::kTile;
-    const int key = (t0 + j) * kKeys + t;
-    // ---- scores: thread t = key t
+    // ---- S^T = K . Q_g^T (keys on the lanes)
+    if (t == 0) {
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = (kk / 4) * (kKeys * 128) + (kk % 4) * 32;
+        const uint32_t qoff = (kk / 4) * (kN * 128) + (kk % 4) * 32;
+        mma_ss(tmem, sdesc_sw128(kt + off, 16, 1024), sdesc_sw128(base + L::kQ + qoff, 16, 1024),
+               idesc_s, kk > 0 ? 1u : 0u);
+      }
+      tc_commit(mma_bar);
+    }
+    if (!__syncthreads_and(mbar_wait(mma_bar, mma_phase & 1, p.status))) {
+      ok = false;
+      break;
+    }
+    ++mma_phase;
+    tc_fence_after();
+    uint32_t sr[16];
+    tmem_ld16(lane_addr, sr);
+    const bool valid_key = (t0 + j) * kKeys + t < kv_len;
     float sc[kMaxGroup];
 #pragma unroll
-    for (int h = 0; h < kMaxGroup; ++h) sc[h] = 0.0f;
-    for (int c = 0; c < D / 64; ++c) {
-      // key t's 64 dims of box c: 16-byte chunk v8 sits at (v8 ^ (t & 7)) * 16
-      const uint8_t *krow = kt + c * (kKeys * 128) + t * 128;
-#pragma unroll
-      for (int v8 = 0; v8 < 8; ++v8) {
-        const uint4 kv = *reinterpret_cast<const uint4 *>(krow + ((v8 ^ (t & 7)) << 4));
-        const __nv_bfloat162 *k2 = reinterpret_cast<const __nv_bfloat162 *>(&kv);
-        float kf[8];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 f = __bfloat1622float2(k2[e]);
-          kf[2 * e] = f.x;
-          kf[2 * e + 1] = f.y;
-        }
-        const int d0 = c * 64 + v8 * 8;
-#pragma unroll
-        for (int h = 0; h < kMaxGroup; ++h) {
-          if (h < G) {
-            const float *qh = q_s + h * D + d0;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) sc[h] = fmaf(qh[e], kf[e], sc[h]);
-          }
-        }
-      }
-    }
-    if (key >= kv_len)
-#pragma unroll
-      for (int h = 0; h < kMaxGroup; ++h) sc[h] = -INFINITY;
-    // ---- per-head tile max (warp shuffle, then across the 4 warps)
-#pragma unroll
     for (int h = 0; h < kMaxGroup; ++h) {
-      if (h < G) {
-        float v = sc[h];
+      sc[h] = valid_key ? __uint_as_float(sr[h]) * sl2 : -INFINITY;
+      float v = sc[h];
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
-        if (lane == 0) red[warp * kMaxGroup + h] = v;
-      }
+      for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+      if (lane == 0) red[warp * kN + h] = v;
     }
     __syncthreads();
     float alpha[kMaxGroup];
 #pragma unroll
     for (int h = 0; h < kMaxGroup; ++h) {
-      alpha[h] = 1.0f;
-      if (h < G) {
-        const float tm = fmaxf(fmaxf(red[h], red[kMaxGroup + h]),
-                               fmaxf(red[2 * kMaxGroup + h], red[3 * kMaxGroup + h]));
-        const float mn = fmaxf(m[h], tm);  // finite: key tile j contains a valid key
-        alpha[h] = ex2_approx(m[h] - mn);  // m = -inf at the first tile: alpha = 0
-        m[h] = mn;
-        const float pr = ex2_approx(sc[h] - mn);
-        p_s[h * kKeys + t] = pr;
-        lsum[h] = lsum[h] * alpha[h] + pr;
-      }
+      const float tm = fmaxf(fmaxf(red[h], red[kN + h]), fmaxf(red[2 * kN + h], red[3 * kN + h]));
+      const float mn = fmaxf(m[h], tm);  // finite: each tile holds a valid key
+      alpha[h] = ex2_approx(m[h] - mn);  // 0 on the first tile (m = -inf)
+      m[h] = mn;
+      const float pr = ex2_approx(sc[h] - mn);
+      lsum[h] = lsum[h] * alpha[h] + pr;
+      if (h < G)
+        *reinterpret_cast<__nv_bfloat16 *>(sm + L::kP + sw_off(h, t, kN)) = __float2bfloat16_rn(pr);
     }
+    fence_proxy_async_shared();
+    tc_fence_before();
     __syncthreads();
-    // ---- P.V: thread t = dimension t (D == 128; for D == 64 threads >= 64 idle)
-    if (t < D) {
-      const int c = t / 64, dd = t % 64;
-      const uint8_t *vcol = vt + c * (kKeys * 128) + dd * 2;
+    // ---- O_t^T = V^T . P^T (dims on the lanes)
+    if (t == 0) {
+      tc_fence_after();
 #pragma unroll
-      for (int h = 0; h < kMaxGroup; ++h)
-        if (h < G) o[h] *= alpha[h];
-      for (int kk = 0; kk < kKeys; ++kk) {
-        const float vv = __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(vcol + kk * 128));
-#pragma unroll
-        for (int h = 0; h < kMaxGroup; ++h)
-          if (h < G) o[h] = fmaf(p_s[h * kKeys + kk], vv, o[h]);
+      for (int kk = 0; kk < kKeys / 16; ++kk) {
+        const uint32_t poff = (kk / 4) * (kN * 128) + (kk % 4) * 32;
+        mma_ss(tmem + kN, sdesc_sw128(vt + kk * 2048, kVAtomStride, 1024),
+               sdesc_sw128(base + L::kP + poff, 16, 1024), idesc_o, kk > 0 ? 1u : 0u);
       }
+      tc_commit(mma_bar);
     }
-    __syncthreads();  // stage s and p_s free again
-    if (t == 0 && j + kStages < n) {
-      issue(t0 + j + kStages, s);
+    if (!__syncthreads_and(mbar_wait(mma_bar, mma_phase & 1, p.status))) {
+      ok = false;
+      break;
+    }
+    ++mma_phase;
+    tc_fence_after();
+    uint32_t orr[16];
+    tmem_ld16(lane_addr + kN, orr);
+#pragma unroll
+    for (int h = 0; h < kMaxGroup; ++h) o[h] = o[h] * alpha[h] + __uint_as_float(orr[h]);
+    tc_fence_before();
+    __syncthreads();  // stage s, P and TMEM are free again
+    if (t == 0 && issued < n) {
+      issue(t0 + issued, issued % kStages);
       ++issued;
     }
   }
   if (!ok) {
-    // copies still in flight land before the CTA exits
-    if (t == 0)
+    if (t == 0) {
       for (int j = max(0, issued - kStages); j < issued; ++j)
         mbar_wait(full(j % kStages), (j / kStages) & 1, p.status, 20000000ull, false);
+      tc_commit(mma_bar);  // drain issued MMAs before TMEM is released
+      mbar_wait(mma_bar, mma_phase & 1, p.status, 20000000ull, false);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+      tc_fence_after();
+      tmem_dealloc(tmem, kTmemCols);
+    }
     return;
   }
-  // ---- row sums: per-thread partials (same rescales) -> block totals
+  // ---- row sums over the block; write this split's partial
 #pragma unroll
   for (int h = 0; h < kMaxGroup; ++h) {
-    if (h < G) {
-      float v = lsum[h];
+    float v = lsum[h];
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      if (lane == 0) red[warp * kMaxGroup + h] = v;
-    }
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane == 0) red[warp * kN + h] = v;
   }
   __syncthreads();
-  const int64_t prow = static_cast<int64_t>(split) * p.n_req + r;
 #pragma unroll
   for (int h = 0; h < kMaxGroup; ++h) {
     if (h < G) {
-      const float l = red[h] + red[kMaxGroup + h] + red[2 * kMaxGroup + h] + red[3 * kMaxGroup + h];
-      const bool any = n > 0 && l > 0.0f;
+      const float l = red[h] + red[kN + h] + red[2 * kN + h] + red[3 * kN + h];
       const int head = g * G + h;
-      if (t < D) p.o_part[(prow * p.n_q_heads + head) * D + t] = any ? o[h] / l : 0.0f;
+      if (t < D) p.o_part[(prow * p.n_q_heads + head) * D + t] = o[h] / l;
       if (t == 0)
         p.lse_part[(static_cast<int64_t>(split) * p.n_q_heads + head) * p.n_req + r] =
-            any ? (m[h] + log2f(l)) * 0.69314718055994530942f : -INFINITY;
+            (m[h] + log2f(l)) * 0.69314718055994530942f;
     }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
   }
 }
 
@@ -280,19 +335,51 @@ bool make_kv_map(CUtensorMap *map, const void *ptr, int64_t rows, int heads, int
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int plan_splits(const int64_t *kv_len, int n_req) {
-  int64_t max_tiles = 1;
-  for (int r = 0; r < n_req; ++r) max_tiles = std::max<int64_t>(max_tiles, (kv_len[r] + kKeys - 1) / kKeys);
-  return static_cast<int>((max_tiles + kTilesPerSplit - 1) / kTilesPerSplit);
+int sm_count_lr() {
+  static int cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+// Tiles per CTA so that all (request, group) key ranges give about
+// kCtasPerSm CTAs per SM in total; the split count is what the longest
+// request needs.
+struct LrPlan {
+  int tiles_per_cta = 1, splits = 1;
+};
+LrPlan plan_splits(const int64_t *kv_len, int n_req, int n_kv_heads) {
+  int64_t total = 0, max_tiles = 1;
+  for (int r = 0; r < n_req; ++r) {
+    const int64_t tr = std::max<int64_t>(1, (kv_len[r] + kKeys - 1) / kKeys);
+    total += tr;
+    max_tiles = std::max(max_tiles, tr);
+  }
+  const int64_t target_ctas = static_cast<int64_t>(kCtasPerSm) * sm_count_lr();
+  int64_t per = (total * n_kv_heads + target_ctas - 1) / target_ctas;
+  per = std::max<int64_t>(1, per);
+  LrPlan pl;
+  pl.tiles_per_cta = static_cast<int>(per);
+  pl.splits = static_cast<int>((max_tiles + per - 1) / per);
+  return pl;
 }
 
 }  // namespace
 }  // namespace mocap
 
 extern "C" size_t mocap_last_row_attn_workspace_size(const int64_t *kv_len, int32_t n_req,
-                                                     int32_t n_q_heads, int32_t head_dim) {
-  if (kv_len == nullptr || n_req < 1 || n_req > mocap::kMaxReq || n_q_heads < 1) return 0;
-  const size_t splits = static_cast<size_t>(mocap::plan_splits(kv_len, n_req));
+                                                     int32_t n_q_heads, int32_t n_kv_heads,
+                                                     int32_t head_dim) {
+  if (kv_len == nullptr || n_req < 1 || n_req > mocap::kMaxReq || n_q_heads < 1 ||
+      n_kv_heads < 1)
+    return 0;
+  const size_t splits = static_cast<size_t>(mocap::plan_splits(kv_len, n_req, n_kv_heads).splits);
   const size_t o = splits * n_req * n_q_heads * head_dim * sizeof(float);
   return (o + 255) / 256 * 256 + splits * n_q_heads * n_req * sizeof(float);
 }
@@ -319,7 +406,8 @@ extern "C" mocap_status mocap_last_row_attn(const void *q_last, const void *k_ca
     if (kv_len[r] < 1 || kv_row[r] < 0 || kv_len[r] > 0x7fffffffLL ||
         kv_row[r] > kv_rows_total - kv_len[r])
       return MOCAP_EINVAL;
-  const size_t need = mocap_last_row_attn_workspace_size(kv_len, n_req, n_q_heads, head_dim);
+  const size_t need =
+      mocap_last_row_attn_workspace_size(kv_len, n_req, n_q_heads, n_kv_heads, head_dim);
   if (workspace_bytes < need) return MOCAP_EINVAL;
   uint32_t *status = device_status_ptr();
   if (status == nullptr) return MOCAP_ECUDA;
@@ -333,11 +421,12 @@ extern "C" mocap_status mocap_last_row_attn(const void *q_last, const void *k_ca
     const auto *kb = static_cast<const uint8_t *>(k_cache) + kv_row[r] * row_bytes;
     const auto *vb = static_cast<const uint8_t *>(v_cache) + kv_row[r] * row_bytes;
     if (!make_kv_map(&prm.tk[r], kb, kv_len[r], n_kv_heads, head_dim, true) ||
-        !make_kv_map(&prm.tv[r], vb, kv_len[r], n_kv_heads, head_dim, false))
+        !make_kv_map(&prm.tv[r], vb, kv_len[r], n_kv_heads, head_dim, true))
       return MOCAP_ECUDA;
     prm.kv_len[r] = static_cast<int32_t>(kv_len[r]);
   }
-  const int splits = plan_splits(kv_len, n_req);
+  const LrPlan plan = plan_splits(kv_len, n_req, n_kv_heads);
+  const int splits = plan.splits;
   const size_t o_bytes = static_cast<size_t>(splits) * n_req * n_q_heads * head_dim * sizeof(float);
   prm.q = static_cast<const __nv_bfloat16 *>(q_last);
   prm.o_part = static_cast<float *>(workspace);
@@ -348,6 +437,7 @@ extern "C" mocap_status mocap_last_row_attn(const void *q_last, const void *k_ca
   prm.n_kv_heads = n_kv_heads;
   prm.group = n_q_heads / n_kv_heads;
   prm.splits = splits;
+  prm.tiles_per_cta = plan.tiles_per_cta;
   prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
   const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const dim3 grid(splits, n_req, n_kv_heads);

@@ -355,6 +355,12 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return d;
 }
 
+// Make this thread's generic-proxy shared-memory writes visible to the async
+// proxy (tensor core / TMA reads) once the following synchronisation is seen.
+__device__ __forceinline__ void fence_proxy_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // 2^x on the special-function unit (PTX ex2.approx.ftz.f32); ex2(-inf) = +0.
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
