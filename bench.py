@@ -58,6 +58,12 @@ def parse_args():
     ap.add_argument("--case", default=None,
                     help="profiling case 'prefix,len,Hq,Hkv,d': one chunk attention launch "
                          "repeated warmup+steps times (no JSON metric line)")
+    ap.add_argument("--case-qkv", default=None,
+                    help="profiling case 'len,hidden,Hq,Hkv,d': one QKV projection launch "
+                         "repeated warmup+steps times")
+    ap.add_argument("--case-last-row", default=None,
+                    help="profiling case 'keys,Hq,Hkv,d': one last-row attention launch "
+                         "repeated warmup+steps times")
     return ap.parse_args()
 
 
@@ -339,6 +345,13 @@ def ours_arm(args, rank, world, local):
     stream = torch.cuda.current_stream(dev)
 
     flops_chunks = attn_flops(pf.bounds, w.n_q_heads, w.head_dim)
+    # chunks whose key range the library splits (each adds a combine launch)
+    n_combines = 0
+    if pf.single and pf.workspace is not None:
+        b = pf.bounds[0]
+        n_combines = sum(1 for i in range(len(b) - 1)
+                         if m.mocap_chunk_attn_workspace_size(b[i], b[i + 1] - b[i], w.n_q_heads,
+                                                              w.n_kv_heads, w.head_dim) > 0)
     # per step (chunk index k): attention FLOP of every (request, k)
     step_flops = [sum(flops_chunks[r][c] for r, c in st) for st in steps_plan]
     total_flops = sum(step_flops)
@@ -421,9 +434,9 @@ def ours_arm(args, rank, world, local):
                      "traffic": None if traffic_full is None else traffic_full / launches_per_step,
                      "traffic_unit": "bytes per launch (avg over the step's launches)"},
         "clocks": clk,
-        # our kernels per timed region: one append per (request, chunk) and
-        # one attention launch per step
-        "gpu_launches": args.steps * sum(1 + len(st) for st in steps_plan),
+        # our kernels per timed region: one append per (request, chunk), one
+        # attention launch per step, one split-KV combine per split chunk
+        "gpu_launches": args.steps * (sum(1 + len(st) for st in steps_plan) + n_combines),
     }
 
     if not args.no_graph:
@@ -620,10 +633,90 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
             "overlap": "per-chunk H2D / compute / D2H on three streams"}
 
 
+def profile_case(args):
+    """A single chunk_attn launch shape, repeated: the small case for ncu."""
+    import torch
+    import paper_2606_22968_gb300 as m
+    prefix, length, hq, hkv, d = (int(x) for x in args.case.split(","))
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(7)
+    q = torch.randn((length, hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    kc = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    vc = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    out = torch.empty_like(q)
+    lse = torch.empty((hq, length), device=dev, dtype=torch.float32)
+    ms = _repeat_timed(args, lambda: m.mocap_chunk_attn(q, kc, vc, prefix, out, lse,
+                                                        1.0 / math.sqrt(d)))
+    if m.mocap_last_device_status() != m.MOCAP_OK:
+        raise RuntimeError("device wait expired")
+    flops = 4 * hq * d * (length * prefix + length * (length + 1) // 2)
+    print(json.dumps({"case": args.case, "ms": ms, "tflops": flops / ms / 1e9,
+                      "kv_bytes": 2 * (prefix + length) * hkv * d * 2}), flush=True)
+    return 0
+
+
+def _repeat_timed(args, fn):
+    import torch
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    times = []
+    for i in range(args.warmup + args.steps):
+        ev[0].record()
+        fn()
+        ev[1].record()
+        torch.cuda.synchronize()
+        if i >= args.warmup:
+            times.append(ev[0].elapsed_time(ev[1]))
+    return statistics.median(times)
+
+
+def profile_case_qkv(args):
+    """One QKV projection + RoPE + append shape, repeated (ncu probe)."""
+    import torch
+    import paper_2606_22968_gb300 as m
+    length, hidden, hq, hkv, d = (int(x) for x in args.case_qkv.split(","))
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(11)
+    x = torch.randn((length, hidden), generator=gen, device=dev, dtype=torch.bfloat16)
+    w = torch.randn(((hq + 2 * hkv) * d, hidden), generator=gen, device=dev, dtype=torch.bfloat16)
+    q = torch.empty((length, hq, d), device=dev, dtype=torch.bfloat16)
+    kc = torch.empty((length, hkv, d), device=dev, dtype=torch.bfloat16)
+    vc = torch.empty_like(kc)
+    ms = _repeat_timed(args, lambda: m.mocap_qkv_rope_append(x, w, q, kc, vc, 0))
+    flops = 2 * length * hidden * (hq + 2 * hkv) * d
+    print(json.dumps({"case_qkv": args.case_qkv, "ms": ms, "tflops": flops / ms / 1e9}), flush=True)
+    return 0
+
+
+def profile_case_last_row(args):
+    """One last-row attention shape, repeated (ncu probe)."""
+    import torch
+    import paper_2606_22968_gb300 as m
+    keys, hq, hkv, d = (int(x) for x in args.case_last_row.split(","))
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(12)
+    k = torch.randn((keys, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    v = torch.randn((keys, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    q = torch.randn((1, hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    out = torch.empty_like(q)
+    lse = torch.empty((hq, 1), device=dev, dtype=torch.float32)
+    ws = torch.empty((max(16, m.mocap_last_row_attn_workspace_size([keys], hq, hkv, d)),),
+                     device=dev, dtype=torch.uint8)
+    ms = _repeat_timed(args, lambda: m.mocap_last_row_attn(q, k, v, [0], [keys], out, lse,
+                                                           1.0 / math.sqrt(d), workspace=ws))
+    byts = keys * hkv * d * 4
+    print(json.dumps({"case_last_row": args.case_last_row, "ms": ms,
+                      "gb_per_s": byts / ms / 1e6}), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
     if args.case:
         return profile_case(args)
+    if args.case_qkv:
+        return profile_case_qkv(args)
+    if args.case_last_row:
+        return profile_case_last_row(args)
     rank, world, local = init_dist(args)
     try:
         if args.impl == "reference":

@@ -198,3 +198,12 @@ def test_dp_partition_invalid_and_limits(lib):
     assert lib.mocap_lbcp_partition_dp(1024, 9, 128, 4, 0, 0, out) == 1      # M g > S
     assert lib.mocap_lbcp_partition_dp(1 << 30, 32, 1, 4, 0, 0, out) == 3    # too large
     assert lib.mocap_lbcp_partition_dp(131072, 32, 128, 16, 0, 0, out) == 0
+
+
+def test_bench_entry_points_exist():
+    """bench.py's probe modes and arms are all defined (they are run on the GPU)."""
+    import bench
+    for name in ["profile_case", "profile_case_qkv", "profile_case_last_row", "ours_arm",
+                 "reference_arm", "measure_e2e", "measure_graph", "measure_projection",
+                 "measure_last_row", "measure_uniform"]:
+        assert callable(getattr(bench, name)), name
