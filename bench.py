@@ -655,17 +655,23 @@ def profile_case(args):
     return 0
 
 
-def _repeat_timed(args, fn):
+def _repeat_timed(args, fn, reps=20):
+    """Median over `steps` samples of the mean time of `reps` back-to-back
+    calls (the host enqueues ahead of the device, so per-call host work stays
+    outside the device time)."""
     import torch
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-    times = []
-    for i in range(args.warmup + args.steps):
-        ev[0].record()
+    for _ in range(args.warmup):
         fn()
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(args.steps):
+        ev[0].record()
+        for _ in range(reps):
+            fn()
         ev[1].record()
         torch.cuda.synchronize()
-        if i >= args.warmup:
-            times.append(ev[0].elapsed_time(ev[1]))
+        times.append(ev[0].elapsed_time(ev[1]) / reps)
     return statistics.median(times)
 
 

@@ -311,15 +311,20 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
  * n_q_heads / n_kv_heads heads of its group), so a dedicated kernel streams
  * K/V tiles through TMA, lets the tensor core form the small products in
  * transposed form (keys, then dimensions, on the 128 TMEM lanes), and splits
- * the requests' keys into ranges (about two CTAs per SM in total) whose fp32
- * partials are merged like split-KV.
+ * the requests' keys into ranges (about three CTAs per SM in total) whose
+ * fp32 partials are merged like split-KV, in the same launch: the last CTA
+ * of each (request, KV group) to finish merges the group's partials.
  *
  *   q_last    bf16 [n_req, Hq, d]: the last row's queries of each request
  *   k_cache,  bf16 [kv_rows_total, Hkv, d]: request r's keys are rows
  *   v_cache   kv_row[r] .. kv_row[r] + kv_len[r] - 1 (rows past them unread)
  *   kv_row, kv_len  HOST arrays of n_req int64 (kv_len[r] >= 1)
  *   out       bf16 [n_req, Hq, d];  lse fp32 [Hq, n_req]
- *   workspace at least mocap_last_row_attn_workspace_size(...) bytes
+ *   workspace at least mocap_last_row_attn_workspace_size(...) bytes, 16-byte
+ *             aligned: fp32 partials plus n_req * Hkv arrival counters, which
+ *             the call zeroes with a memset on `stream` before its launch.
+ *             Calls that may run concurrently need separate workspaces.
+ * Enqueues one memset and one kernel.
  * 1 <= n_req <= 64; Hq / Hkv <= 16; head_dim in {64, 128}.
  */
 size_t mocap_last_row_attn_workspace_size(const int64_t *kv_len, int32_t n_req,

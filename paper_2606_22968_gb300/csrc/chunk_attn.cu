@@ -48,6 +48,7 @@ namespace {
 
 constexpr int kBlockM = 128;   // query rows per tile = TMEM lanes
 constexpr int kBlockN = 128;   // keys per K/V tile
+constexpr int kMaxSplits = 4;  // key-range splits of one chunk (split-KV)
 constexpr int kStages = 4;     // ring stages, each holds one K or one V tile
 constexpr int kThreads = 384;  // 3 warpgroups: {producer, MMA, 2 idle}, softmax 0, softmax 1
 // Register split (setmaxnreg): the kernel is built for 168 registers per
@@ -589,7 +590,7 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(
   const int lane = threadIdx.x & 31;
   const int64_t row = idx / n_q_heads;
   const int h = static_cast<int>(idx % n_q_heads);
-  float lk[8];
+  float lk[kMaxSplits];
   float mx = -INFINITY;
   for (int k = 0; k < splits; ++k) {
     lk[k] = lse_part[(static_cast<int64_t>(k) * n_q_heads + h) * len + row];
@@ -720,7 +721,7 @@ int choose_splits(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads, in
   double best_t = 0.0;
   int best = 1;
   std::vector<double> sm(static_cast<size_t>(sms));
-  for (int sp = 1; sp <= 4 && sp <= min_tiles; ++sp) {
+  for (int sp = 1; sp <= kMaxSplits && sp <= min_tiles; ++sp) {
     std::fill(sm.begin(), sm.end(), 0.0);
     for (int64_t qb = q_blocks - 1; qb >= 0; --qb) {
       const int64_t kv_end = std::min<int64_t>(prefix + qb * kBlockM + kBlockM, prefix + len);
@@ -793,7 +794,7 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
   prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
   prm.splits = sp.splits;
   if (sp.splits > 1) {
-    if (n != 1 || workspace == nullptr) return MOCAP_EINVAL;
+    if (n != 1 || workspace == nullptr || sp.splits > kMaxSplits) return MOCAP_EINVAL;
     prm.o_part = static_cast<float *>(workspace);
     prm.lse_part = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + sp.lse_off);
   }
@@ -845,22 +846,6 @@ constexpr int64_t kMaxRows = 0x7fffffffLL;
 
 }  // namespace
 
-// Merge split partials (o_part [splits, len, Hq, d], lse_part [splits, Hq,
-// len]) into bf16 out [len, Hq, d] and fp32 lse [Hq, lse_stride].
-mocap_status launch_attn_combine(const float *o_part, const float *lse_part, int splits,
-                                 int64_t len, int n_q_heads, int head_dim, void *out, float *lse,
-                                 int64_t lse_stride, cudaStream_t stream) {
-  const int64_t warps = len * n_q_heads;
-  const unsigned blocks = static_cast<unsigned>((warps + 7) / 8);
-  auto *o = static_cast<__nv_bfloat16 *>(out);
-  if (head_dim == 128)
-    attn_combine_kernel<128><<<blocks, 256, 0, stream>>>(o_part, lse_part, splits, len, n_q_heads,
-                                                         o, lse, lse_stride);
-  else
-    attn_combine_kernel<64><<<blocks, 256, 0, stream>>>(o_part, lse_part, splits, len, n_q_heads,
-                                                        o, lse, lse_stride);
-  return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
-}
 }  // namespace mocap
 
 using mocap::HostItem;
@@ -879,7 +864,7 @@ mocap::SplitPlan plan_for(int64_t prefix, int64_t len, int32_t n_q_heads, int32_
   // capped so the first row block still has a key tile per split.
   if (const char *env = std::getenv("MOCAP_SPLIT_KV")) {
     const int forced = std::atoi(env);
-    if (forced >= 0 && forced <= 4) {
+    if (forced >= 0 && forced <= mocap::kMaxSplits) {
       const int64_t min_tiles = (std::min<int64_t>(prefix + mocap::kBlockM, prefix + len) +
                                  mocap::kBlockN - 1) / mocap::kBlockN;
       splits = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(forced, min_tiles)));

@@ -12,8 +12,10 @@
 // Thread t owns key t for the softmax (per-head max / sum by block
 // reductions, fp32, log2 domain) and dimension t for the output accumulator
 // (registers, rescaled per tile).  grid = (key-range split, request, KV
-// group); each CTA writes an fp32 partial (O / l, LSE) that the split-KV
-// combine kernel merges.
+// group); each CTA writes an fp32 partial (O / l, LSE) and bumps a counter of
+// its (request, group); the CTA that completes the count merges the group's
+// partials (the split-KV combine, O = sum_s e^(LSE_s - LSE) O_s) in the same
+// launch, so no second kernel and no launch gap follow.
 #include <cmath>
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -28,12 +30,6 @@
 #include "sm103_ptx.cuh"
 
 namespace mocap {
-
-// Shared with the chunk kernel's translation unit: merges split partials.
-mocap_status launch_attn_combine(const float *o_part, const float *lse_part, int splits,
-                                 int64_t len, int n_q_heads, int head_dim, void *out, float *lse,
-                                 int64_t lse_stride, cudaStream_t stream);
-
 namespace {
 
 constexpr int kKeys = 128;     // keys per tile = TMEM lanes of S^T
@@ -46,6 +42,7 @@ constexpr int kThreads = 128;
 constexpr int kMaxGroup = 16;  // q-heads per KV head (MMA N = 16)
 constexpr int kN = 16;
 constexpr int kMaxReq = 64;
+constexpr int kMaxParts = 512;  // key-range splits of one request (merge scratch)
 constexpr uint32_t kTmemCols = 32;  // S^T [0, 16), O^T tile [16, 32)
 
 struct LastRowParams {
@@ -54,6 +51,9 @@ struct LastRowParams {
   const __nv_bfloat16 *q;   // [n_req, Hq, D]
   float *o_part;            // [splits, n_req, Hq, D]
   float *lse_part;          // [splits, Hq, n_req]
+  uint32_t *arrived;        // [n_req, Hkv] CTAs done per (request, group); zero at launch
+  __nv_bfloat16 *out;       // [n_req, Hq, D]
+  float *lse;               // [Hq, n_req]
   uint32_t *status;
   int32_t kv_len[kMaxReq];
   int32_t n_req, n_q_heads, n_kv_heads, group, splits, tiles_per_cta;
@@ -93,8 +93,91 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       : "memory");
 }
 
+// Split-KV merge of one (request, group) by one CTA, in shared memory below
+// the `red` area (the drained K/V ring, Q_g and P regions):
+//   1. the parts' LSEs, w[k][h] for k < n_parts, h < 16;
+//   2. per head the maximum M_h (one warp per head, lanes over the parts);
+//   3. w[k][h] = exp(LSE_kh - M_h) and their sums W_h;
+//   4. each thread owns (head, 4 dims) pairs and sums w * O_k over the parts
+//      with eight independent loads in flight, then scales by 1 / W_h.
+// Every merged part holds at least one key, so each LSE_kh is finite.
 template <int D>
-__global__ void __launch_bounds__(kThreads) last_row_kernel(const __grid_constant__ LastRowParams p) {
+__device__ __forceinline__ void merge_group(const LastRowParams &p, uint8_t *sm, int r, int g,
+                                            int n_parts) {
+  constexpr int kCols = D / 4;  // float4 columns of a head row
+  static_assert(kMaxParts * kMaxGroup * 4 + 2 * kMaxGroup * 4 <= LrLayout<D>::kRed, "merge scratch");
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int G = p.group, Hq = p.n_q_heads;
+  float *w = reinterpret_cast<float *>(sm);   // [n_parts][16]
+  float *mh = w + kMaxParts * kMaxGroup;      // [16]
+  float *wh = mh + kMaxGroup;                 // [16]
+  const int n_items = n_parts * kMaxGroup;
+  for (int i0 = t; i0 < n_items; i0 += 4 * kThreads) {
+    float v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = i0 + u * kThreads, k = i / kMaxGroup, h = i % kMaxGroup;
+      v[u] = i < n_items && h < G
+                 ? __ldcg(p.lse_part + (static_cast<int64_t>(k) * Hq + g * G + h) * p.n_req + r)
+                 : 0.0f;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (i0 + u * kThreads < n_items) w[i0 + u * kThreads] = v[u];
+  }
+  __syncthreads();
+  for (int h = warp; h < G; h += kThreads / 32) {
+    float m = -INFINITY;
+    for (int k = lane; k < n_parts; k += 32) m = fmaxf(m, w[k * kMaxGroup + h]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+    float sum = 0.0f;
+    for (int k = lane; k < n_parts; k += 32) {
+      const float e = expf(w[k * kMaxGroup + h] - m);
+      w[k * kMaxGroup + h] = e;
+      sum += e;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    if (lane == 0) {
+      mh[h] = m;
+      wh[h] = sum;
+    }
+  }
+  __syncthreads();
+  const float4 *o4 = reinterpret_cast<const float4 *>(p.o_part);
+  const int64_t part_stride = static_cast<int64_t>(p.n_req) * Hq * kCols;  // float4s per part
+  for (int pair = t; pair < G * kCols; pair += kThreads) {
+    const int h = pair / kCols, c = pair % kCols;
+    const float4 *src = o4 + (static_cast<int64_t>(r) * Hq + g * G + h) * kCols + c;
+    float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    for (int k0 = 0; k0 < n_parts; k0 += 8) {
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        v[u] = k0 + u < n_parts ? __ldcg(src + (k0 + u) * part_stride)
+                                : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float wk = k0 + u < n_parts ? w[(k0 + u) * kMaxGroup + h] : 0.0f;
+        acc.x += wk * v[u].x;
+        acc.y += wk * v[u].y;
+        acc.z += wk * v[u].z;
+        acc.w += wk * v[u].w;
+      }
+    }
+    const float inv = 1.0f / wh[h];
+    const int head = g * G + h;
+    __nv_bfloat162 *dst =
+        reinterpret_cast<__nv_bfloat162 *>(p.out + (static_cast<int64_t>(r) * Hq + head) * D + 4 * c);
+    dst[0] = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+    dst[1] = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+    if (c == 0) p.lse[static_cast<int64_t>(head) * p.n_req + r] = mh[h] + logf(wh[h]);
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) last_row_kernel(const __grid_constant__ LastRowParams p) {
   using L = LrLayout<D>;
   extern __shared__ uint8_t sm_raw[];
   uint8_t *sm = sm_raw + ((1024u - (smem_u32(sm_raw) & 1023u)) & 1023u);
@@ -115,13 +198,8 @@ __global__ void __launch_bounds__(kThreads) last_row_kernel(const __grid_constan
   if (t == 0) abort_flag = *reinterpret_cast<volatile uint32_t *>(p.status);
   __syncthreads();
   if (abort_flag != 0u) return;
-  if (n <= 0) {  // no key in this split: an empty partial (weight 0 in the merge)
-    for (int h = 0; h < G; ++h) {
-      if (t < D) p.o_part[(prow * p.n_q_heads + g * G + h) * D + t] = 0.0f;
-      if (t == 0) p.lse_part[(static_cast<int64_t>(split) * p.n_q_heads + g * G + h) * p.n_req + r] = -INFINITY;
-    }
-    return;
-  }
+  if (n <= 0) return;  // past the request's keys: this split takes no part
+  const int n_parts = (tiles + p.tiles_per_cta - 1) / p.tiles_per_cta;  // splits with keys
 
   // Q_g (unscaled bf16) and a zeroed P tile, in the MMA's swizzled layout.
   for (int i = t; i < kN * D; i += kThreads) {
@@ -301,6 +379,19 @@ __global__ void __launch_bounds__(kThreads) last_row_kernel(const __grid_constan
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+
+  // ---- the last of the group's n_parts CTAs merges their partials
+  __shared__ uint32_t is_last;
+  __threadfence();  // this CTA's partial is visible device-wide before the count
+  __syncthreads();
+  if (t == 0) {
+    const uint32_t before = atomicAdd(p.arrived + r * p.n_kv_heads + g, 1u);
+    is_last = before + 1u == static_cast<uint32_t>(n_parts) ? 1u : 0u;
+  }
+  __syncthreads();
+  if (is_last == 0u) return;
+  __threadfence();  // order the partial reads after the count that completed
+  merge_group<D>(p, sm, r, g, n_parts);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn3() {
@@ -364,9 +455,10 @@ LrPlan plan_splits(const int64_t *kv_len, int n_req, int n_kv_heads) {
   const int64_t target_ctas = static_cast<int64_t>(kCtasPerSm) * sm_count_lr();
   int64_t per = (total * n_kv_heads + target_ctas - 1) / target_ctas;
   per = std::max<int64_t>(1, per);
+  per = std::max<int64_t>(per, (max_tiles + kMaxParts - 1) / kMaxParts);
   LrPlan pl;
   pl.tiles_per_cta = static_cast<int>(per);
-  pl.splits = static_cast<int>((max_tiles + per - 1) / per);
+  pl.splits = static_cast<int>((max_tiles + per - 1) / per);  // <= kMaxParts
   return pl;
 }
 
@@ -381,7 +473,9 @@ extern "C" size_t mocap_last_row_attn_workspace_size(const int64_t *kv_len, int3
     return 0;
   const size_t splits = static_cast<size_t>(mocap::plan_splits(kv_len, n_req, n_kv_heads).splits);
   const size_t o = splits * n_req * n_q_heads * head_dim * sizeof(float);
-  return (o + 255) / 256 * 256 + splits * n_q_heads * n_req * sizeof(float);
+  const size_t l = splits * n_q_heads * n_req * sizeof(float);
+  return (o + 255) / 256 * 256 + (l + 255) / 256 * 256 +
+         static_cast<size_t>(n_req) * n_kv_heads * sizeof(uint32_t);
 }
 
 extern "C" mocap_status mocap_last_row_attn(const void *q_last, const void *k_cache,
@@ -428,9 +522,15 @@ extern "C" mocap_status mocap_last_row_attn(const void *q_last, const void *k_ca
   const LrPlan plan = plan_splits(kv_len, n_req, n_kv_heads);
   const int splits = plan.splits;
   const size_t o_bytes = static_cast<size_t>(splits) * n_req * n_q_heads * head_dim * sizeof(float);
+  const size_t l_bytes = static_cast<size_t>(splits) * n_q_heads * n_req * sizeof(float);
+  auto *ws = static_cast<uint8_t *>(workspace);
   prm.q = static_cast<const __nv_bfloat16 *>(q_last);
-  prm.o_part = static_cast<float *>(workspace);
-  prm.lse_part = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + (o_bytes + 255) / 256 * 256);
+  prm.o_part = reinterpret_cast<float *>(ws);
+  prm.lse_part = reinterpret_cast<float *>(ws + (o_bytes + 255) / 256 * 256);
+  prm.arrived = reinterpret_cast<uint32_t *>(ws + (o_bytes + 255) / 256 * 256 +
+                                             (l_bytes + 255) / 256 * 256);
+  prm.out = static_cast<__nv_bfloat16 *>(out);
+  prm.lse = lse;
   prm.status = status;
   prm.n_req = n_req;
   prm.n_q_heads = n_q_heads;
@@ -440,6 +540,9 @@ extern "C" mocap_status mocap_last_row_attn(const void *q_last, const void *k_ca
   prm.tiles_per_cta = plan.tiles_per_cta;
   prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
   const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(prm.arrived, 0, static_cast<size_t>(n_req) * n_kv_heads * sizeof(uint32_t),
+                      st) != cudaSuccess)
+    return MOCAP_ECUDA;
   const dim3 grid(splits, n_req, n_kv_heads);
   if (head_dim == 128) {
     static bool attr = false;
@@ -460,7 +563,5 @@ extern "C" mocap_status mocap_last_row_attn(const void *q_last, const void *k_ca
     }
     last_row_kernel<64><<<grid, kThreads, LrLayout<64>::kBytes, st>>>(prm);
   }
-  if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
-  return launch_attn_combine(prm.o_part, prm.lse_part, splits, n_req, n_q_heads, head_dim, out,
-                             lse, n_req, st);
+  return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
 }

@@ -6,6 +6,11 @@
 //   [Q | K | V] = X W^T                     (X [len, hidden], W [Nout, hidden])
 //   Q, K rotated by RoPE at positions offset + r (rotate-half convention:
 //     dims j and j + d/2 of a head turn by pos * theta^(-2j/d))
+//   The angle is formed in integer fixed point, in turns: the host gives
+//   step_j = theta^(-2j/d) / (2 pi) as a 64-bit binary fraction, and
+//   pos * step_j modulo 2^64 is the angle's fraction of a full turn exactly
+//   up to step_j's rounding (2^-64), with no floating-point reduction; its
+//   top 32 bits, read as a signed integer, give the angle in [-pi, pi).
 //   Q -> q_out [len, Hq, d];  K, V -> cache rows [offset, offset + len)
 //
 // Persistent warp-specialised tcgen05 GEMM, one CTA per SM:
@@ -34,7 +39,10 @@ namespace mocap {
 namespace {
 
 constexpr int kBM = 128, kBN = 256, kBK = 64;
-constexpr int kStages = 4;
+#ifndef MOCAP_QKV_STAGES
+#define MOCAP_QKV_STAGES 4
+#endif
+constexpr int kStages = MOCAP_QKV_STAGES;
 constexpr int kThreads = 192;  // 6 warps
 constexpr int kABytes = kBM * kBK * 2;  // 16 KB
 constexpr int kBBytes = kBN * kBK * 2;  // 32 KB
@@ -51,7 +59,7 @@ struct QkvParams {
   int64_t pos0;            // position of row 0
   int32_t len, hidden, n_q_heads, n_kv_heads, head_dim;
   int32_t m_tiles, n_tiles, k_steps;
-  double inv_freq[kMaxHalfDim];  // theta^(-2j/d), host-computed in double
+  uint64_t turn_step[kMaxHalfDim];  // theta^(-2j/d) / (2 pi) * 2^64, rounded down
 };
 
 struct QkvLayout {
@@ -74,8 +82,8 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
 // Epilogue for one head's d columns of one row: RoPE (if `rotate`), bf16,
 // stores.  `taddr` is this lane's TMEM address of the head's first column.
 template <int D>
-__device__ __forceinline__ void emit_head(uint32_t taddr, bool rotate, double pos,
-                                          const double *inv_freq, __nv_bfloat16 *dst,
+__device__ __forceinline__ void emit_head(uint32_t taddr, bool rotate, uint64_t pos,
+                                          const uint64_t *turn_step, __nv_bfloat16 *dst,
                                           bool valid) {
   constexpr int H = D / 2;
 #pragma unroll
@@ -92,11 +100,12 @@ __device__ __forceinline__ void emit_head(uint32_t taddr, bool rotate, double po
     if (rotate) {
 #pragma unroll 4
       for (int e = 0; e < 32; ++e) {
-        // angle reduced to [-pi, pi] in double, then single-precision sincos
-        double ang = pos * inv_freq[c + e];
-        ang -= rint(ang * 0.15915494309189533577) * 6.283185307179586477;
+        // fraction of a turn, modulo 1 by the wrap-around of the product
+        const uint64_t turns = pos * turn_step[c + e];
+        const float ang = static_cast<float>(static_cast<int32_t>(turns >> 32)) *
+                          1.46291807926715968e-9f;  // 2 pi / 2^32
         float sn, cs;
-        __sincosf(static_cast<float>(ang), &sn, &cs);
+        __sincosf(ang, &sn, &cs);
         const float x0 = a[e], x1 = b[e];
         a[e] = x0 * cs - x1 * sn;
         b[e] = x1 * cs + x0 * sn;
@@ -241,7 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1) qkv_rope_kernel(const __grid_cons
       const int mt = t % p.m_tiles, nt = t / p.m_tiles;
       const int row = mt * kBM + row_in_tile;
       const bool valid = row < p.len;
-      const double pos = static_cast<double>(p.pos0 + row);
+      const uint64_t pos = static_cast<uint64_t>(p.pos0 + row);
 #pragma unroll 1
       for (int hs = 0; hs < kBN / D; ++hs) {
         const int col = nt * kBN + hs * D;  // first output feature of this head
@@ -256,7 +265,7 @@ __global__ void __launch_bounds__(kThreads, 1) qkv_rope_kernel(const __grid_cons
                 (static_cast<int64_t>(row) * p.n_kv_heads + (col - q_cols - k_cols) / D) * D;
           rotate = false;
         }
-        emit_head<D>(lane_addr + buf * kBN + hs * D, rotate, pos, p.inv_freq, dst, valid);
+        emit_head<D>(lane_addr + buf * kBN + hs * D, rotate, pos, p.turn_step, dst, valid);
       }
       tc_fence_before();
       __syncwarp();
@@ -358,8 +367,11 @@ extern "C" mocap_status mocap_qkv_rope_append(const void *x, const void *w_qkv, 
   prm.m_tiles = static_cast<int32_t>((len + kBM - 1) / kBM);
   prm.n_tiles = static_cast<int32_t>(n_out / kBN);
   prm.k_steps = (hidden + kBK - 1) / kBK;
-  for (int j = 0; j < head_dim / 2; ++j)
-    prm.inv_freq[j] = std::pow(static_cast<double>(rope_theta), -2.0 * j / head_dim);
+  for (int j = 0; j < head_dim / 2; ++j) {
+    const double turns = std::pow(static_cast<double>(rope_theta), -2.0 * j / head_dim) /
+                         6.283185307179586477;  // < 1/(2 pi): fits below 2^62 once scaled
+    prm.turn_step[j] = static_cast<uint64_t>(std::ldexp(turns, 64));
+  }
 
   const int64_t tiles = static_cast<int64_t>(prm.m_tiles) * prm.n_tiles;
   const int grid = static_cast<int>(std::min<int64_t>(tiles, sm_count_qkv()));

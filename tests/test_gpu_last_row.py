@@ -28,6 +28,7 @@ CASES = [
     ([1, 2, 127, 128, 129, 300, 4097], 8, 2, 128),                    # ragged, tiny
     ([1000, 50], 4, 4, 64),
     ([3000], 16, 1, 128),                                              # group of 16
+    ([int(x) for x in np.random.default_rng(5).integers(1, 2500, 64)], 16, 4, 64),  # 64 requests
 ]
 
 
@@ -74,3 +75,37 @@ def test_last_row_rejects_bad_arguments(m):
         m.mocap_last_row_attn(q, k, k, [0, 60], [50, 50], out, lse, 0.1)
     with pytest.raises(m.MocapError):   # empty request
         m.mocap_last_row_attn(q, k, k, [0, 10], [50, 0], out, lse, 0.1)
+
+
+def test_last_row_workspace_garbage_and_reuse(m):
+    """The per-group arrival counters live in the caller's workspace: the call
+    zeroes them itself, so a workspace full of garbage, and the same workspace
+    reused, give bit-identical results (the merge order does not depend on
+    which CTA finishes last)."""
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(11)
+    lens = [131072, 4096]
+    hq, hkv, d = 64, 8, 128
+    total = sum(lens)
+    k = torch.randn((total, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    v = torch.randn((total, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    q = torch.randn((2, hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    rows = [0, lens[0]]
+    need = m.mocap_last_row_attn_workspace_size(lens, hq, hkv, d)
+    ws = torch.full((need,), 0xFF, device=dev, dtype=torch.uint8)
+    outs = []
+    for _ in range(3):
+        out = torch.empty((2, hq, d), device=dev, dtype=torch.bfloat16)
+        lse = torch.empty((hq, 2), device=dev, dtype=torch.float32)
+        m.mocap_last_row_attn(q, k, v, rows, lens, out, lse, 0.088, workspace=ws)
+        outs.append((out, lse))
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    for out, lse in outs[1:]:
+        assert torch.equal(out.view(torch.int16), outs[0][0].view(torch.int16))
+        assert torch.equal(lse.view(torch.int32), outs[0][1].view(torch.int32))
+    # and the result is the attention of the last row (the oracle, request 1)
+    a = lens[0]
+    o_ref, l_ref = A.chunk_attention(f64(q[1:2]), f64(k[a:]), f64(v[a:]), lens[1] - 1, 0.088)
+    assert_close(outs[0][0][1:2].float().cpu().numpy(), outs[0][1][:, 1:2].cpu().numpy(), o_ref,
+                 l_ref, "request 1")
