@@ -128,8 +128,11 @@ class ChunkedPrefill:
         on a copy stream, in chunk order; the compute stream starts chunk i as
         soon as its rows have landed, and a third stream copies chunk i's O
         and LSE back to ``host_out`` / ``host_lse`` (shaped like ``self.out``
-        and ``self.lse``) as soon as its attention is done.  The caller's
-        current stream waits for everything before this returns."""
+        and ``self.lse``) as soon as its attention is done.  With several
+        requests a chunk's LSE columns are strided in the ``[Hq, T]`` array, so
+        the whole LSE (4 Hq T bytes) goes back in one contiguous copy after the
+        last step instead.  The caller's current stream waits for everything
+        before this returns."""
         compute = torch.cuda.current_stream(self.device)
         h2d = torch.cuda.Stream(self.device)
         d2h = torch.cuda.Stream(self.device)
@@ -148,8 +151,6 @@ class ChunkedPrefill:
                 ev.record(h2d)
                 landed.append(ev)
         d2h.wait_stream(compute)
-        lse2d = None if self.single else self.lse_packed()
-        host_lse2d = None if self.single else host_lse.view(hq, self.w.total_tokens)
         for i, step in enumerate(steps):
             compute.wait_event(landed[i])
             self.run_step(q, k, v, step, compute)
@@ -163,8 +164,10 @@ class ChunkedPrefill:
                     if self.single:
                         host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
                                                         non_blocking=True)
-                    else:
-                        host_lse2d[:, rows].copy_(lse2d[:, rows], non_blocking=True)
+        if not self.single:
+            d2h.wait_stream(compute)
+            with torch.cuda.stream(d2h):
+                host_lse.copy_(self.lse, non_blocking=True)
         compute.wait_stream(d2h)
         compute.wait_stream(h2d)
 
