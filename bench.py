@@ -406,8 +406,7 @@ def ours_arm(args, rank, world, local):
     peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAK_TFLOPS))
     attn_avg_ms = statistics.mean(attn_step_ms)
     achieved = total_flops / (attn_avg_ms * 1e-3) / 1e12
-    launches_per_step = n_chunks  # attention launches
-    traffic_full = ncu_traffic(w.name)
+    traffic_per_launch = ncu_traffic(w.name)
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     app_gbs = append_bytes / (statistics.mean(app_step_ms) * 1e-3) / 1e9
 
@@ -431,7 +430,7 @@ def ours_arm(args, rank, world, local):
                      "frac": achieved / peak,
                      "peak_source": f"bf16_tflops_sustained ({peak_src})",
                      "kernel": "chunk_attn_kernel",
-                     "traffic": None if traffic_full is None else traffic_full / launches_per_step,
+                     "traffic": traffic_per_launch,
                      "traffic_unit": "bytes per launch (avg over the step's launches)"},
         "clocks": clk,
         # our kernels per timed region: one append per (request, chunk), one
