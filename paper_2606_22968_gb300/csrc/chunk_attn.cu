@@ -12,7 +12,12 @@
 //                 through a 4-deep ring of 128-byte-swizzled smem stages.
 //   warp 1        MMA issuer (one thread): S_s = Q_s K_j^T into TMEM, then
 //                 O_s += P_s V_j with P_s read from TMEM; tcgen05.commit
-//                 signals S ready / stage free / O final.
+//                 signals S ready / stage free / O final.  The next tile's
+//                 K/V barriers are checked while a P V half is still queued,
+//                 and V_j is released right after its last MMA, so no wait
+//                 sits between the last MMA of a tile and the first of the
+//                 next (a clock64 trace showed ~640 idle tensor cycles per
+//                 tile there).
 //   warps 4-7     softmax for head slot 0, warps 8-11 for slot 1 (a warp may
 //                 touch only TMEM lanes 32*(warp%4) .. +31).  Thread r
 //                 owns TMEM lane r = query row r, so row max / row sum are
@@ -264,45 +269,51 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
         tc_commit(bar(L::kBarEmpty + 0));
       }
       __syncwarp();
-      for (int j = 0; j < n_kv && ok; ++j) {
-        const int sv = 2 * j + 1;
-        const int sk = 2 * j + 2;
-        const bool has_next = j + 1 < n_kv;
-        ok = wait(L::kBarFull + sv % kStages, sv / kStages);
-        if (ok && has_next) ok = wait(L::kBarFull + sk % kStages, sk / kStages);
+      // tile 0's V and tile 1's K; later tiles' are checked one tile ahead,
+      // while P V MMAs are still queued on the tensor core
+      ok = wait(L::kBarFull + 1, 0);
+      if (ok && n_kv > 1) ok = wait(L::kBarFull + 2 % kStages, 2 / kStages);
+    }
+    for (int j = 0; j < n_kv && ok; ++j) {
+      const int sv = 2 * j + 1;  // V_j
+      const int sk = 2 * j + 2;  // K_{j+1}
+      const bool has_next = j + 1 < n_kv;
+      for (int s = 0; s < nslots; ++s) {
+        // P arrives in two halves (keys 0..63 on kBarP, 64..127 on kBarPHi),
+        // each barrier completing once per tile.
+        ok = wait(L::kBarP + s, j);
         if (!ok) break;
-        for (int s = 0; s < nslots; ++s) {
-          // P arrives in two halves (keys 0..63 on kBarP, 64..127 on kBarPHi),
-          // each barrier completing once per tile.
-          ok = wait(L::kBarP + s, j);
+        tc_fence_after();
+        if (leader)
+          issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
+                           j > 0, 0);
+        __syncwarp();
+        if (s == nslots - 1 && has_next) {
+          // V_{j+1} and K_{j+2}: waited here, with this P V half queued,
+          // rather than at the next tile's start with the queue empty
+          ok = wait(L::kBarFull + (sv + 2) % kStages, (sv + 2) / kStages);
+          if (ok && j + 2 < n_kv) ok = wait(L::kBarFull + (sk + 2) % kStages, (sk + 2) / kStages);
           if (!ok) break;
-          tc_fence_after();
-          if (leader)
-            issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
-                             j > 0, 0);
-          __syncwarp();
-          ok = wait(L::kBarPHi + s, j);
-          if (!ok) break;
-          tc_fence_after();
-          if (leader) {
-            issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
-                             true, 1);
-            if (has_next) {
-              issue_qk<D>(tmem + s * kBlockN, q_desc(s), k_desc(sk % kStages));
-              tc_commit(bar(L::kBarS + s));
-            } else {
-              tc_commit(bar(L::kBarO + s));
-            }
-          }
-          __syncwarp();
         }
+        ok = wait(L::kBarPHi + s, j);
         if (!ok) break;
+        tc_fence_after();
         if (leader) {
-          tc_commit(bar(L::kBarEmpty + sv % kStages));
-          if (has_next) tc_commit(bar(L::kBarEmpty + sk % kStages));
+          issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
+                           true, 1);
+          if (s == nslots - 1) tc_commit(bar(L::kBarEmpty + sv % kStages));  // V_j read
+          if (has_next) {
+            issue_qk<D>(tmem + s * kBlockN, q_desc(s), k_desc(sk % kStages));
+            tc_commit(bar(L::kBarS + s));
+          } else {
+            tc_commit(bar(L::kBarO + s));
+          }
         }
         __syncwarp();
       }
+      if (!ok) break;
+      if (leader && has_next) tc_commit(bar(L::kBarEmpty + sk % kStages));  // K_{j+1} read
+      __syncwarp();
     }
     // Every issued MMA completes before TMEM is released.
     if (leader) {
