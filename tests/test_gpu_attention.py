@@ -224,6 +224,12 @@ def test_workload4_128k_lbcp_sampled(m):
                      chunks=[0, 1, 15, 29, 30, 31])
 
 
+def test_workload4_every_chunk_first_and_last_row(m):
+    # all 32 chunks at full size: each chunk's first row and its last row,
+    # which attends to the whole prefix plus the whole chunk
+    _workload_parity(m, 4, lambda n, i: np.array([0, n - 1]))
+
+
 def test_workload5_varlen_sampled(m):
     from paper_2606_22968_gb300 import workloads
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill

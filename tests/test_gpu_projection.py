@@ -76,3 +76,36 @@ def test_qkv_rope_rejects_bad_shapes(m):
     kc2 = torch.zeros((12, 1, 128), device=dev, dtype=torch.bfloat16)
     with pytest.raises(m.MocapError):   # offset + len past the cache
         m.mocap_qkv_rope_append(x2, w2, q2, kc2, kc2.clone(), 5)
+
+
+@pytest.mark.parametrize("length,offset", [(4096, 61440), (2000, 129024)])
+def test_qkv_rope_full_size_sampled_rows(m, length, offset):
+    """Llama-3-70B projection shapes as the benchmark launches them (hidden
+    8192, 64 + 2 x 8 heads of 128; a 4096-row chunk and a ragged 2000-row one
+    near the end of a 131072-token prompt): sampled rows, including the tile
+    edges of the 256-row pair tiles and the ragged tail, against the oracle
+    row by row (each at its own position)."""
+    from tests.parity_utils import sample_rows
+    hidden, hq, hkv, d, theta = 8192, 64, 8, 128, 500000.0
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(length + offset)
+    x = torch.randn((length, hidden), generator=gen, device=dev).bfloat16()
+    n_out = (hq + 2 * hkv) * d
+    w = (torch.randn((n_out, hidden), generator=gen, device=dev) / math.sqrt(hidden)).bfloat16()
+    cap = offset + length
+    kc = torch.zeros((cap, hkv, d), device=dev, dtype=torch.bfloat16)
+    vc = torch.zeros_like(kc)
+    q = torch.full((length, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    m.mocap_qkv_rope_append(x, w, q, kc, vc, offset, rope_theta=theta)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    rows = sample_rows(length, every=509, edge=2, seed=length)
+    rows = np.unique(np.concatenate([rows, [r for r in (255, 256, 511, 512) if r < length]]))
+    wf = f64(w)
+    for r in rows:
+        q_ref, k_ref, v_ref = R.qkv_rope(f64(x[r:r + 1]), wf, hq, hkv, d, offset + int(r), theta)
+        for got, ref, name in [(q[r:r + 1], q_ref, "Q"), (kc[offset + r:offset + r + 1], k_ref, "K"),
+                               (vc[offset + r:offset + r + 1], v_ref, "V")]:
+            err = np.abs(got.float().cpu().numpy() - ref)
+            assert err.max() <= TOL_MAX and err.mean() <= TOL_MEAN, (name, int(r), err.max(),
+                                                                   err.mean())
