@@ -6,6 +6,13 @@
 // balances.  The kernel computes, for query head h (KV head h / group) and
 // global row t, O_t = softmax_{j<=t}(scale q_t.k_j) V and LSE_t = ln sum exp.
 //
+// Two forms.  CTA pairs (single-item launches, d = 128, a multiple of four
+// query heads per KV group; see control_roles_pair): two CTAs on two SMs
+// share the KV group, row block and keys, each holds two heads, and
+// tcgen05 cta_group::2 MMAs (M = 256) read K and V halves from both CTAs, so
+// each SM stages and each SM's L2 traffic carries half of every K/V tile.
+// Single CTAs (every other shape) as follows.
+//
 // Design (one CTA = 128 query rows x up to two query heads of one KV group;
 // CTAs are ordered KV-group-major, heaviest row block first within a group):
 //   warp 0        TMA producer: Q tiles once, then K_j, V_j tiles (128 keys)
@@ -54,7 +61,6 @@ namespace {
 constexpr int kBlockM = 128;   // query rows per tile = TMEM lanes
 constexpr int kBlockN = 128;   // keys per K/V tile
 constexpr int kMaxSplits = 4;  // key-range splits of one chunk (split-KV)
-constexpr int kStages = 4;     // ring stages, each holds one K or one V tile
 constexpr int kThreads = 384;  // 3 warpgroups: {producer, MMA, 2 idle}, softmax 0, softmax 1
 // Register split (setmaxnreg): the kernel is built for 168 registers per
 // thread (384 x 168 = 64512 <= 65536); warpgroup 0 gives up to 56 and the two
@@ -85,6 +91,7 @@ struct AttnParams {
   CUtensorMap tq[MAXI];  // Q  [len, Hq, D]           box {64, 1, 128}
   CUtensorMap tk[MAXI];  // K  [prefix+len, Hkv, D]   box {64, 1, 128}
   CUtensorMap tv[MAXI];  // V  [prefix+len, Hkv, D]   box {64, 1, 128}
+  CUtensorMap tk_half;   // K of item 0, box {64, 1, 64}: a CTA pair's half K tile
   ItemDesc items[MAXI];
   __nv_bfloat16 *out;
   float *lse;
@@ -105,12 +112,18 @@ struct AttnParams {
   int32_t splits;
 };
 
-template <int D>
+// Shared memory of one CTA.  Single-CTA form: two Q tiles and a ring of four
+// stages, each holding one K or one V tile.  CTA-pair form (PAIR): each CTA
+// stages only its half of every K tile (64 keys) and of every V tile (64
+// dims), so a stage is half as large and the ring eight deep.
+template <int D, bool PAIR = false>
 struct Layout {
-  static constexpr int kTileBytes = kBlockM * D * 2;  // one Q, K or V tile
+  static constexpr int kTileBytes = kBlockM * D * 2;  // one Q tile (one K or V tile)
+  static constexpr int kStages = PAIR ? 8 : 4;
+  static constexpr int kStageBytes = PAIR ? kTileBytes / 2 : kTileBytes;
   static constexpr int kQ = 0;                         // 2 Q tiles
   static constexpr int kRing = 2 * kTileBytes;
-  static constexpr int kBars = kRing + kStages * kTileBytes;
+  static constexpr int kBars = kRing + kStages * kStageBytes;
   // barrier slots (8 bytes each)
   static constexpr int kBarQ = 0;
   static constexpr int kBarFull = 1;               // kStages
@@ -123,8 +136,13 @@ struct Layout {
   static constexpr int kNumBars = 10 + 2 * kStages;
   static constexpr int kTmemSlot = kBars + 8 * kNumBars;
   static constexpr int kFlag = kTmemSlot + 4;
-  static constexpr int kBytes = kFlag + 4 + 1024;  // + slack for 1024-byte alignment
+  // + slack for 1024-byte alignment; a CTA pair also keeps one K/V half of
+  // slack past the barriers, so every MMA operand read stays inside this
+  // CTA's allocation even if it reached past the last stage's half
+  static constexpr int kBytes = kFlag + 4 + 1024 + (PAIR ? kStageBytes : 0);
 };
+static_assert(Layout<128>::kBytes <= 232448, "shared memory");
+static_assert(Layout<128, true>::kBytes <= 232448, "shared memory");
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -218,28 +236,28 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
       bool ok = true;
       int seq = 0;
       for (; seq < n_seq; ++seq) {
-        const int st = seq % kStages;
-        if (seq >= kStages && !mbar_wait(bar(L::kBarEmpty + st), ((seq / kStages) - 1) & 1,
+        const int st = seq % L::kStages;
+        if (seq >= L::kStages && !mbar_wait(bar(L::kBarEmpty + st), ((seq / L::kStages) - 1) & 1,
                                          p.status, kWaitLimitNs, true, kHintProducer)) {
           ok = false;
           break;
         }
-        mbar_arrive_expect_tx(bar(L::kBarFull + st), L::kTileBytes);
+        mbar_arrive_expect_tx(bar(L::kBarFull + st), L::kStageBytes);
         const CUtensorMap *m = (seq & 1) ? mv : mk;
         const int key0 = (t0 + (seq >> 1)) * kBlockN;
         for (int c = 0; c < D / kBoxCols; ++c)
-          tma_load_3d(base + L::kRing + st * L::kTileBytes + c * kBoxBytes, m,
+          tma_load_3d(base + L::kRing + st * L::kStageBytes + c * kBoxBytes, m,
                       bar(L::kBarFull + st), c * kBoxCols, g, key0);
       }
       // Copies still in flight land before the CTA may exit.
       mbar_wait(bar(L::kBarQ), 0, p.status, kDrainLimitNs, false);
-      for (int s2 = max(0, seq - kStages); s2 < seq; ++s2)
-        mbar_wait(bar(L::kBarFull + s2 % kStages), (s2 / kStages) & 1, p.status, kDrainLimitNs,
+      for (int s2 = max(0, seq - L::kStages); s2 < seq; ++s2)
+        mbar_wait(bar(L::kBarFull + s2 % L::kStages), (s2 / L::kStages) & 1, p.status, kDrainLimitNs,
                   false);
       // Normal exit: the last stage releases (tcgen05.commit arrivals) landed.
       if (ok)
-        for (int s2 = max(0, n_seq - kStages); s2 < n_seq; ++s2)
-          if (!mbar_wait(bar(L::kBarEmpty + s2 % kStages), (s2 / kStages) & 1, p.status)) break;
+        for (int s2 = max(0, n_seq - L::kStages); s2 < n_seq; ++s2)
+          if (!mbar_wait(bar(L::kBarEmpty + s2 % L::kStages), (s2 / L::kStages) & 1, p.status)) break;
     }
   } else if (warp == 1) {
     // ===================== MMA issuer =======================================
@@ -272,7 +290,7 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
       // tile 0's V and tile 1's K; later tiles' are checked one tile ahead,
       // while P V MMAs are still queued on the tensor core
       ok = wait(L::kBarFull + 1, 0);
-      if (ok && n_kv > 1) ok = wait(L::kBarFull + 2 % kStages, 2 / kStages);
+      if (ok && n_kv > 1) ok = wait(L::kBarFull + 2 % L::kStages, 2 / L::kStages);
     }
     for (int j = 0; j < n_kv && ok; ++j) {
       const int sv = 2 * j + 1;  // V_j
@@ -285,25 +303,25 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
         if (!ok) break;
         tc_fence_after();
         if (leader)
-          issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
+          issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % L::kStages),
                            j > 0, 0);
         __syncwarp();
         if (s == nslots - 1 && has_next) {
           // V_{j+1} and K_{j+2}: waited here, with this P V half queued,
           // rather than at the next tile's start with the queue empty
-          ok = wait(L::kBarFull + (sv + 2) % kStages, (sv + 2) / kStages);
-          if (ok && j + 2 < n_kv) ok = wait(L::kBarFull + (sk + 2) % kStages, (sk + 2) / kStages);
+          ok = wait(L::kBarFull + (sv + 2) % L::kStages, (sv + 2) / L::kStages);
+          if (ok && j + 2 < n_kv) ok = wait(L::kBarFull + (sk + 2) % L::kStages, (sk + 2) / L::kStages);
           if (!ok) break;
         }
         ok = wait(L::kBarPHi + s, j);
         if (!ok) break;
         tc_fence_after();
         if (leader) {
-          issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % kStages),
+          issue_pv_half<D>(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN, v_desc(sv % L::kStages),
                            true, 1);
-          if (s == nslots - 1) tc_commit(bar(L::kBarEmpty + sv % kStages));  // V_j read
+          if (s == nslots - 1) tc_commit(bar(L::kBarEmpty + sv % L::kStages));  // V_j read
           if (has_next) {
-            issue_qk<D>(tmem + s * kBlockN, q_desc(s), k_desc(sk % kStages));
+            issue_qk<D>(tmem + s * kBlockN, q_desc(s), k_desc(sk % L::kStages));
             tc_commit(bar(L::kBarS + s));
           } else {
             tc_commit(bar(L::kBarO + s));
@@ -312,7 +330,7 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
         __syncwarp();
       }
       if (!ok) break;
-      if (leader && has_next) tc_commit(bar(L::kBarEmpty + sk % kStages));  // K_{j+1} read
+      if (leader && has_next) tc_commit(bar(L::kBarEmpty + sk % L::kStages));  // K_{j+1} read
       __syncwarp();
     }
     // Every issued MMA completes before TMEM is released.
@@ -324,17 +342,188 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
   }
 }
 
+// CTA-pair control roles (d = 128, heads of a KV group taken four at a
+// time: CTA r of the pair holds head slots {h0, h0 + 1} of its own head
+// pair; both CTAs share the KV group, row block and key range).  Per key
+// tile, CTA r stages keys 64 r .. 64 r + 63 of K and dims 64 r .. 64 r + 63
+// of V; the first CTA's warp 1 issues cta_group::2 MMAs:
+//   S_s = Q_s K^T   M = 256 (128 rows of each CTA's slot s), N = 128 keys
+//   O_s += P_s V    M = 256 (P in each CTA's TMEM), N = 128 dims
+// and its commits arrive on both CTAs' barriers.  Both CTAs' copies count on
+// the first CTA's barriers, and so do both CTAs' P arrivals.
+template <int MAXI>
+__device__ __forceinline__ void control_roles_pair(const AttnParams<MAXI> &p, uint32_t base,
+                                                   uint32_t bars, uint32_t tmem, uint32_t warp,
+                                                   uint32_t lane, uint32_t rank, int item, int g,
+                                                   int h0, int r0, int nslots, int t0, int n_kv) {
+  constexpr int D = 128;
+  using L = Layout<D, true>;
+  constexpr int S = L::kStages;
+  auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
+  const bool first = rank == 0;
+  if (warp == 0) {
+    // ===================== TMA producer (both CTAs) =========================
+    if (lane == 0) {
+      const CUtensorMap *mq = &p.tq[item];
+      const CUtensorMap *mk = &p.tk_half;
+      const CUtensorMap *mv = &p.tv[item];
+      prefetch_tmap(mq);
+      prefetch_tmap(mk);
+      prefetch_tmap(mv);
+      const uint32_t q_bar = cluster_addr(bar(L::kBarQ), 0);
+      const uint32_t full0 = cluster_addr(bar(L::kBarFull), 0);
+      if (first) mbar_arrive_expect_tx(bar(L::kBarQ), 2 * nslots * L::kTileBytes);
+      for (int s = 0; s < nslots; ++s)
+        for (int c = 0; c < D / kBoxCols; ++c)
+          tma_load_3d_pair(base + L::kQ + s * L::kTileBytes + c * kBoxBytes, mq, q_bar,
+                           c * kBoxCols, h0 + s, r0);
+      const int n_seq = 2 * n_kv;  // K_0, V_0, K_1, V_1, ...
+      bool ok = true;
+      int seq = 0;
+      for (; seq < n_seq; ++seq) {
+        const int st = seq % S;
+        if (seq >= S && !mbar_wait(bar(L::kBarEmpty + st), ((seq / S) - 1) & 1, p.status,
+                                   kWaitLimitNs, true, kHintProducer)) {
+          ok = false;
+          break;
+        }
+        const uint32_t dst = base + L::kRing + st * L::kStageBytes;
+        const int key0 = (t0 + (seq >> 1)) * kBlockN;
+        if (first) mbar_arrive_expect_tx(bar(L::kBarFull + st), 2 * L::kStageBytes);
+        if ((seq & 1) == 0) {  // K: this CTA's 64 keys, two 64-dim boxes of 8 KB
+          for (int c = 0; c < D / kBoxCols; ++c)
+            tma_load_3d_pair(dst + c * (kBoxBytes / 2), mk, full0 + 8u * st, c * kBoxCols, g,
+                             key0 + 64 * static_cast<int>(rank));
+        } else {  // V: this CTA's 64 dims of all 128 keys, one box of 16 KB
+          tma_load_3d_pair(dst, mv, full0 + 8u * st, 64 * static_cast<int>(rank), g, key0);
+        }
+      }
+      if (ok) {
+        // the last stages' releases (commits after their MMAs) have arrived,
+        // so every copy of this CTA has landed
+        for (int s2 = max(0, n_seq - S); s2 < n_seq; ++s2)
+          if (!mbar_wait(bar(L::kBarEmpty + s2 % S), (s2 / S) & 1, p.status)) break;
+      } else if (first) {
+        // copies still in flight (both CTAs' count here) land before exit
+        mbar_wait(bar(L::kBarQ), 0, p.status, kDrainLimitNs, false);
+        for (int s2 = max(0, seq - S); s2 < seq; ++s2)
+          mbar_wait(bar(L::kBarFull + s2 % S), (s2 / S) & 1, p.status, kDrainLimitNs, false);
+      }
+    }
+  } else if (warp == 1 && first) {
+    // ===================== MMA issuer (first CTA) ===========================
+    const bool leader = elect_one();
+    auto wait = [&](int b, int parity) {
+      return mbar_wait_warp(bar(b), parity & 1, p.status, kHintMma);
+    };
+    constexpr uint32_t idesc_s = idesc_bf16_f32(2 * kBlockM, kBlockN, false, false);
+    constexpr uint32_t idesc_o = idesc_bf16_f32(2 * kBlockM, D, false, true);
+    constexpr uint64_t kTileStep = static_cast<uint64_t>(L::kTileBytes >> 4);
+    constexpr uint64_t kStageStep = static_cast<uint64_t>(L::kStageBytes >> 4);
+    const uint64_t q_desc0 = sdesc_sw128(base + L::kQ, 16, 1024);
+    const uint64_t k_desc0 = sdesc_sw128(base + L::kRing, 16, 1024);
+    // V half: one 64-dim column of 128-byte atoms (no second column)
+    const uint64_t v_desc0 = sdesc_sw128(base + L::kRing, kBoxBytes, 1024);
+    // S_s = Q_s K^T: Q in 128-row boxes of 16 KB, the K half in 64-row boxes of 8 KB
+    auto qk = [&](int s, int st) {
+      const uint64_t qd = q_desc0 + static_cast<uint64_t>(s) * kTileStep;
+      const uint64_t kd = k_desc0 + static_cast<uint64_t>(st) * kStageStep;
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint64_t qo = static_cast<uint64_t>(((kk / 4) * kBoxBytes + (kk % 4) * 32) >> 4);
+        const uint64_t ko =
+            static_cast<uint64_t>(((kk / 4) * (kBoxBytes / 2) + (kk % 4) * 32) >> 4);
+        mma_pair(tmem + s * kBlockN, qd + qo, kd + ko, idesc_s, kk > 0 ? 1u : 0u);
+      }
+    };
+    // half h of O_s += P_s V: keys 64h .. 64h+63 (four K=16 steps of 2 KB)
+    auto pv_half = [&](int s, int st, bool accumulate, int h) {
+      const uint64_t vd = v_desc0 + static_cast<uint64_t>(st) * kStageStep;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int kk = 4 * h + k;
+        mma_ts_pair(tmem + 2 * kBlockN + s * D, tmem + s * kBlockN + kk * 8,
+                    vd + static_cast<uint64_t>((kk * 2048) >> 4), idesc_o,
+                    (accumulate || k > 0) ? 1u : 0u);
+      }
+    };
+    bool ok = wait(L::kBarQ, 0) && wait(L::kBarFull + 0, 0);
+    if (ok) {
+      tc_fence_after();
+      if (leader) {
+        for (int s = 0; s < nslots; ++s) {
+          qk(s, 0);
+          commit_pair(bar(L::kBarS + s), 0x3);
+        }
+        commit_pair(bar(L::kBarEmpty + 0), 0x3);
+      }
+      __syncwarp();
+      ok = wait(L::kBarFull + 1, 0);
+      if (ok && n_kv > 1) ok = wait(L::kBarFull + 2 % S, 2 / S);
+    }
+    for (int j = 0; j < n_kv && ok; ++j) {
+      const int sv = 2 * j + 1;  // V_j
+      const int sk = 2 * j + 2;  // K_{j+1}
+      const bool has_next = j + 1 < n_kv;
+      for (int s = 0; s < nslots; ++s) {
+        ok = wait(L::kBarP + s, j);  // both CTAs' keys 0..63 of P
+        if (!ok) break;
+        tc_fence_after();
+        if (leader) pv_half(s, sv % S, j > 0, 0);
+        __syncwarp();
+        if (s == nslots - 1 && has_next) {  // V_{j+1}, K_{j+2} with this P V half queued
+          ok = wait(L::kBarFull + (sv + 2) % S, (sv + 2) / S);
+          if (ok && j + 2 < n_kv) ok = wait(L::kBarFull + (sk + 2) % S, (sk + 2) / S);
+          if (!ok) break;
+        }
+        ok = wait(L::kBarPHi + s, j);
+        if (!ok) break;
+        tc_fence_after();
+        if (leader) {
+          pv_half(s, sv % S, true, 1);
+          if (s == nslots - 1) commit_pair(bar(L::kBarEmpty + sv % S), 0x3);  // V_j read
+          if (has_next) {
+            qk(s, sk % S);
+            commit_pair(bar(L::kBarS + s), 0x3);
+          } else {
+            commit_pair(bar(L::kBarO + s), 0x3);
+          }
+        }
+        __syncwarp();
+      }
+      if (!ok) break;
+      if (leader && has_next) commit_pair(bar(L::kBarEmpty + sk % S), 0x3);  // K_{j+1} read
+      __syncwarp();
+    }
+    // Every issued MMA completes before TMEM is released.
+    if (leader) {
+      commit_pair(bar(L::kBarDrain), 0x1);
+      mbar_wait(bar(L::kBarDrain), 0, p.status, kDrainLimitNs, false);
+    }
+    __syncwarp();
+  }
+}
+
 // Warpgroups 1 and 2: online softmax for head slot (warp - 4) / 4, then the
 // epilogue (O / l -> bf16, LSE).
-template <int D, int MAXI>
+template <int D, int MAXI, bool PAIR = false>
 __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t bars,
                                              uint32_t tmem, uint32_t warp, uint32_t lane,
                                              const ItemDesc &it, int h0, int r0, int nslots,
                                              int split, int t0, int n_kv, int qpos0,
                                              int n_unmasked) {
-  using L = Layout<D>;
+  using L = Layout<D, PAIR>;
   auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
   const int s = static_cast<int>(warp - 4) / 4;
+  // P-ready arrivals go to the barriers of the CTA that issues the MMAs:
+  // this CTA, or the first CTA of a pair
+  auto arrive_p = [&](int b) {
+    if constexpr (PAIR) {
+      mbar_arrive_cluster(cluster_addr(bar(b), 0));
+    } else {
+      mbar_arrive(bar(b));
+    }
+  };
   if (s < nslots) {
     const uint32_t quarter = warp & 3u;
     const int row = static_cast<int>(quarter * 32 + lane);
@@ -402,7 +591,7 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
           tmem_st_wait();
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(bar(L::kBarP + s));
+          if (lane == 0) arrive_p(L::kBarP + s);
         }
       }
       float sum0, sum1, sum2, sum3, sum4, sum5, sum6, sum7;
@@ -416,7 +605,7 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(bar(L::kBarPHi + s));
+      if (lane == 0) arrive_p(L::kBarPHi + s);
     }
     if (ok) ok = mbar_wait_warp(bar(L::kBarO + s), 0, p.status);
     if (ok && p.splits > 1) {
@@ -478,10 +667,10 @@ __device__ __forceinline__ void cta_barrier() {
   asm volatile("barrier.sync 1, %0;" ::"n"(kThreads) : "memory");
 }
 
-template <int D, int MAXI>
+template <int D, int MAXI, bool PAIR = false>
 __global__ void __launch_bounds__(kThreads, 1)
     chunk_attn_kernel(const __grid_constant__ AttnParams<MAXI> p) {
-  using L = Layout<D>;
+  using L = Layout<D, PAIR>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -494,10 +683,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t warp = threadIdx.x >> 5;
   const uint32_t lane = threadIdx.x & 31u;
 
-  // A launch after an expired wait does nothing (CTA-uniform decision).
+  // A launch after an expired wait does nothing (CTA-uniform decision; a
+  // CTA pair takes its first CTA's reading after the set-up below, since
+  // both CTAs must allocate TMEM together).
   if (threadIdx.x == 0) *flag = *reinterpret_cast<volatile uint32_t *>(p.status);
   __syncthreads();
-  if (*flag != 0u) return;
+  if (!PAIR && *flag != 0u) return;
 
   // ---- work item --------------------------------------------------------
   int item = 0;
@@ -546,44 +737,76 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---- setup --------------------------------------------------------------
   if (warp == 1) {
-    tmem_alloc(base + L::kTmemSlot, kTmemCols);
-    tmem_relinquish();
+    if constexpr (PAIR) {
+      tmem_alloc_pair(base + L::kTmemSlot, kTmemCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(base + L::kTmemSlot, kTmemCols);
+      tmem_relinquish();
+    }
   }
   if (threadIdx.x == 0) {
     mbar_init(bar(L::kBarQ), 1);
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < L::kStages; ++s) {
       mbar_init(bar(L::kBarFull + s), 1);
       mbar_init(bar(L::kBarEmpty + s), 1);
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(bar(L::kBarS + s), 1);
-      mbar_init(bar(L::kBarP + s), 4);  // one arrive per softmax warp
+      mbar_init(bar(L::kBarP + s), PAIR ? 8 : 4);  // one arrive per softmax warp (both CTAs')
       mbar_init(bar(L::kBarO + s), 1);
     }
     mbar_init(bar(L::kBarDrain), 1);
-    for (int s = 0; s < 2; ++s) mbar_init(bar(L::kBarPHi + s), 4);
+    for (int s = 0; s < 2; ++s) mbar_init(bar(L::kBarPHi + s), PAIR ? 8 : 4);
     fence_mbar_init();
   }
   tc_fence_before();
-  __syncthreads();
+  if constexpr (PAIR) {
+    cluster_barrier();  // both CTAs' barriers exist before any copy, commit or remote arrive
+  } else {
+    __syncthreads();
+  }
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  if (warp < 4) {
-    setmaxnreg_dec<kRegsControl>();
-    control_roles<D, MAXI>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, t0,
-                           n_kv);
+  if constexpr (PAIR) {
+    const uint32_t rank = cta_rank_in_cluster();
+    const bool run = ld_shared_cluster_u32(cluster_addr(smem_u32(const_cast<uint32_t *>(flag)), 0)) == 0u;
+    if (run) {
+      if (warp < 4) {
+        setmaxnreg_dec<kRegsControl>();
+        control_roles_pair<MAXI>(p, base, bar(0), tmem, warp, lane, rank, item, g, h0, r0, nslots,
+                                 t0, n_kv);
+      } else {
+        setmaxnreg_inc<kRegsSoftmax>();
+        softmax_role<D, MAXI, true>(p, bar(0), tmem, warp, lane, it, h0, r0, nslots, split, t0,
+                                    n_kv, qpos0, n_unmasked);
+      }
+    }
     tc_fence_before();
-    cta_barrier();
+    cluster_barrier();  // MMAs drained, softmax and copies done in both CTAs
     if (warp == 1) {
       tc_fence_after();
-      tmem_dealloc(tmem, kTmemCols);
+      tmem_dealloc_pair(tmem, kTmemCols);
     }
+    cluster_barrier();  // neither CTA leaves while the pair still shares state
   } else {
-    setmaxnreg_inc<kRegsSoftmax>();
-    softmax_role<D, MAXI>(p, bar(0), tmem, warp, lane, it, h0, r0, nslots, split, t0, n_kv, qpos0,
-                          n_unmasked);
-    tc_fence_before();
-    cta_barrier();
+    if (warp < 4) {
+      setmaxnreg_dec<kRegsControl>();
+      control_roles<D, MAXI>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, t0,
+                             n_kv);
+      tc_fence_before();
+      cta_barrier();
+      if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+      }
+    } else {
+      setmaxnreg_inc<kRegsSoftmax>();
+      softmax_role<D, MAXI>(p, bar(0), tmem, warp, lane, it, h0, r0, nslots, split, t0, n_kv,
+                            qpos0, n_unmasked);
+      tc_fence_before();
+      cta_barrier();
+    }
   }
 }
 
@@ -654,15 +877,17 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// [rows, heads, d] bf16 tensor, box = 64 columns x 1 head x 128 rows, 128B swizzle.
-bool make_map(CUtensorMap *map, const void *ptr, int64_t rows, int heads, int d) {
+// [rows, heads, d] bf16 tensor, box = 64 columns x 1 head x box_rows rows,
+// 128B swizzle.
+bool make_map(CUtensorMap *map, const void *ptr, int64_t rows, int heads, int d,
+              int box_rows = kBlockM) {
   auto fn = encode_fn();
   if (fn == nullptr) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(heads),
                         static_cast<cuuint64_t>(rows)};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2,
                            static_cast<cuuint64_t>(heads) * static_cast<cuuint64_t>(d) * 2};
-  cuuint32_t box[3] = {static_cast<cuuint32_t>(kBoxCols), 1u, static_cast<cuuint32_t>(kBlockM)};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(kBoxCols), 1u, static_cast<cuuint32_t>(box_rows)};
   cuuint32_t elem[3] = {1u, 1u, 1u};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box,
             elem, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -756,6 +981,14 @@ int choose_splits(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads, in
   return best;
 }
 
+// CTA pairs (cta_group::2) serve single-item launches with d = 128 and a
+// multiple of four query heads per KV group.  MOCAP_ATTN_PAIR=0 selects the
+// single-CTA kernel for every shape (tests compare the two).
+bool pair_enabled() {
+  const char *env = std::getenv("MOCAP_ATTN_PAIR");
+  return env == nullptr || std::atoi(env) != 0;
+}
+
 template <int D, int MAXI>
 mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
                     const std::vector<HostItem> &items, int64_t lse_stride, const Shape &sh,
@@ -810,20 +1043,55 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     prm.lse_part = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + sp.lse_off);
   }
 
-  auto kern = chunk_attn_kernel<D, MAXI>;
-  static bool attr_done[64] = {};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
-  if (!attr_done[dev]) {
+  // one-time per kernel and device: register count check, shared-memory size
+  auto prepare = [&](auto kern, int smem, bool *done) -> mocap_status {
+    if (done[dev]) return MOCAP_OK;
     cudaFuncAttributes fa{};
     if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) return MOCAP_ECUDA;
     if (fa.numRegs != kLaunchRegs) return MOCAP_EUNSUPPORTED;  // split would not balance
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes) !=
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
         cudaSuccess)
       return MOCAP_ECUDA;
-    attr_done[dev] = true;
+    done[dev] = true;
+    return MOCAP_OK;
+  };
+  bool launched = false;
+  if constexpr (D == 128 && MAXI == 1) {
+    if (pair_enabled() && group % 4 == 0 && ctas % 2 == 0) {
+      const HostItem &h = items[0];
+      const auto *kb = static_cast<const uint8_t *>(k_cache) + h.kv_row * kvrow_bytes;
+      if (!make_map(&prm.tk_half, kb, h.prefix + h.len, sh.n_kv_heads, D, kBlockN / 2))
+        return MOCAP_ECUDA;
+      using LP = Layout<D, true>;
+      auto kern = chunk_attn_kernel<D, MAXI, true>;
+      static bool done[64] = {};
+      const mocap_status st = prepare(kern, LP::kBytes, done);
+      if (st != MOCAP_OK) return st;
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(static_cast<unsigned>(ctas));
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = LP::kBytes;
+      cfg.stream = stream;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 2;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      if (cudaLaunchKernelEx(&cfg, kern, prm) != cudaSuccess) return MOCAP_ECUDA;
+      launched = true;
+    }
   }
-  kern<<<static_cast<unsigned>(ctas), kThreads, L::kBytes, stream>>>(prm);
+  if (!launched) {
+    auto kern = chunk_attn_kernel<D, MAXI>;
+    static bool done[64] = {};
+    const mocap_status st = prepare(kern, L::kBytes, done);
+    if (st != MOCAP_OK) return st;
+    kern<<<static_cast<unsigned>(ctas), kThreads, L::kBytes, stream>>>(prm);
+  }
   if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
   if (sp.splits > 1) {
     const int64_t len = items[0].len;

@@ -350,3 +350,48 @@ def test_graph_replay_matches_eager_run(m, index):
         assert m.mocap_last_device_status() == 0
         assert torch.equal(pf.out, out_ref) and torch.equal(pf.lse, lse_ref)
         assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
+
+
+PAIR_CASES = [
+    # (prefix, len, Hq, Hkv, d, forced splits or None): shapes the CTA-pair
+    # kernel serves (d = 128, a multiple of four query heads per KV group)
+    (0, 300, 8, 2, 128, None),             # 4:1, ragged, no prefix
+    (1000, 129, 16, 2, 128, None),         # 8:1, one row past a tile
+    (61440 + 77, 700, 64, 8, 128, None),   # Llama-3-70B heads, unaligned prefix
+    (100000, 256, 8, 2, 128, None),        # the library splits the key range
+    (200, 2000, 8, 2, 128, 3),             # three forced splits
+]
+
+
+@pytest.mark.parametrize("prefix,length,hq,hkv,d,forced", PAIR_CASES)
+def test_cta_pair_matches_single_cta_and_oracle(m, monkeypatch, prefix, length, hq, hkv, d,
+                                                forced):
+    """The CTA-pair kernel (tcgen05 cta_group::2: K and V halves in each CTA
+    of a pair) against the single-CTA kernel (MOCAP_ATTN_PAIR=0) and both
+    against the oracle."""
+    if forced is not None:
+        monkeypatch.setenv("MOCAP_SPLIT_KV", str(forced))
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(prefix + length + hq)
+    s = prefix + length
+    q = _randn((length, hq, d), gen, dev)
+    k, v = _randn((s, hkv, d), gen, dev), _randn((s, hkv, d), gen, dev)
+    scale = 1.0 / math.sqrt(d)
+    ws_bytes = m.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d)
+    ws = torch.empty((max(ws_bytes, 16),), device=dev, dtype=torch.uint8)
+    outs = []
+    for pair in ("1", "0"):
+        monkeypatch.setenv("MOCAP_ATTN_PAIR", pair)
+        o = torch.full((length, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+        lse = torch.full((hq, length), float("nan"), device=dev, dtype=torch.float32)
+        m.mocap_chunk_attn(q, k, v, prefix, o, lse, scale, workspace=ws)
+        torch.cuda.synchronize()
+        assert m.mocap_last_device_status() == 0
+        outs.append((o, lse))
+    rows = np.arange(length) if length <= 512 else sample_rows(length, every=37)
+    idx = torch.as_tensor(rows, device=dev)
+    o_ref, l_ref = chunk_rows_oracle(f64(q[idx]), f64(k), f64(v), prefix, rows, scale)
+    for (o, lse), name in zip(outs, ("pair", "single")):
+        assert_close(o[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref, l_ref, name)
+    assert (outs[0][0].float() - outs[1][0].float()).abs().max().item() <= 1e-2
+    assert (outs[0][1] - outs[1][1]).abs().max().item() <= 1e-4
