@@ -89,9 +89,8 @@ struct ItemDesc {
 template <int MAXI>
 struct AttnParams {
   CUtensorMap tq[MAXI];  // Q  [len, Hq, D]           box {64, 1, 128}
-  CUtensorMap tk[MAXI];  // K  [prefix+len, Hkv, D]   box {64, 1, 128}
+  CUtensorMap tk[MAXI];  // K  [prefix+len, Hkv, D]   box {64, 1, 128} ({64, 1, 64}: CTA pairs)
   CUtensorMap tv[MAXI];  // V  [prefix+len, Hkv, D]   box {64, 1, 128}
-  CUtensorMap tk_half;   // K of item 0, box {64, 1, 64}: a CTA pair's half K tile
   ItemDesc items[MAXI];
   __nv_bfloat16 *out;
   float *lse;
@@ -365,7 +364,7 @@ __device__ __forceinline__ void control_roles_pair(const AttnParams<MAXI> &p, ui
     // ===================== TMA producer (both CTAs) =========================
     if (lane == 0) {
       const CUtensorMap *mq = &p.tq[item];
-      const CUtensorMap *mk = &p.tk_half;
+      const CUtensorMap *mk = &p.tk[item];  // 64-row boxes: this CTA's half K tile
       const CUtensorMap *mv = &p.tv[item];
       prefetch_tmap(mq);
       prefetch_tmap(mk);
@@ -515,16 +514,18 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
   using L = Layout<D, PAIR>;
   auto bar = [&](int i) -> uint32_t { return bars + 8u * static_cast<uint32_t>(i); };
   const int s = static_cast<int>(warp - 4) / 4;
-  // P-ready arrivals go to the barriers of the CTA that issues the MMAs:
-  // this CTA, or the first CTA of a pair
-  auto arrive_p = [&](int b) {
-    if constexpr (PAIR) {
-      mbar_arrive_cluster(cluster_addr(bar(b), 0));
-    } else {
-      mbar_arrive(bar(b));
-    }
-  };
   if (s < nslots) {
+    // P-ready arrivals go to the barriers of the CTA that issues the MMAs:
+    // this CTA, or the first CTA of a pair
+    const uint32_t p_lo = PAIR ? cluster_addr(bar(L::kBarP + s), 0) : bar(L::kBarP + s);
+    const uint32_t p_hi = PAIR ? cluster_addr(bar(L::kBarPHi + s), 0) : bar(L::kBarPHi + s);
+    auto arrive_p = [&](uint32_t b) {
+      if constexpr (PAIR) {
+        mbar_arrive_cluster(b);
+      } else {
+        mbar_arrive(b);
+      }
+    };
     const uint32_t quarter = warp & 3u;
     const int row = static_cast<int>(quarter * 32 + lane);
     const uint32_t lane_addr = tmem + ((quarter * 32u) << 16);
@@ -591,7 +592,7 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
           tmem_st_wait();
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) arrive_p(L::kBarP + s);
+          if (lane == 0) arrive_p(p_lo);
         }
       }
       float sum0, sum1, sum2, sum3, sum4, sum5, sum6, sum7;
@@ -605,7 +606,7 @@ __device__ __forceinline__ void softmax_role(const AttnParams<MAXI> &p, uint32_t
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) arrive_p(L::kBarPHi + s);
+      if (lane == 0) arrive_p(p_hi);
     }
     if (ok) ok = mbar_wait_warp(bar(L::kBarO + s), 0, p.status);
     if (ok && p.splits > 1) {
@@ -981,9 +982,9 @@ int choose_splits(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads, in
   return best;
 }
 
-// CTA pairs (cta_group::2) serve single-item launches with d = 128 and a
-// multiple of four query heads per KV group.  MOCAP_ATTN_PAIR=0 selects the
-// single-CTA kernel for every shape (tests compare the two).
+// CTA pairs (cta_group::2) serve d = 128 with a multiple of four query heads
+// per KV group.  MOCAP_ATTN_PAIR=0 selects the single-CTA kernel for every
+// shape (tests compare the two).
 bool pair_enabled() {
   const char *env = std::getenv("MOCAP_ATTN_PAIR");
   return env == nullptr || std::atoi(env) != 0;
@@ -1005,6 +1006,8 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
   const int pairs = (group + 1) / 2;
   int64_t ctas = 0;
   int n = 0;
+  // CTA pairs need an even number of head pairs per KV group
+  const bool pair = D == 128 && group % 4 == 0 && pair_enabled();
   const size_t qrow_bytes = static_cast<size_t>(sh.n_q_heads) * D * 2;
   const size_t kvrow_bytes = static_cast<size_t>(sh.n_kv_heads) * D * 2;
   for (const HostItem &h : items) {
@@ -1012,7 +1015,8 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     const auto *kb = static_cast<const uint8_t *>(k_cache) + h.kv_row * kvrow_bytes;
     const auto *vb = static_cast<const uint8_t *>(v_cache) + h.kv_row * kvrow_bytes;
     if (!make_map(&prm.tq[n], qb, h.len, sh.n_q_heads, D) ||
-        !make_map(&prm.tk[n], kb, h.prefix + h.len, sh.n_kv_heads, D) ||
+        !make_map(&prm.tk[n], kb, h.prefix + h.len, sh.n_kv_heads, D,
+                  pair ? kBlockN / 2 : kBlockN) ||
         !make_map(&prm.tv[n], vb, h.prefix + h.len, sh.n_kv_heads, D))
       return MOCAP_ECUDA;
     ItemDesc &d = prm.items[n];
@@ -1058,12 +1062,9 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     return MOCAP_OK;
   };
   bool launched = false;
-  if constexpr (D == 128 && MAXI == 1) {
-    if (pair_enabled() && group % 4 == 0 && ctas % 2 == 0) {
-      const HostItem &h = items[0];
-      const auto *kb = static_cast<const uint8_t *>(k_cache) + h.kv_row * kvrow_bytes;
-      if (!make_map(&prm.tk_half, kb, h.prefix + h.len, sh.n_kv_heads, D, kBlockN / 2))
-        return MOCAP_ECUDA;
+  if constexpr (D == 128) {
+    if (pair) {
+      if (ctas % 2 != 0) return MOCAP_EINVAL;  // whole pairs by construction
       using LP = Layout<D, true>;
       auto kern = chunk_attn_kernel<D, MAXI, true>;
       static bool done[64] = {};
