@@ -41,7 +41,11 @@ def test_expired_wait_is_reported_and_cleared(m):
     assert m.mocap_last_device_status() == m.MOCAP_OK  # read clears it
 
 
-def test_launch_after_expired_wait_does_nothing_then_recovers(m):
+@pytest.mark.parametrize("pair", ["1", "0"])
+def test_launch_after_expired_wait_does_nothing_then_recovers(m, monkeypatch, pair):
+    # both attention forms: CTA pairs (both CTAs act on the first CTA's
+    # reading of the status word) and single CTAs
+    monkeypatch.setenv("MOCAP_ATTN_PAIR", pair)
     dev = torch.device("cuda")
     q, k, v = _small(dev)
     out = torch.full_like(q, float("nan"))
