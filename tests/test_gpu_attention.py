@@ -395,3 +395,36 @@ def test_cta_pair_matches_single_cta_and_oracle(m, monkeypatch, prefix, length, 
         assert_close(o[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref, l_ref, name)
     assert (outs[0][0].float() - outs[1][0].float()).abs().max().item() <= 1e-2
     assert (outs[0][1] - outs[1][1]).abs().max().item() <= 1e-4
+
+
+@pytest.mark.parametrize("hq,hkv,d", [(8, 2, 128), (4, 4, 64)])
+def test_varlen_64_items_and_the_limit(m, hq, hkv, d):
+    """The most items one varlen launch takes (64), with ragged lengths and
+    prefixes (the CTA-pair path at d = 128, GQA 4:1; the single-CTA path at
+    d = 64, 1:1), every element against the oracle; 65 items are refused."""
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(64 + d)
+    rng = np.random.default_rng(64 + d)
+    lens = [int(x) for x in rng.integers(1, 200, 64)]
+    prefixes = [int(x) for x in rng.integers(0, 300, 64)]
+    q_off = np.concatenate([[0], np.cumsum(lens)]).tolist()
+    kv_off = np.concatenate([[0], np.cumsum([p + n for p, n in zip(prefixes, lens)])]).tolist()
+    q = _randn((q_off[-1], hq, d), gen, dev)
+    k = _randn((kv_off[-1], hkv, d), gen, dev)
+    v = _randn((kv_off[-1], hkv, d), gen, dev)
+    out = torch.full((q_off[-1], hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    lse = torch.full((hq, q_off[-1]), float("nan"), device=dev, dtype=torch.float32)
+    items = [(q_off[i], kv_off[i], prefixes[i], lens[i]) for i in range(64)]
+    scale = 1.0 / math.sqrt(d)
+    m.mocap_chunk_attn_varlen(q, k, v, items, out, lse, scale)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    for i in range(64):
+        a, n, kv, pre = q_off[i], lens[i], kv_off[i], prefixes[i]
+        rows = np.arange(n)
+        o_ref, l_ref = chunk_rows_oracle(f64(q[a:a + n]), f64(k[kv:kv + pre + n]),
+                                         f64(v[kv:kv + pre + n]), pre, rows, scale)
+        assert_close(out[a:a + n].float().cpu().numpy(), lse[:, a:a + n].cpu().numpy(), o_ref,
+                     l_ref, f"item {i}")
+    with pytest.raises(m.MocapError):
+        m.mocap_chunk_attn_varlen(q, k, v, items + [items[0]], out, lse, scale)
