@@ -93,13 +93,15 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       : "memory");
 }
 
-// Split-KV merge of one (request, group) by one CTA, in shared memory below
-// the `red` area (the drained K/V ring, Q_g and P regions):
-//   1. the parts' LSEs, w[k][h] for k < n_parts, h < 16;
-//   2. per head the maximum M_h (one warp per head, lanes over the parts);
-//   3. w[k][h] = exp(LSE_kh - M_h) and their sums W_h;
-//   4. each thread owns (head, 4 dims) pairs and sums w * O_k over the parts
-//      with eight independent loads in flight, then scales by 1 / W_h.
+// Split-KV merge of one (request, group) by one CTA, with the weights in
+// shared memory below the `red` area (the drained K/V ring, Q_g and P):
+//   1. one warp per head reads the parts' LSEs (lanes over the parts),
+//      takes their maximum M_h, and keeps w[k][h] = exp(LSE_kh - M_h) and
+//      their sum W_h;
+//   2. each thread owns (head, 4 dims) pairs and sums w * O_k over the parts,
+//      eight parts at a time, then scales by 1 / W_h.  With exactly two
+//      pairs per thread (8 heads at d = 128, 16 at d = 64) both pairs' loads
+//      go out together, sixteen in flight per thread.
 // Every merged part holds at least one key, so each LSE_kh is finite.
 template <int D>
 __device__ __forceinline__ void merge_group(const LastRowParams &p, uint8_t *sm, int r, int g,
@@ -111,28 +113,21 @@ __device__ __forceinline__ void merge_group(const LastRowParams &p, uint8_t *sm,
   float *w = reinterpret_cast<float *>(sm);   // [n_parts][16]
   float *mh = w + kMaxParts * kMaxGroup;      // [16]
   float *wh = mh + kMaxGroup;                 // [16]
-  const int n_items = n_parts * kMaxGroup;
-  for (int i0 = t; i0 < n_items; i0 += 4 * kThreads) {
-    float v[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int i = i0 + u * kThreads, k = i / kMaxGroup, h = i % kMaxGroup;
-      v[u] = i < n_items && h < G
-                 ? __ldcg(p.lse_part + (static_cast<int64_t>(k) * Hq + g * G + h) * p.n_req + r)
-                 : 0.0f;
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-      if (i0 + u * kThreads < n_items) w[i0 + u * kThreads] = v[u];
-  }
-  __syncthreads();
   for (int h = warp; h < G; h += kThreads / 32) {
+    const float *lse_h = p.lse_part + static_cast<int64_t>(g * G + h) * p.n_req + r;
+    const int64_t part_step = static_cast<int64_t>(Hq) * p.n_req;
     float m = -INFINITY;
-    for (int k = lane; k < n_parts; k += 32) m = fmaxf(m, w[k * kMaxGroup + h]);
+    for (int k = lane; k < n_parts; k += 64) {  // two independent loads per lane and round
+      const float a = __ldcg(lse_h + k * part_step);
+      const float b = k + 32 < n_parts ? __ldcg(lse_h + (k + 32) * part_step) : -INFINITY;
+      w[k * kMaxGroup + h] = a;
+      if (k + 32 < n_parts) w[(k + 32) * kMaxGroup + h] = b;
+      m = fmaxf(m, fmaxf(a, b));
+    }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
     float sum = 0.0f;
-    for (int k = lane; k < n_parts; k += 32) {
+    for (int k = lane; k < n_parts; k += 32) {  // entries this lane wrote itself
       const float e = expf(w[k * kMaxGroup + h] - m);
       w[k * kMaxGroup + h] = e;
       sum += e;
@@ -147,9 +142,51 @@ __device__ __forceinline__ void merge_group(const LastRowParams &p, uint8_t *sm,
   __syncthreads();
   const float4 *o4 = reinterpret_cast<const float4 *>(p.o_part);
   const int64_t part_stride = static_cast<int64_t>(p.n_req) * Hq * kCols;  // float4s per part
+  auto src_of = [&](int h, int c) {
+    return o4 + (static_cast<int64_t>(r) * Hq + g * G + h) * kCols + c;
+  };
+  auto store = [&](int h, int c, float4 acc) {
+    const float inv = 1.0f / wh[h];
+    const int head = g * G + h;
+    __nv_bfloat162 *dst = reinterpret_cast<__nv_bfloat162 *>(
+        p.out + (static_cast<int64_t>(r) * Hq + head) * D + 4 * c);
+    dst[0] = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+    dst[1] = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+    if (c == 0) p.lse[static_cast<int64_t>(head) * p.n_req + r] = mh[h] + logf(wh[h]);
+  };
+  auto fma4 = [](float4 &acc, float wk, const float4 &v) {
+    acc.x += wk * v.x;
+    acc.y += wk * v.y;
+    acc.z += wk * v.z;
+    acc.w += wk * v.w;
+  };
+  if (G * kCols == 2 * kThreads) {
+    // pairs t and t + kThreads: same dims, heads h0 and h0 + kThreads / kCols
+    const int c = t % kCols, h0 = t / kCols, h1 = h0 + kThreads / kCols;
+    const float4 *s0 = src_of(h0, c), *s1 = src_of(h1, c);
+    float4 a0 = make_float4(0.0f, 0.0f, 0.0f, 0.0f), a1 = a0;
+    for (int k0 = 0; k0 < n_parts; k0 += 8) {
+      float4 v0[8], v1[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const bool in = k0 + u < n_parts;
+        v0[u] = in ? __ldcg(s0 + (k0 + u) * part_stride) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        v1[u] = in ? __ldcg(s1 + (k0 + u) * part_stride) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const bool in = k0 + u < n_parts;
+        fma4(a0, in ? w[(k0 + u) * kMaxGroup + h0] : 0.0f, v0[u]);
+        fma4(a1, in ? w[(k0 + u) * kMaxGroup + h1] : 0.0f, v1[u]);
+      }
+    }
+    store(h0, c, a0);
+    store(h1, c, a1);
+    return;
+  }
   for (int pair = t; pair < G * kCols; pair += kThreads) {
     const int h = pair / kCols, c = pair % kCols;
-    const float4 *src = o4 + (static_cast<int64_t>(r) * Hq + g * G + h) * kCols + c;
+    const float4 *src = src_of(h, c);
     float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
     for (int k0 = 0; k0 < n_parts; k0 += 8) {
       float4 v[8];
@@ -158,21 +195,9 @@ __device__ __forceinline__ void merge_group(const LastRowParams &p, uint8_t *sm,
         v[u] = k0 + u < n_parts ? __ldcg(src + (k0 + u) * part_stride)
                                 : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const float wk = k0 + u < n_parts ? w[(k0 + u) * kMaxGroup + h] : 0.0f;
-        acc.x += wk * v[u].x;
-        acc.y += wk * v[u].y;
-        acc.z += wk * v[u].z;
-        acc.w += wk * v[u].w;
-      }
+      for (int u = 0; u < 8; ++u) fma4(acc, k0 + u < n_parts ? w[(k0 + u) * kMaxGroup + h] : 0.0f, v[u]);
     }
-    const float inv = 1.0f / wh[h];
-    const int head = g * G + h;
-    __nv_bfloat162 *dst =
-        reinterpret_cast<__nv_bfloat162 *>(p.out + (static_cast<int64_t>(r) * Hq + head) * D + 4 * c);
-    dst[0] = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-    dst[1] = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-    if (c == 0) p.lse[static_cast<int64_t>(head) * p.n_req + r] = mh[h] + logf(wh[h]);
+    store(h, c, acc);
   }
 }
 
