@@ -196,6 +196,11 @@ mocap_status mocap_qkv_rope_append(const void *x, const void *w_qkv, void *q_out
  * (0 = no-op); prefix + len < 2^31; 16-byte aligned pointers.
  * Device-side bounded waits that expire are reported by
  * mocap_last_device_status(); the kernel never traps.
+ * With head_dim 128 and a multiple of four query heads per KV head the
+ * kernel runs on pairs of CTAs (thread-block clusters of two, tcgen05
+ * cta_group::2; results equal to the single-CTA kernel up to fp32 rounding
+ * order).  Environment: MOCAP_ATTN_PAIR=0 selects the single-CTA kernel for
+ * every shape; it is read on every call.
  */
 mocap_status mocap_chunk_attn(const void *q, const void *k_cache, const void *v_cache,
                               int64_t prefix, int64_t len,
