@@ -453,6 +453,15 @@ def ours_arm(args, rank, world, local):
         line["last_row"] = measure_last_row(args, m, w, pf, q, dev, stream, hbm)
     if pf.mode == workloads.MODE_LBCP and pf.single and not args.no_uniform:
         line["uniform_boundaries"] = measure_uniform(w, q, k, v, dev, stream)
+        # Algorithm 1 stage 1 (the DP over 128-row units, N = 16 pipeline
+        # stages) with the causal cost c (p + c / 2) and with Eq. 1's c (p + c)
+        s_len, n_chunks = w.seq_lens[0], w.num_chunks[0]
+        for key, model in (("dp_causal_boundaries", m.MOCAP_COST_CAUSAL),
+                           ("dp_eq1_boundaries", m.MOCAP_COST_EQ1)):
+            b = m.mocap_lbcp_partition_dp(s_len, n_chunks, 128, 16, model, 0)
+            line[key] = measure_uniform(w, q, k, v, dev, stream, bounds=[b])
+            line[key]["first_chunk_rows"] = b[1] - b[0]
+            line[key]["last_chunk_rows"] = b[-1] - b[-2]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         times, flops, done, threads = run_oracle_sample(
             q, k, v, pf.bounds[0], w.scale, 1, args.cpu_rows_per_chunk, 20.0)
@@ -578,13 +587,14 @@ def measure_last_row(args, m, w, pf, q, dev, stream, hbm):
             "requests": n, "note": "back-to-back calls; K/V may be partly L2-resident"}
 
 
-def measure_uniform(w, q, k, v, dev, stream, reps=3):
+def measure_uniform(w, q, k, v, dev, stream, reps=3, bounds=None):
     """Per-chunk attention latency with uniform boundaries (outside the timed
-    region): without latency-balanced chunks the late chunks dominate."""
+    region): without latency-balanced chunks the late chunks dominate.  With
+    ``bounds`` the same measurement for that explicit split."""
     import torch
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
     from paper_2606_22968_gb300 import workloads
-    pu = ChunkedPrefill(w, dev, mode=workloads.MODE_UNIFORM)
+    pu = ChunkedPrefill(w, dev, mode=workloads.MODE_UNIFORM, bounds=bounds)
     n = len(pu.steps())
     times = []
     for _ in range(reps):

@@ -28,10 +28,14 @@ class ChunkedPrefill:
     ``[Hq, T]`` array over the packed rows.
     """
 
-    def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True):
+    def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True,
+                 bounds: Optional[List[List[int]]] = None):
+        """``bounds`` (one boundary list per request) replaces the workload's
+        partition rule, e.g. with the Algorithm 1 stage-1 DP's split."""
         self.w = w
         self.device = torch.device(device)
         self.mode = w.mode if mode is None else mode
+        self.fixed_bounds = None if bounds is None else [list(b) for b in bounds]
         self.bounds: List[List[int]] = []
         self.partition()
         self.cu = request_offsets(w)
@@ -54,6 +58,9 @@ class ChunkedPrefill:
 
     def partition(self):
         """Chunk boundaries of every request (host call into the library)."""
+        if self.fixed_bounds is not None:
+            self.bounds = [list(b) for b in self.fixed_bounds]
+            return self.bounds
         part_mode = MOCAP_PART_LBCP if self.mode == 1 else MOCAP_PART_UNIFORM
         self.bounds = [mocap_lbcp_partition(s, m, GRANULARITY, part_mode)
                        for s, m in zip(self.w.seq_lens, self.w.num_chunks)]

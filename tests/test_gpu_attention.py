@@ -428,3 +428,23 @@ def test_varlen_64_items_and_the_limit(m, hq, hkv, d):
                      l_ref, f"item {i}")
     with pytest.raises(m.MocapError):
         m.mocap_chunk_attn_varlen(q, k, v, items + [items[0]], out, lse, scale)
+
+
+def test_dp_boundaries_pipeline_parity(m):
+    """A prompt split by the stage-1 DP of Algorithm 1 (Eq. 1's cost, N = 16)
+    instead of the closed form runs through the same pipeline and matches
+    the oracle on sampled rows of every chunk."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(3)
+    b = m.mocap_lbcp_partition_dp(w.seq_lens[0], w.num_chunks[0], 128, 16, m.MOCAP_COST_EQ1, 0)
+    assert b == P.dp_boundaries(w.seq_lens[0], w.num_chunks[0], 128, 16, P.COST_EQ1, 0)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev, bounds=[b])
+    pf.partition()
+    assert pf.bounds == [b]
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    check_single_request(pf, q, k, v, rows_fn=lambda n, i: sample_rows(n, every=509, edge=2, seed=i))
