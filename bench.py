@@ -544,11 +544,54 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
     if m.mocap_last_device_status() != m.MOCAP_OK:
         raise RuntimeError("device wait expired in the projection measurement")
     gemm_tf = gemm_flops / (ms_gemm * 1e-3) / 1e12
-    return {"hidden": hidden, "n_out": n_out, "flop_per_step": gemm_flops,
+    line = {"hidden": hidden, "n_out": n_out, "flop_per_step": gemm_flops,
             "ms_per_step": ms_gemm, "tflops": gemm_tf, "frac_of_peak": gemm_tf / peak,
             "stage_ms_per_step": ms_stage,
             "stage_tflops": (gemm_flops + attn_flops) / (ms_stage * 1e-3) / 1e12,
             "stage_tokens_per_s": w.total_tokens / (ms_stage * 1e-3)}
+
+    # Per-chunk stage latency (projection + attention of one chunk), for the
+    # workload's split and for the stage-1 DP of Algorithm 1 fed with this
+    # run's measured rates: per chunk a * pairs + b * rows, i.e. in the DP's
+    # doubled 128-row units k (2 s + k) + gemm_weight * k with
+    # gemm_weight = 2 b / (128 a).
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    s_len, n_chunks = w.seq_lens[0], w.num_chunks[0]
+    a_pair = (ms_stage - ms_gemm) * 1e-3 / (s_len * (s_len + 1) / 2)
+    b_row = ms_gemm * 1e-3 / s_len
+    gemm_weight = max(0, int(round(2.0 * b_row / (128.0 * a_pair))))
+
+    def per_chunk_stage(pfx, reps=3):
+        bx = pfx.bounds[0]
+        nx = len(bx) - 1
+        times = []
+        for _ in range(reps):
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                  for _ in range(nx)]
+            for c in range(nx):
+                ev[c][0].record(stream)
+                m.mocap_qkv_rope_append(x[bx[c]:bx[c + 1]], wq, qbuf[bx[c]:bx[c + 1]],
+                                        pfx.k_cache, pfx.v_cache, bx[c], stream=stream)
+                m.mocap_chunk_attn(qbuf[bx[c]:bx[c + 1]], pfx.k_cache, pfx.v_cache, bx[c],
+                                   pfx.out[bx[c]:bx[c + 1]], pfx.chunk_lse(c), w.scale,
+                                   workspace=pfx.workspace, stream=stream)
+                ev[c][1].record(stream)
+            torch.cuda.synchronize(dev)
+            times.append([e0.elapsed_time(e1) for e0, e1 in ev])
+        pc = [statistics.median(t[c] for t in times) for c in range(nx)]
+        return {"min": min(pc), "max": max(pc), "max_over_min": max(pc) / min(pc),
+                "cv": statistics.pstdev(pc) / statistics.mean(pc), "ms_per_step": sum(pc)}
+
+    line["stage_per_chunk_ms"] = {"workload_split": per_chunk_stage(pf)}
+    b_dp = m.mocap_lbcp_partition_dp(s_len, n_chunks, 128, 16, m.MOCAP_COST_CAUSAL, gemm_weight)
+    pf_dp = ChunkedPrefill(w, dev, bounds=[b_dp])
+    line["stage_per_chunk_ms"]["dp_with_gemm_term"] = {
+        **per_chunk_stage(pf_dp), "gemm_weight": gemm_weight,
+        "first_chunk_rows": b_dp[1] - b_dp[0], "last_chunk_rows": b_dp[-1] - b_dp[-2]}
+    del pf_dp
+    if m.mocap_last_device_status() != m.MOCAP_OK:
+        raise RuntimeError("device wait expired in the per-chunk stage measurement")
+    return line
 
 
 def measure_last_row(args, m, w, pf, q, dev, stream, hbm):
