@@ -555,11 +555,10 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
     # run's measured rates: per chunk a * pairs + b * rows, i.e. in the DP's
     # doubled 128-row units k (2 s + k) + gemm_weight * k with
     # gemm_weight = 2 b / (128 a).
-    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill, gemm_weight, stage_balanced_bounds
     s_len, n_chunks = w.seq_lens[0], w.num_chunks[0]
     a_pair = (ms_stage - ms_gemm) * 1e-3 / (s_len * (s_len + 1) / 2)
     b_row = ms_gemm * 1e-3 / s_len
-    gemm_weight = max(0, int(round(2.0 * b_row / (128.0 * a_pair))))
 
     def per_chunk_stage(pfx, reps=3):
         bx = pfx.bounds[0]
@@ -583,10 +582,10 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
                 "cv": statistics.pstdev(pc) / statistics.mean(pc), "ms_per_step": sum(pc)}
 
     line["stage_per_chunk_ms"] = {"workload_split": per_chunk_stage(pf)}
-    b_dp = m.mocap_lbcp_partition_dp(s_len, n_chunks, 128, 16, m.MOCAP_COST_CAUSAL, gemm_weight)
+    b_dp = stage_balanced_bounds(s_len, n_chunks, a_pair, b_row)
     pf_dp = ChunkedPrefill(w, dev, bounds=[b_dp])
     line["stage_per_chunk_ms"]["dp_with_gemm_term"] = {
-        **per_chunk_stage(pf_dp), "gemm_weight": gemm_weight,
+        **per_chunk_stage(pf_dp), "gemm_weight": gemm_weight(a_pair, b_row),
         "first_chunk_rows": b_dp[1] - b_dp[0], "last_chunk_rows": b_dp[-1] - b_dp[-2]}
     del pf_dp
     if m.mocap_last_device_status() != m.MOCAP_OK:

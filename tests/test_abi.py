@@ -207,3 +207,22 @@ def test_bench_entry_points_exist():
                  "reference_arm", "measure_e2e", "measure_graph", "measure_projection",
                  "measure_last_row", "measure_uniform"]:
         assert callable(getattr(bench, name)), name
+
+
+def test_stage_balanced_bounds_weight_and_dp():
+    """The GEMM weight follows from the per-chunk stage cost a * pairs + b * rows
+    in the DP's doubled 128-row units, and the split is the DP's (bit-exact
+    against the oracle's DP with that weight)."""
+    from paper_2606_22968_gb300.pipeline import gemm_weight, stage_balanced_bounds
+    from oracle import partition as P
+    # a chunk of k units at s: pairs ~ 128^2 k (s + k/2), rows 128 k
+    # a * 128^2 / 2 * [k (2s + k) + w k] = a * 128^2 k (s + k/2) + b * 128 k  =>  w = 2 b / (128 a)
+    assert gemm_weight(1.0, 64.0) == 1
+    assert gemm_weight(1.84e-11, 1.06e-7) == 90
+    assert gemm_weight(1.0, 0.0) == 0
+    for bad in ((0.0, 1.0), (1.0, -1.0)):
+        with pytest.raises(ValueError):
+            gemm_weight(*bad)
+    for a, b in ((1.84e-11, 1.06e-7), (1e-11, 0.0)):
+        got = stage_balanced_bounds(32768, 16, a, b)
+        assert got == P.dp_boundaries(32768, 16, 128, 16, P.COST_CAUSAL, gemm_weight(a, b))
