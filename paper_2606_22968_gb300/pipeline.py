@@ -9,6 +9,7 @@ into libmocap.so; torch only allocates memory and provides the stream.
 
 from __future__ import annotations
 
+import os
 from typing import List, Optional
 
 import torch
@@ -109,7 +110,15 @@ class ChunkedPrefill:
     def run_step(self, q, k, v, step, stream=None, events=None):
         """Append + attention for one step (one chunk index).  ``events`` is
         an optional triple of CUDA events recorded before the appends, between
-        appends and attention, and after the attention."""
+        appends and attention, and after the attention.  With MOCAP_NVTX=1 in
+        the environment each step is an NVTX range ("mocap chunk <index>")
+        for timeline profilers."""
+        if os.environ.get("MOCAP_NVTX", "0") != "0":
+            with torch.cuda.nvtx.range(f"mocap chunk {step[0][1]}"):
+                return self._run_step(q, k, v, step, stream, events)
+        return self._run_step(q, k, v, step, stream, events)
+
+    def _run_step(self, q, k, v, step, stream=None, events=None):
         w = self.w
         if events is not None:
             events[0].record(stream)
