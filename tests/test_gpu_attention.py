@@ -448,3 +448,22 @@ def test_dp_boundaries_pipeline_parity(m):
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == 0
     check_single_request(pf, q, k, v, rows_fn=lambda n, i: sample_rows(n, every=509, edge=2, seed=i))
+
+
+def test_nvtx_ranges_leave_results_unchanged(m, monkeypatch):
+    """MOCAP_NVTX=1 wraps each chunk step in an NVTX range; the launches and
+    results are the same."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(2)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev)
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    out, lse = pf.out.clone(), pf.lse.clone()
+    monkeypatch.setenv("MOCAP_NVTX", "1")
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    assert torch.equal(pf.out, out) and torch.equal(pf.lse, lse)
