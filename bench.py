@@ -443,6 +443,7 @@ def ours_arm(args, rank, world, local):
         # thermal state of the GPU (the auxiliary measurements below add
         # about a minute of load first)
         line["e2e"] = measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world)
+    line["append"].update(measure_append_graph(m, w, pf, k, v, dev, append_bytes, hbm))
     if not args.no_graph:
         line["graph_replay"] = measure_graph(args, pf, q, k, v, dev, stream, total_flops,
                                              w.total_tokens, world)
@@ -474,6 +475,43 @@ def ours_arm(args, rank, world, local):
     if rank == 0:
         print(json.dumps(line), flush=True)
     return 0
+
+
+def measure_append_graph(m, w, pf, k, v, dev, append_bytes, hbm, reps=5):
+    """Device time of the step's appends alone: all of them captured in one
+    CUDA graph and replayed back to back (no launch gaps, no attention in
+    between), so the figure is the append kernel's own bandwidth."""
+    import torch
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(torch.cuda.current_stream(dev))
+    graph = torch.cuda.CUDAGraph()
+
+    def appends(stream):
+        for step in pf.steps():
+            for r, c in step:
+                b0, b1 = pf.bounds[r][c], pf.bounds[r][c + 1]
+                base = pf.cu[r]
+                m.mocap_kv_append(k[base + b0:base + b1], v[base + b0:base + b1],
+                                  pf.k_cache[base:base + w.seq_lens[r]],
+                                  pf.v_cache[base:base + w.seq_lens[r]], b0, stream=stream)
+
+    with torch.cuda.stream(side):
+        appends(side)  # outside the capture: one-time set-up
+        with torch.cuda.graph(graph, stream=side):
+            appends(side)
+    torch.cuda.current_stream(dev).wait_stream(side)
+    graph.replay()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        graph.replay()
+    e1.record()
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1) / reps
+    gbs = append_bytes / (ms * 1e-3) / 1e9
+    return {"kernel_ms_per_step": ms, "kernel_gb_per_s": gbs, "kernel_frac_of_hbm": gbs / hbm,
+            "kernel_note": "the step's appends replayed as one CUDA graph"}
 
 
 def measure_graph(args, pf, q, k, v, dev, stream, total_flops, tokens, world):
