@@ -6,11 +6,12 @@
 // balances.  The kernel computes, for query head h (KV head h / group) and
 // global row t, O_t = softmax_{j<=t}(scale q_t.k_j) V and LSE_t = ln sum exp.
 //
-// Two forms.  CTA pairs (single-item launches, d = 128, a multiple of four
-// query heads per KV group; see control_roles_pair): two CTAs on two SMs
-// share the KV group, row block and keys, each holds two heads, and
+// Two forms.  CTA pairs (d = 128 with a multiple of four query heads per KV
+// group, single and varlen launches; see control_roles_pair): two CTAs on
+// two SMs share the KV group, row block and keys, each holds two heads, and
 // tcgen05 cta_group::2 MMAs (M = 256) read K and V halves from both CTAs, so
 // each SM stages and each SM's L2 traffic carries half of every K/V tile.
+// The softmax warps and the layout of TMEM are the same in both forms.
 // Single CTAs (every other shape) as follows.
 //
 // Design (one CTA = 128 query rows x up to two query heads of one KV group;
