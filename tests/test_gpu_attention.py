@@ -360,6 +360,8 @@ PAIR_CASES = [
     (61440 + 77, 700, 64, 8, 128, None),   # Llama-3-70B heads, unaligned prefix
     (100000, 256, 8, 2, 128, None),        # the library splits the key range
     (200, 2000, 8, 2, 128, 3),             # three forced splits
+    (500, 700, 96, 8, 128, None),          # 12:1, six head pairs per KV group
+    (0, 257, 16, 1, 128, 2),               # 16:1 over one KV head, two splits
 ]
 
 
