@@ -559,11 +559,6 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
         m.mocap_qkv_rope_append(x[b[c]:b[c + 1]], wq, qbuf[b[c]:b[c + 1]], pf.k_cache,
                                 pf.v_cache, b[c], stream=stream)
 
-    def attend(c):
-        m.mocap_chunk_attn(qbuf[b[c]:b[c + 1]], pf.k_cache, pf.v_cache, b[c],
-                           pf.out[b[c]:b[c + 1]], pf.chunk_lse(c), w.scale,
-                           workspace=pf.workspace, stream=stream)
-
     def timed(fn):
         for _ in range(args.warmup):
             fn()
@@ -578,7 +573,7 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
 
     n = len(b) - 1
     ms_gemm = timed(lambda: [project(c) for c in range(n)])
-    ms_stage = timed(lambda: [(project(c), attend(c)) for c in range(n)])
+    ms_stage = timed(lambda: pf.run_stage(x, wq, qbuf, stream))
     if m.mocap_last_device_status() != m.MOCAP_OK:
         raise RuntimeError("device wait expired in the projection measurement")
     gemm_tf = gemm_flops / (ms_gemm * 1e-3) / 1e12
@@ -599,20 +594,12 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
     b_row = ms_gemm * 1e-3 / s_len
 
     def per_chunk_stage(pfx, reps=3):
-        bx = pfx.bounds[0]
-        nx = len(bx) - 1
+        nx = len(pfx.bounds[0]) - 1
         times = []
         for _ in range(reps):
             ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                   for _ in range(nx)]
-            for c in range(nx):
-                ev[c][0].record(stream)
-                m.mocap_qkv_rope_append(x[bx[c]:bx[c + 1]], wq, qbuf[bx[c]:bx[c + 1]],
-                                        pfx.k_cache, pfx.v_cache, bx[c], stream=stream)
-                m.mocap_chunk_attn(qbuf[bx[c]:bx[c + 1]], pfx.k_cache, pfx.v_cache, bx[c],
-                                   pfx.out[bx[c]:bx[c + 1]], pfx.chunk_lse(c), w.scale,
-                                   workspace=pfx.workspace, stream=stream)
-                ev[c][1].record(stream)
+            pfx.run_stage(x, wq, qbuf, stream, chunk_events=ev)
             torch.cuda.synchronize(dev)
             times.append([e0.elapsed_time(e1) for e0, e1 in ev])
         pc = [statistics.median(t[c] for t in times) for c in range(nx)]

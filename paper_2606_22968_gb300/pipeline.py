@@ -16,7 +16,7 @@ import torch
 
 from . import (MOCAP_COST_CAUSAL, MOCAP_PART_LBCP, MOCAP_PART_UNIFORM, mocap_chunk_attn,
                mocap_chunk_attn_varlen, mocap_chunk_attn_workspace_size, mocap_kv_append,
-               mocap_lbcp_partition, mocap_lbcp_partition_dp)
+               mocap_lbcp_partition, mocap_lbcp_partition_dp, mocap_qkv_rope_append)
 from .workloads import GRANULARITY, Workload, request_offsets
 
 
@@ -152,6 +152,29 @@ class ChunkedPrefill:
         for i, step in enumerate(self.steps()):
             self.run_step(q, k, v, step, stream,
                           None if chunk_events is None else chunk_events[i])
+
+    def run_stage(self, x, w_qkv, q_buf, stream=None, rope_theta: float = 500000.0,
+                  chunk_events=None):
+        """One attention layer's chunk stage for a single request (Eq. 1 with
+        its GEMM term): per chunk, in order, the fused QKV projection of the
+        chunk's hidden states ``x`` [S, hidden] with ``w_qkv`` [(Hq + 2 Hkv) d,
+        hidden] (RoPE at the chunk's global positions; Q to ``q_buf`` [S, Hq,
+        d], K and V straight into the caches), then the chunk's attention over
+        the cache.  ``chunk_events`` optionally holds one (start, end) event
+        pair per chunk."""
+        if not self.single:
+            raise ValueError("run_stage takes a single-request workload")
+        w, b = self.w, self.bounds[0]
+        for c in range(len(b) - 1):
+            if chunk_events is not None:
+                chunk_events[c][0].record(stream)
+            mocap_qkv_rope_append(x[b[c]:b[c + 1]], w_qkv, q_buf[b[c]:b[c + 1]], self.k_cache,
+                                  self.v_cache, b[c], rope_theta=rope_theta, stream=stream)
+            mocap_chunk_attn(q_buf[b[c]:b[c + 1]], self.k_cache, self.v_cache, b[c],
+                             self.out[b[c]:b[c + 1]], self.chunk_lse(c), w.scale,
+                             workspace=self.workspace, stream=stream)
+            if chunk_events is not None:
+                chunk_events[c][1].record(stream)
 
     # -- from host memory ------------------------------------------------------------
     def _rows(self, r, c):

@@ -109,3 +109,44 @@ def test_qkv_rope_full_size_sampled_rows(m, length, offset):
             err = np.abs(got.float().cpu().numpy() - ref)
             assert err.max() <= TOL_MAX and err.mean() <= TOL_MEAN, (name, int(r), err.max(),
                                                                    err.mean())
+
+
+def test_run_stage_projection_then_attention(m):
+    """ChunkedPrefill.run_stage: per chunk the fused projection writes Q and
+    the chunk's K/V rows, then attention reads the cache.  The projection
+    outputs match the projection oracle, and the attention matches the
+    attention oracle on the exact Q/K/V bits the projection produced (every
+    chunk, sampled rows), so positions and cache rows line up across the
+    two kernels."""
+    from oracle import attention as A
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    from tests.parity_utils import assert_close, chunk_rows_oracle, sample_rows
+    w = workloads.custom("stage-8k-lbcp8-h16-g4-d128", (8192,), (8,), workloads.MODE_LBCP, 16, 4,
+                         128)
+    hidden, theta = 256, 500000.0
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(8192)
+    x = torch.randn((8192, hidden), generator=gen, device=dev).bfloat16()
+    n_out = (w.n_q_heads + 2 * w.n_kv_heads) * w.head_dim
+    wq = (torch.randn((n_out, hidden), generator=gen, device=dev) / math.sqrt(hidden)).bfloat16()
+    pf = ChunkedPrefill(w, dev)
+    qbuf = torch.full((8192, w.n_q_heads, w.head_dim), float("nan"), device=dev,
+                      dtype=torch.bfloat16)
+    pf.run_stage(x, wq, qbuf, rope_theta=theta)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    q_ref, k_ref, v_ref = R.qkv_rope(f64(x), f64(wq), w.n_q_heads, w.n_kv_heads, w.head_dim, 0,
+                                     theta)
+    for got, ref, name in [(qbuf, q_ref, "Q"), (pf.k_cache, k_ref, "K"), (pf.v_cache, v_ref, "V")]:
+        err = np.abs(got.float().cpu().numpy() - ref)
+        assert err.max() <= TOL_MAX and err.mean() <= TOL_MEAN, (name, err.max(), err.mean())
+    b = pf.bounds[0]
+    kf, vf = f64(pf.k_cache), f64(pf.v_cache)
+    for i in range(len(b) - 1):
+        rows = sample_rows(b[i + 1] - b[i], every=211, edge=2, seed=i)
+        idx = torch.as_tensor(rows, device=dev)
+        o_ref, l_ref = chunk_rows_oracle(f64(qbuf[b[i]:b[i + 1]][idx]), kf[:b[i + 1]],
+                                         vf[:b[i + 1]], b[i], rows, w.scale)
+        assert_close(pf.out[b[i]:b[i + 1]][idx].float().cpu().numpy(),
+                     pf.chunk_lse(i)[:, idx].cpu().numpy(), o_ref, l_ref, f"chunk {i}")
