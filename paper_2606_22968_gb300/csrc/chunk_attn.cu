@@ -48,9 +48,12 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <functional>
 #include <cstdlib>
 #include <cstring>
+#include <map>
 #include <mutex>
+#include <tuple>
 #include <vector>
 
 #include "internal.h"
@@ -947,8 +950,8 @@ int sm_count_cached() {
 // Cost units: one 128-key tile of a head pair ~ 1.4 us; a CTA's fixed cost
 // ~ 4 us; the combine reads splits x (4D + 4) and writes 2D + 4 bytes per
 // (row, head) at ~5 TB/s, plus ~3 us for its launch.
-int choose_splits(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads, int head_dim,
-                  int sms) {
+int choose_splits_uncached(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads,
+                           int head_dim, int sms) {
   const int group = n_q_heads / n_kv_heads;
   const int64_t pairs = (group + 1) / 2;
   const int64_t q_blocks = (len + kBlockM - 1) / kBlockM;
@@ -958,17 +961,19 @@ int choose_splits(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads, in
   const double tile_us = 1.4 * (head_dim / 128.0), cta_us = 4.0;
   double best_t = 0.0;
   int best = 1;
-  std::vector<double> sm(static_cast<size_t>(sms));
   for (int sp = 1; sp <= kMaxSplits && sp <= min_tiles; ++sp) {
-    std::fill(sm.begin(), sm.end(), 0.0);
+    // SM loads as a min-heap: each CTA goes to a least-loaded SM (which of
+    // several equally loaded SMs does not change the multiset of loads)
+    std::vector<double> sm(static_cast<size_t>(sms), 0.0);
     for (int64_t qb = q_blocks - 1; qb >= 0; --qb) {
       const int64_t kv_end = std::min<int64_t>(prefix + qb * kBlockM + kBlockM, prefix + len);
       const int64_t tiles = (kv_end + kBlockN - 1) / kBlockN;
       for (int64_t u = 0; u < n_kv_heads * pairs; ++u)
         for (int k = 0; k < sp; ++k) {
           const int64_t nk = (k + 1) * tiles / sp - k * tiles / sp;
-          auto it = std::min_element(sm.begin(), sm.end());
-          *it += cta_us + tile_us * static_cast<double>(nk);
+          std::pop_heap(sm.begin(), sm.end(), std::greater<double>());
+          sm.back() += cta_us + tile_us * static_cast<double>(nk);
+          std::push_heap(sm.begin(), sm.end(), std::greater<double>());
         }
     }
     double t = *std::max_element(sm.begin(), sm.end());
@@ -981,6 +986,27 @@ int choose_splits(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads, in
     }
   }
   return best;
+}
+
+// The plan depends only on the shape and the SM count, and a prompt repeats
+// its chunk shapes step after step, so plans are kept (up to 4096 shapes;
+// the table is cleared when full).
+int choose_splits(int64_t prefix, int64_t len, int n_q_heads, int n_kv_heads, int head_dim,
+                  int sms) {
+  using Key = std::tuple<int64_t, int64_t, int, int, int, int>;
+  static std::map<Key, int> cache;
+  static std::mutex mu;
+  const Key key{prefix, len, n_q_heads, n_kv_heads, head_dim, sms};
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    const auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+  }
+  const int splits = choose_splits_uncached(prefix, len, n_q_heads, n_kv_heads, head_dim, sms);
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache.size() >= 4096) cache.clear();
+  cache.emplace(key, splits);
+  return splits;
 }
 
 // CTA pairs (cta_group::2) serve d = 128 with a multiple of four query heads
