@@ -232,6 +232,86 @@ class ChunkedPrefill:
         compute.wait_stream(d2h)
         compute.wait_stream(h2d)
 
+    def run_prompts_from_host(self, prompts, buffers):
+        """Several prompts of this workload's shape in a row, each from (pinned)
+        host memory, with the next prompt's inputs going up while the current
+        one computes.
+
+        ``prompts``: a sequence of (host_q, host_k, host_v, host_out,
+        host_lse), shaped like ``run_from_host``'s arguments.  ``buffers``: two
+        (q, k, v) device buffer sets used alternately; prompt p's inputs go
+        into set p % 2 once prompt p - 2 has finished computing from it.
+        Within a prompt, chunk i starts as soon as its rows have landed and
+        its O and LSE go back as soon as its attention is done, as in
+        ``run_from_host``; prompt p + 1's chunks start after prompt p's
+        results have left the shared output buffers.  The caller's current
+        stream waits for everything before this returns."""
+        if len(buffers) != 2:
+            raise ValueError("two device buffer sets expected")
+        compute = torch.cuda.current_stream(self.device)
+        h2d = torch.cuda.Stream(self.device)
+        d2h = torch.cuda.Stream(self.device)
+        steps = self.steps()
+        hq = self.w.n_q_heads
+        h2d.wait_stream(compute)
+        d2h.wait_stream(compute)
+        computed = [None, None]   # per buffer set: the end of the last prompt computed from it
+        outputs_gone = None       # the end of the last prompt's D2H copies
+        landed = []               # per prompt: per step, the event its inputs landed on
+
+        def upload(p):
+            q, k, v = buffers[p % 2]
+            host_q, host_k, host_v = prompts[p][:3]
+            evs = []
+            with torch.cuda.stream(h2d):
+                if computed[p % 2] is not None:
+                    h2d.wait_event(computed[p % 2])
+                for step in steps:
+                    for r, c in step:
+                        rows, _, _ = self._rows(r, c)
+                        q[rows].copy_(host_q[rows], non_blocking=True)
+                        k[rows].copy_(host_k[rows], non_blocking=True)
+                        v[rows].copy_(host_v[rows], non_blocking=True)
+                    ev = torch.cuda.Event()
+                    ev.record(h2d)
+                    evs.append(ev)
+            landed.append(evs)
+
+        if prompts:
+            upload(0)
+        for p in range(len(prompts)):
+            if p + 1 < len(prompts):
+                upload(p + 1)  # overlaps this prompt's compute (other buffer set)
+            q, k, v = buffers[p % 2]
+            host_out, host_lse = prompts[p][3], prompts[p][4]
+            if outputs_gone is not None:
+                compute.wait_event(outputs_gone)
+            for i, step in enumerate(steps):
+                compute.wait_event(landed[p][i])
+                self.run_step(q, k, v, step, compute)
+                done = torch.cuda.Event()
+                done.record(compute)
+                d2h.wait_event(done)
+                with torch.cuda.stream(d2h):
+                    for r, c in step:
+                        rows, b0, b1 = self._rows(r, c)
+                        host_out[rows].copy_(self.out[rows], non_blocking=True)
+                        if self.single:
+                            host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
+                                                            non_blocking=True)
+            end = torch.cuda.Event()
+            end.record(compute)
+            computed[p % 2] = end
+            if not self.single:
+                d2h.wait_event(end)
+                with torch.cuda.stream(d2h):
+                    host_lse.copy_(self.lse, non_blocking=True)
+            gone = torch.cuda.Event()
+            gone.record(d2h)
+            outputs_gone = gone
+        compute.wait_stream(d2h)
+        compute.wait_stream(h2d)
+
     # -- CUDA graph ------------------------------------------------------------------
     def capture(self, q, k, v, stream=None):
         """Record the whole prompt's launch sequence (every append, attention

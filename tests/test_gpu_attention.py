@@ -469,3 +469,35 @@ def test_nvtx_ranges_leave_results_unchanged(m, monkeypatch):
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == 0
     assert torch.equal(pf.out, out) and torch.equal(pf.lse, lse)
+
+
+@pytest.mark.parametrize("index", [3, 5])
+def test_run_prompts_from_host_matches_device_runs(m, index):
+    """Three different prompts streamed from pinned host memory, each
+    prompt's inputs going up during the previous prompt's compute: every
+    prompt's O and LSE equal a device-resident run of that prompt, bitwise."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(index)
+    dev = torch.device("cuda")
+    pf = ChunkedPrefill(w, dev)
+    prompts, refs = [], []
+    for p in range(3):
+        gen = torch.Generator(device=dev).manual_seed(100 + p)
+        t = w.total_tokens
+        q = torch.randn((t, w.n_q_heads, w.head_dim), generator=gen, device=dev).bfloat16()
+        k = torch.randn((t, w.n_kv_heads, w.head_dim), generator=gen, device=dev).bfloat16()
+        v = torch.randn((t, w.n_kv_heads, w.head_dim), generator=gen, device=dev).bfloat16()
+        pf.run(q, k, v)
+        torch.cuda.synchronize()
+        refs.append((pf.out.cpu().clone(), pf.lse.cpu().clone()))
+        ho = torch.full(pf.out.shape, float("nan"), dtype=pf.out.dtype).pin_memory()
+        hl = torch.full(pf.lse.shape, float("nan"), dtype=pf.lse.dtype).pin_memory()
+        prompts.append((q.cpu().pin_memory(), k.cpu().pin_memory(), v.cpu().pin_memory(), ho, hl))
+    bufs = [tuple(torch.full_like(x, float("nan"), device=dev) for x in prompts[0][:3])
+            for _ in range(2)]
+    pf.run_prompts_from_host(prompts, bufs)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    for (ho, hl), (ro, rl) in zip([pr[3:] for pr in prompts], refs):
+        assert torch.equal(ho, ro) and torch.equal(hl, rl)
