@@ -817,13 +817,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // Split-KV combine: the softmax over the union of disjoint key ranges weighs
 // each range's normalised output by exp(LSE_k - LSE), LSE = ln sum_k exp(LSE_k).
-// One warp per (row, head); each lane owns D/32 consecutive columns.
+// One warp per (row, head); each lane owns D/32 consecutive columns.  Like
+// the attention launch before it, it does nothing once a bounded wait has
+// expired (the status word is set), so the outputs keep their contents.
 template <int D>
 __global__ void __launch_bounds__(256) attn_combine_kernel(
     const float *__restrict__ o_part, const float *__restrict__ lse_part, int splits,
     int64_t len, int n_q_heads, __nv_bfloat16 *__restrict__ out, float *__restrict__ lse,
-    int64_t lse_stride) {
+    int64_t lse_stride, const uint32_t *status) {
   constexpr int kPer = D / 32;
+  if (*reinterpret_cast<const volatile uint32_t *>(status) != 0u) return;
   const int64_t idx = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
   if (idx >= len * n_q_heads) return;
   const int lane = threadIdx.x & 31;
@@ -1125,7 +1128,7 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     const int64_t len = items[0].len;
     const int64_t warps = len * sh.n_q_heads;
     attn_combine_kernel<D><<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
-        prm.o_part, prm.lse_part, sp.splits, len, sh.n_q_heads, prm.out, lse, lse_stride);
+        prm.o_part, prm.lse_part, sp.splits, len, sh.n_q_heads, prm.out, lse, lse_stride, status);
     if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
   }
   return MOCAP_OK;

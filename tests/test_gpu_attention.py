@@ -501,3 +501,59 @@ def test_run_prompts_from_host_matches_device_runs(m, index):
     assert m.mocap_last_device_status() == 0
     for (ho, hl), (ro, rl) in zip([pr[3:] for pr in prompts], refs):
         assert torch.equal(ho, ro) and torch.equal(hl, rl)
+
+
+@pytest.mark.parametrize("prefix,length,hq,hkv,d,forced,pair", [
+    (200, 2000, 8, 2, 128, 3, "0"),
+    (400, 2000, 8, 2, 128, 4, "0"),
+    (1000, 130, 4, 4, 64, 2, "0"),
+    (129024 - 2 * 128 + 77, 2048, 64, 8, 128, 2, "1"),
+    (300, 257, 16, 1, 128, 2, "1"),
+])
+def test_split_combine_formula_and_determinism(m, monkeypatch, prefix, length, hq, hkv, d,
+                                               forced, pair):
+    """The split-KV combine checked three ways: the output is the formula
+    O = sum_k exp(LSE_k - LSE) O_k, LSE = ln sum_k exp(LSE_k) applied in
+    PyTorch fp32 to the partials the call left in the workspace; repeated
+    calls on freshly garbaged workspaces give bitwise equal results; and it
+    stays within the parity tolerances of the oracle."""
+    monkeypatch.setenv("MOCAP_SPLIT_KV", str(forced))
+    monkeypatch.setenv("MOCAP_ATTN_PAIR", pair)
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(prefix + 3 * length + hq)
+    s = prefix + length
+    q = _randn((length, hq, d), gen, dev)
+    k, v = _randn((s, hkv, d), gen, dev), _randn((s, hkv, d), gen, dev)
+    scale = 1.0 / math.sqrt(d)
+    ws_bytes = m.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d)
+    o_bytes = forced * length * hq * d * 4
+    lse_off = (o_bytes + 255) // 256 * 256
+    assert ws_bytes >= lse_off + forced * hq * length * 4
+    results = []
+    for fill in (0xFF, 0x00, 0x7F):
+        ws = torch.full((ws_bytes,), fill, device=dev, dtype=torch.uint8)
+        out = torch.full((length, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+        lse = torch.full((hq, length), float("nan"), device=dev, dtype=torch.float32)
+        m.mocap_chunk_attn(q, k, v, prefix, out, lse, scale, workspace=ws)
+        torch.cuda.synchronize()
+        assert m.mocap_last_device_status() == 0
+        results.append((out.clone(), lse.clone(), ws.clone()))
+    for out, lse, _ in results[1:]:
+        assert torch.equal(out, results[0][0]) and torch.equal(lse, results[0][1])
+    out, lse, ws = results[0]
+    o_part = ws[:o_bytes].view(torch.float32).view(forced, length, hq, d)
+    l_part = ws[lse_off:lse_off + forced * hq * length * 4].view(torch.float32).view(
+        forced, hq, length)
+    assert torch.isfinite(o_part).all()
+    mx = l_part.max(dim=0).values                               # [hq, len]
+    w = torch.where(l_part > -math.inf, torch.exp(l_part - mx), torch.zeros_like(l_part))
+    wsum = w.sum(dim=0)
+    o_ref = (w / wsum).permute(0, 2, 1).unsqueeze(-1).mul(o_part).sum(dim=0)  # [len, hq, d]
+    torch.testing.assert_close(lse, mx + torch.log(wsum), rtol=0, atol=2e-6)
+    # bf16 output of an fp32 sum: within one bf16 rounding of the formula
+    err = (out.float() - o_ref).abs()
+    assert (err <= o_ref.abs() * 2.0 ** -8 + 4e-6).all(), err.max().item()
+    rows = np.arange(length) if length <= 512 else sample_rows(length, every=37)
+    idx = torch.as_tensor(rows, device=dev)
+    o_or, l_or = chunk_rows_oracle(f64(q[idx]), f64(k), f64(v), prefix, rows, scale)
+    assert_close(out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_or, l_or, "merged")

@@ -41,26 +41,37 @@ def test_expired_wait_is_reported_and_cleared(m):
     assert m.mocap_last_device_status() == m.MOCAP_OK  # read clears it
 
 
-@pytest.mark.parametrize("pair", ["1", "0"])
-def test_launch_after_expired_wait_does_nothing_then_recovers(m, monkeypatch, pair):
+@pytest.mark.parametrize("pair,split", [("1", None), ("0", None), ("1", 2), ("0", 2)])
+def test_launch_after_expired_wait_does_nothing_then_recovers(m, monkeypatch, pair, split):
     # both attention forms: CTA pairs (both CTAs act on the first CTA's
-    # reading of the status word) and single CTAs
+    # reading of the status word) and single CTAs.  With split-KV (rows
+    # 128..299 over two key tiles) no split arrives, so nothing is merged,
+    # and the next call's counters start at 0 again.
     monkeypatch.setenv("MOCAP_ATTN_PAIR", pair)
     dev = torch.device("cuda")
-    q, k, v = _small(dev)
+    q_all, k, v = _small(dev)
+    prefix = 0 if split is None else 128
+    q = q_all[prefix:].contiguous()
+    rows = q.shape[0]
+    ws = None
+    if split is not None:
+        monkeypatch.setenv("MOCAP_SPLIT_KV", str(split))
+        need = m.mocap_chunk_attn_workspace_size(prefix, rows, 8, 2, 128)
+        assert need > 0
+        ws = torch.empty((need,), device=dev, dtype=torch.uint8)
     out = torch.full_like(q, float("nan"))
-    lse = torch.full((8, 300), float("nan"), device=dev, dtype=torch.float32)
+    lse = torch.full((8, rows), float("nan"), device=dev, dtype=torch.float32)
     m.mocap_selftest_bounded_wait(20000)
-    m.mocap_chunk_attn(q, k, v, 0, out, lse, 0.088)   # queued behind the expired wait
+    m.mocap_chunk_attn(q, k, v, prefix, out, lse, 0.088, workspace=ws)  # behind the expired wait
     torch.cuda.synchronize()
     assert torch.isnan(out.float()).all() and torch.isnan(lse).all()
     assert m.mocap_last_device_status() == m.MOCAP_ETIMEOUT
     # the context is usable: the same launch now computes the right answer
-    m.mocap_chunk_attn(q, k, v, 0, out, lse, 0.088)
+    m.mocap_chunk_attn(q, k, v, prefix, out, lse, 0.088, workspace=ws)
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == m.MOCAP_OK
-    o_ref, l_ref = A.causal_attention(f64(q), f64(k), f64(v), 0.088)
-    assert_close(out.float().cpu().numpy(), lse.cpu().numpy(), o_ref, l_ref)
+    o_ref, l_ref = A.causal_attention(f64(q_all), f64(k), f64(v), 0.088)
+    assert_close(out.float().cpu().numpy(), lse.cpu().numpy(), o_ref[prefix:], l_ref[:, prefix:])
 
 
 def test_selftest_rejects_bad_limits(m):
