@@ -357,7 +357,8 @@ mocap_status mocap_last_device_status(mocap_stream_t stream);
  * the same bounded wait, on a barrier nothing ever completes, for limit_us
  * microseconds (1 .. 1000000, else MOCAP_EINVAL).  Afterwards
  * mocap_last_device_status() reports MOCAP_ETIMEOUT, and until it is read
- * every attention launch returns without doing work.  No counterpart in the
+ * every attention launch (split-KV combine included) returns without doing
+ * work, leaving its outputs as they were.  No counterpart in the
  * paper: failure detection for shared GPUs.
  */
 mocap_status mocap_selftest_bounded_wait(uint32_t limit_us, mocap_stream_t stream);
