@@ -121,6 +121,19 @@ def mocap_chunk_attn(q, k_cache, v_cache, prefix: int, out, lse, scale: float,
            "mocap_chunk_attn")
 
 
+def mocap_chunk_attn_noalloc(q, k_cache, v_cache, prefix: int, out, lse, scale: float,
+                             stream=None):
+    """mocap_chunk_attn without a caller workspace: split-KV partials go to
+    the library's fixed device scratch (MOCAP_NOALLOC_SCRATCH_BYTES); calls
+    whose work overlaps on the GPU must not share it."""
+    length, n_q, d = q.shape
+    n_kv = k_cache.shape[1]
+    _check(_lib.load().mocap_chunk_attn_noalloc(_ptr(q), _ptr(k_cache), _ptr(v_cache), prefix,
+                                                length, n_q, n_kv, d, scale, _ptr(out), _ptr(lse),
+                                                _stream(stream)),
+           "mocap_chunk_attn_noalloc")
+
+
 def mocap_chunk_attn_varlen(q, k_cache, v_cache, items: Sequence[tuple], out, lse, scale: float,
                             stream=None):
     """Many (q_row, kv_row, prefix, len) items in one launch; lse is [Hq, q_rows_total]."""

@@ -871,25 +871,12 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(
 }
 
 // ------------------------------------------------------------------ host --
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void *ptr = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  });
-  return fn;
-}
 
 // [rows, heads, d] bf16 tensor, box = 64 columns x 1 head x box_rows rows,
 // 128B swizzle.
 bool make_map(CUtensorMap *map, const void *ptr, int64_t rows, int heads, int d,
               int box_rows = kBlockM) {
-  auto fn = encode_fn();
+  auto fn = tensor_map_encoder();
   if (fn == nullptr) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(heads),
                         static_cast<cuuint64_t>(rows)};
@@ -933,19 +920,6 @@ SplitPlan split_layout(int splits, int64_t len, int n_q_heads, int head_dim) {
   sp.lse_off = (sp.o_bytes + 255) / 256 * 256;
   sp.bytes = sp.lse_off + static_cast<size_t>(splits) * n_q_heads * len * sizeof(float);
   return sp;
-}
-
-int sm_count_cached() {
-  static int cached[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-  if (cached[dev] == 0) {
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-      n = 148;
-    cached[dev] = n;
-  }
-  return cached[dev];
 }
 
 // Split count for one chunk: list-schedule the CTAs (heaviest first, one per
@@ -1169,7 +1143,7 @@ mocap::SplitPlan plan_for(int64_t prefix, int64_t len, int32_t n_q_heads, int32_
       prefix > mocap::kMaxRows - len)
     return mocap::SplitPlan();
   int splits =
-      mocap::choose_splits(prefix, len, n_q_heads, n_kv_heads, head_dim, mocap::sm_count_cached());
+      mocap::choose_splits(prefix, len, n_q_heads, n_kv_heads, head_dim, mocap::device_sm_count());
   // MOCAP_SPLIT_KV: 0 never splits; 1..4 forces that count (tests, tuning),
   // capped so the first row block still has a key tile per split.
   if (const char *env = std::getenv("MOCAP_SPLIT_KV")) {

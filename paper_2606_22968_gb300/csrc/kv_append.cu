@@ -50,19 +50,6 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(const uint4 *__rest
   }
 }
 
-int sm_count() {
-  static int cached[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-  if (cached[dev] == 0) {
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-      n = 148;
-    cached[dev] = n;
-  }
-  return cached[dev];
-}
-
 }  // namespace
 
 extern "C" mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk, void *k_cache,
@@ -83,7 +70,7 @@ extern "C" mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk
   const int64_t n = len * row_elems / 8;  // 16-byte vectors per tensor
   const int64_t dst_off = offset * row_elems / 8;
   const int64_t want = (2 * n + kThreads * kUnroll - 1) / (kThreads * kUnroll);
-  const int64_t cap = static_cast<int64_t>(sm_count()) * kCtasPerSm;
+  const int64_t cap = static_cast<int64_t>(mocap::device_sm_count()) * kCtasPerSm;
   const int blocks = static_cast<int>(std::max<int64_t>(1, std::min(want, cap)));
   kv_append_kernel<<<blocks, kThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
       static_cast<const uint4 *>(k_chunk), static_cast<const uint4 *>(v_chunk),

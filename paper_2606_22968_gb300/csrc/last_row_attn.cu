@@ -419,25 +419,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) last_row_kernel(const __
   merge_group<D>(p, sm, r, g, n_parts);
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn3() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void *ptr = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  });
-  return fn;
-}
-
 // [rows, heads, d] bf16, box {64, 1, 128}: row t of a 64-dim box sits at
 // t * 128 bytes, its 16-byte chunks permuted by t & 7 when swizzled.
 bool make_kv_map(CUtensorMap *map, const void *ptr, int64_t rows, int heads, int d,
                  bool swizzle) {
-  auto fn = encode_fn3();
+  auto fn = tensor_map_encoder();
   if (fn == nullptr) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(heads),
                         static_cast<cuuint64_t>(rows)};
@@ -449,19 +435,6 @@ bool make_kv_map(CUtensorMap *map, const void *ptr, int64_t rows, int heads, int
             elem, CU_TENSOR_MAP_INTERLEAVE_NONE,
             swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-int sm_count_lr() {
-  static int cached[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-  if (cached[dev] == 0) {
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-      n = 148;
-    cached[dev] = n;
-  }
-  return cached[dev];
 }
 
 // Tiles per CTA so that all (request, group) key ranges give about
@@ -477,7 +450,7 @@ LrPlan plan_splits(const int64_t *kv_len, int n_req, int n_kv_heads) {
     total += tr;
     max_tiles = std::max(max_tiles, tr);
   }
-  const int64_t target_ctas = static_cast<int64_t>(kCtasPerSm) * sm_count_lr();
+  const int64_t target_ctas = static_cast<int64_t>(kCtasPerSm) * device_sm_count();
   int64_t per = (total * n_kv_heads + target_ctas - 1) / target_ctas;
   per = std::max<int64_t>(1, per);
   per = std::max<int64_t>(per, (max_tiles + kMaxParts - 1) / kMaxParts);

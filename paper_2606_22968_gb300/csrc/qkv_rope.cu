@@ -335,23 +335,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   cluster_barrier();  // neither CTA leaves while the pair still shares state
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn2() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void *ptr = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  });
-  return fn;
-}
-
 // 2-D bf16 [rows, cols] row-major, box {64 cols, box_rows}, 128-byte swizzle.
 bool make_map_2d(CUtensorMap *map, const void *ptr, int64_t rows, int64_t cols, int box_rows) {
-  auto fn = encode_fn2();
+  auto fn = tensor_map_encoder();
   if (fn == nullptr) return false;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
   cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
@@ -360,19 +346,6 @@ bool make_map_2d(CUtensorMap *map, const void *ptr, int64_t rows, int64_t cols, 
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box,
             elem, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-int sm_count_qkv() {
-  static int cached[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-  if (cached[dev] == 0) {
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-      n = 148;
-    cached[dev] = n;
-  }
-  return cached[dev];
 }
 
 }  // namespace
@@ -430,7 +403,7 @@ extern "C" mocap_status mocap_qkv_rope_append(const void *x, const void *w_qkv, 
   }
 
   const int64_t tiles = static_cast<int64_t>(prm.m_pairs) * prm.n_tiles;
-  const int grid = 2 * static_cast<int>(std::min<int64_t>(tiles, std::max(1, sm_count_qkv() / 2)));
+  const int grid = 2 * static_cast<int>(std::min<int64_t>(tiles, std::max(1, device_sm_count() / 2)));
   auto launch = [&](auto kern) -> mocap_status {
     static bool attr_done[2][64] = {};
     int dev = 0;

@@ -1,4 +1,6 @@
-// status.cu -- device status word for bounded-wait timeouts, status strings.
+// status.cu -- per-device runtime state shared by the kernels' host code:
+// the status word for bounded-wait timeouts, the SM count, the tensor-map
+// encoder; status strings.
 #include <mutex>
 
 #include "internal.h"
@@ -13,6 +15,33 @@ std::mutex g_status_mu;
 }  // namespace
 
 namespace mocap {
+
+int device_sm_count() {
+  static int cached[kMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 152;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 152;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *ptr = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
 
 uint32_t *device_status_ptr() {
   int dev = 0;

@@ -39,6 +39,13 @@ def test_library_exports_every_declared_symbol(lib):
         assert hasattr(lib, name), name
 
 
+def test_binding_has_every_declared_entry_point():
+    # the Python layer carries the C names (argument marshalling only)
+    import paper_2606_22968_gb300 as m
+    for name in _declared():
+        assert callable(getattr(m, name, None)), name
+
+
 def test_build_entry_compiles_for_sm103a():
     import __graft_entry__  # noqa: F401
     from paper_2606_22968_gb300 import _build

@@ -101,3 +101,21 @@ def test_noalloc_rejects_split_beyond_scratch(lib, monkeypatch):
     assert _call_noalloc(lib, q, k, v, prefix, out, lse, 0.088) == 1  # MOCAP_EINVAL
     torch.cuda.synchronize()
     assert torch.count_nonzero(out).item() == 0  # nothing was enqueued
+
+
+def test_python_binding_noalloc_equals_c_call(lib, monkeypatch):
+    # the package's same-named function marshals the same call
+    import paper_2606_22968_gb300 as m
+    monkeypatch.setenv("MOCAP_SPLIT_KV", "2")
+    prefix, length, hq, hkv, d = 1000, 300, 8, 2, 128
+    q, k, v = _inputs(prefix, length, hq, hkv, d, seed=11)
+    scale = 1.0 / math.sqrt(d)
+    out_c = torch.empty_like(q)
+    lse_c = torch.empty((hq, length), device=q.device, dtype=torch.float32)
+    assert _call_noalloc(lib, q, k, v, prefix, out_c, lse_c, scale) == 0
+    out_p = torch.full_like(q, float("nan"))
+    lse_p = torch.full((hq, length), float("nan"), device=q.device, dtype=torch.float32)
+    m.mocap_chunk_attn_noalloc(q, k, v, prefix, out_p, lse_p, scale)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == m.MOCAP_OK
+    assert torch.equal(out_p, out_c) and torch.equal(lse_p, lse_c)
