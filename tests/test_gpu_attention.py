@@ -557,3 +557,56 @@ def test_split_combine_formula_and_determinism(m, monkeypatch, prefix, length, h
     idx = torch.as_tensor(rows, device=dev)
     o_or, l_or = chunk_rows_oracle(f64(q[idx]), f64(k), f64(v), prefix, rows, scale)
     assert_close(out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_or, l_or, "merged")
+
+
+def _random_case(i):
+    """Case i of a seeded sweep: prefix, ragged length, head ratio, head dim,
+    kernel form, forced split count, and whether the cache has NaN rows past
+    prefix + len."""
+    rng = np.random.default_rng(20261202 + i)
+    heads = [(4, 4), (8, 2), (12, 4), (16, 2), (32, 8), (16, 1), (64, 8)]
+    hq, hkv = heads[int(rng.integers(len(heads)))]
+    d = 128 if rng.random() < 0.7 else 64
+    prefix = int(rng.choice([0, int(rng.integers(1, 128)), int(rng.integers(128, 8192))]))
+    length = int(rng.choice([int(rng.integers(1, 129)), int(rng.integers(129, 3000))]))
+    pair = str(int(rng.integers(2)))
+    split = [None, "1", "2", "3", "4"][int(rng.integers(5))]
+    extra = int(rng.integers(0, 300)) if rng.random() < 0.35 else 0
+    return prefix, length, hq, hkv, d, pair, split, extra
+
+
+@pytest.mark.parametrize("case", range(100))
+def test_random_shapes_sweep(m, monkeypatch, case):
+    """Seeded random shapes against the oracle on sampled rows (first and
+    last rows, both sides of every tile boundary, a stride, random rows);
+    every output row must be finite.  Rows of the cache past prefix + len
+    hold NaN in some cases and must never be read."""
+    prefix, length, hq, hkv, d, pair, split, extra = _random_case(case)
+    monkeypatch.setenv("MOCAP_ATTN_PAIR", pair)
+    if split is None:
+        monkeypatch.delenv("MOCAP_SPLIT_KV", raising=False)
+    else:
+        monkeypatch.setenv("MOCAP_SPLIT_KV", split)
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(1000 + case)
+    s = prefix + length
+    q = _randn((length, hq, d), gen, dev)
+    k = torch.full((s + extra, hkv, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    v = torch.full((s + extra, hkv, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    k[:s] = _randn((s, hkv, d), gen, dev)
+    v[:s] = _randn((s, hkv, d), gen, dev)
+    scale = 1.0 / math.sqrt(d)
+    ws_bytes = m.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d)
+    ws = torch.full((max(ws_bytes, 16),), 0xFF, device=dev, dtype=torch.uint8)
+    out = torch.full((length, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    lse = torch.full((hq, length), float("nan"), device=dev, dtype=torch.float32)
+    m.mocap_chunk_attn(q, k, v, prefix, out, lse, scale, workspace=ws)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    assert torch.isfinite(out.float()).all() and torch.isfinite(lse).all()
+    rows = sample_rows(length, every=211, seed=case)
+    idx = torch.as_tensor(rows, device=dev)
+    o_ref, l_ref = chunk_rows_oracle(f64(q[idx]), f64(k[:s]), f64(v[:s]), prefix, rows, scale)
+    assert_close(out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref, l_ref,
+                 f"case {case}: prefix {prefix} len {length} heads {hq}/{hkv} d {d} "
+                 f"pair {pair} split {split} extra {extra}")
