@@ -610,3 +610,49 @@ def test_random_shapes_sweep(m, monkeypatch, case):
     assert_close(out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref, l_ref,
                  f"case {case}: prefix {prefix} len {length} heads {hq}/{hkv} d {d} "
                  f"pair {pair} split {split} extra {extra}")
+
+
+@pytest.mark.parametrize("case", range(30))
+def test_random_varlen_sweep(m, monkeypatch, case):
+    """Seeded random varlen launches: 1..64 requests, each with a random
+    prefix and chunk (some empty), heads and head dim drawn per case.  The
+    launched rows match the oracle on sampled rows; rows outside every item
+    keep their contents."""
+    rng = np.random.default_rng(777 + case)
+    heads = [(4, 4), (8, 2), (16, 2), (32, 8), (16, 1), (64, 8)]
+    hq, hkv = heads[int(rng.integers(len(heads)))]
+    d = 128 if rng.random() < 0.7 else 64
+    monkeypatch.setenv("MOCAP_ATTN_PAIR", str(int(rng.integers(2))))
+    n_req = int(rng.choice([1, int(rng.integers(2, 9)), int(rng.integers(9, 65))]))
+    lens = [int(x) for x in rng.integers(1, 1500 if n_req > 8 else 5000, n_req)]
+    cu = np.concatenate([[0], np.cumsum(lens)]).tolist()
+    t = cu[-1]
+    items = []
+    for r, n in enumerate(lens):
+        pre = int(rng.integers(0, n))
+        ln = int(rng.integers(0, n - pre + 1)) if rng.random() < 0.9 else 0
+        items.append((cu[r] + pre, cu[r], pre, ln))
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(5000 + case)
+    q, k, v = _randn((t, hq, d), gen, dev), _randn((t, hkv, d), gen, dev), _randn((t, hkv, d), gen, dev)
+    out = torch.full((t, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    lse = torch.full((hq, t), float("nan"), device=dev, dtype=torch.float32)
+    scale = 1.0 / math.sqrt(d)
+    m.mocap_chunk_attn_varlen(q, k, v, items, out, lse, scale)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    covered = torch.zeros(t, dtype=torch.bool)
+    for (qr, _, _, ln) in items:
+        covered[qr:qr + ln] = True
+    cov = covered.to(dev)
+    assert torch.isfinite(out[cov].float()).all() and torch.isfinite(lse[:, cov]).all()
+    assert torch.isnan(out[~cov].float()).all() and torch.isnan(lse[:, ~cov]).all()
+    for j, (qr, kr, pre, ln) in enumerate(items[:16]):  # the oracle on the first 16 items
+        if ln == 0:
+            continue
+        rows = sample_rows(ln, every=257, seed=j)
+        idx = torch.as_tensor(rows + qr, device=dev)
+        o_ref, l_ref = chunk_rows_oracle(f64(q[idx]), f64(k[kr:kr + pre + ln]),
+                                         f64(v[kr:kr + pre + ln]), pre, rows, scale)
+        assert_close(out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref, l_ref,
+                     f"case {case} item {j}: prefix {pre} len {ln} heads {hq}/{hkv} d {d}")

@@ -109,3 +109,37 @@ def test_last_row_workspace_garbage_and_reuse(m):
     o_ref, l_ref = A.chunk_attention(f64(q[1:2]), f64(k[a:]), f64(v[a:]), lens[1] - 1, 0.088)
     assert_close(outs[0][0][1:2].float().cpu().numpy(), outs[0][1][:, 1:2].cpu().numpy(), o_ref,
                  l_ref, "request 1")
+
+
+@pytest.mark.parametrize("case", range(30))
+def test_random_last_row_sweep(m, case):
+    """Seeded random last-row calls: 1..64 requests of 1..20000 keys, group
+    sizes up to 16, head dim 64 or 128, NaN cache rows past every request;
+    each request's row against the oracle."""
+    rng = np.random.default_rng(31337 + case)
+    heads = [(4, 4), (8, 2), (16, 2), (32, 8), (16, 1), (64, 8), (64, 4)]
+    hq, hkv = heads[int(rng.integers(len(heads)))]
+    d = 128 if rng.random() < 0.7 else 64
+    n = int(rng.choice([1, int(rng.integers(2, 9)), int(rng.integers(9, 65))]))
+    lens = [int(x) for x in rng.integers(1, 20001 if n <= 8 else 3000, n)]
+    cu = np.concatenate([[0], np.cumsum(lens)]).tolist()
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(900 + case)
+    total = cu[-1] + 5
+    k = torch.randn((total, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    v = torch.randn((total, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    k[cu[-1]:] = float("nan")
+    v[cu[-1]:] = float("nan")
+    q = torch.randn((n, hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    scale = 1.0 / math.sqrt(d)
+    out = torch.full((n, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    lse = torch.full((hq, n), float("nan"), device=dev, dtype=torch.float32)
+    m.mocap_last_row_attn(q, k, v, cu[:-1], lens, out, lse, scale)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    for r, length in enumerate(lens):
+        a = cu[r]
+        o_ref, l_ref = A.chunk_attention(f64(q[r:r + 1]), f64(k[a:a + length]),
+                                         f64(v[a:a + length]), length - 1, scale)
+        assert_close(out[r:r + 1].float().cpu().numpy(), lse[:, r:r + 1].cpu().numpy(), o_ref,
+                     l_ref, f"case {case} request {r} (len {length}, heads {hq}/{hkv}, d {d})")
