@@ -150,3 +150,28 @@ def test_run_stage_projection_then_attention(m):
                                          vf[:b[i + 1]], b[i], rows, w.scale)
         assert_close(pf.out[b[i]:b[i + 1]][idx].float().cpu().numpy(),
                      pf.chunk_lse(i)[:, idx].cpu().numpy(), o_ref, l_ref, f"chunk {i}")
+
+
+def _random_projection_case(i):
+    rng = np.random.default_rng(4242 + i)
+    while True:
+        hkv = int(rng.choice([1, 2, 4, 8]))
+        hq = hkv * int(rng.choice([1, 2, 4, 8]))
+        d = 128 if rng.random() < 0.7 else 64
+        if (hq + 2 * hkv) * d % 256 == 0 and (hq + 2 * hkv) * d <= 4096:
+            break
+    hidden = 8 * int(rng.integers(1, 129))
+    length = int(rng.choice([int(rng.integers(1, 129)), int(rng.integers(129, 1500))]))
+    offset = int(rng.choice([0, int(rng.integers(1, 1000)), int(rng.integers(1000, 200000))]))
+    theta = float(rng.choice([10000.0, 500000.0, 1000000.0]))
+    return length, hidden, hq, hkv, d, offset, theta
+
+
+@pytest.mark.parametrize("case", range(25))
+def test_random_projection_sweep(m, case):
+    """Seeded random shapes of the fused QKV projection + RoPE + append
+    (any hidden size that keeps 16-byte rows, whole 256-column output
+    tiles, positions up to 200000) against the oracle, every element; cache
+    rows outside the chunk keep their bytes."""
+    length, hidden, hq, hkv, d, offset, theta = _random_projection_case(case)
+    test_qkv_rope_append_matches_oracle(m, length, hidden, hq, hkv, d, offset, theta)
