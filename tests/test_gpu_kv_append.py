@@ -53,3 +53,16 @@ def test_append_rejects_overflow(m):
     k = torch.zeros((4, 8, 128), device=dev, dtype=torch.bfloat16)
     with pytest.raises(m.MocapError):
         m.mocap_kv_append(k, k, kc, kc.clone(), 7)
+
+
+@pytest.mark.parametrize("case", range(30))
+def test_random_append_sweep(m, case):
+    """Seeded random appends (rows a whole number of 16-byte vectors):
+    bitwise equal to the oracle's copy, every other cache row untouched."""
+    rng = np.random.default_rng(60 + case)
+    hkv = int(rng.choice([1, 2, 4, 8, 16]))
+    d = int(rng.choice([8, 16, 64, 128, 256]))
+    length = int(rng.choice([int(rng.integers(1, 64)), int(rng.integers(64, 20000))]))
+    offset = int(rng.integers(0, 50000))
+    cap = offset + length + int(rng.integers(0, 100))
+    test_append_bitwise_with_sentinels(m, cap, offset, length, hkv, d)
