@@ -295,6 +295,13 @@ typedef struct {
  *   items        HOST array of n_items descriptors (read during the call only)
  *   q_rows_total rows of the packed q / out buffers and row stride of lse
  *   kv_rows_total rows of the packed caches (bounds check only)
+ *   workspace, workspace_bytes: optional caller-owned device scratch
+ *                (16-byte aligned).  Used only when exactly one item has
+ *                rows: with at least mocap_chunk_attn_workspace_size(prefix,
+ *                len, ...) bytes for that item, its key range may be split
+ *                as in mocap_chunk_attn (a late chunk of one long request
+ *                fills the GPU's SMs instead of leaving a second, almost
+ *                empty wave).  Several items never split.
  * Items must not write overlapping output rows.  Same requirements and
  * errors as mocap_chunk_attn; n_items == 0 is a no-op.
  */
@@ -303,6 +310,7 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
                                      int64_t q_rows_total, int64_t kv_rows_total,
                                      int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
                                      float scale, void *out, float *lse,
+                                     void *workspace, size_t workspace_bytes,
                                      mocap_stream_t stream);
 
 /*

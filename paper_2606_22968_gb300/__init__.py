@@ -135,16 +135,21 @@ def mocap_chunk_attn_noalloc(q, k_cache, v_cache, prefix: int, out, lse, scale: 
 
 
 def mocap_chunk_attn_varlen(q, k_cache, v_cache, items: Sequence[tuple], out, lse, scale: float,
-                            stream=None):
-    """Many (q_row, kv_row, prefix, len) items in one launch; lse is [Hq, q_rows_total]."""
+                            workspace=None, stream=None):
+    """Many (q_row, kv_row, prefix, len) items in one launch; lse is [Hq, q_rows_total].
+    With one non-empty item, ``workspace`` (as for mocap_chunk_attn) lets it split."""
     q_rows, n_q, d = q.shape
     n_kv = k_cache.shape[1]
     arr = (VarlenItem * max(1, len(items)))()
     for i, (q_row, kv_row, prefix, length) in enumerate(items):
         arr[i] = VarlenItem(q_row, kv_row, prefix, length)
+    if workspace is not None and not workspace.is_contiguous():
+        raise ValueError("workspace must be contiguous")
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(_lib.load().mocap_chunk_attn_varlen(_ptr(q), _ptr(k_cache), _ptr(v_cache), arr,
                                                len(items), q_rows, k_cache.shape[0], n_q, n_kv,
-                                               d, scale, _ptr(out), _ptr(lse), _stream(stream)),
+                                               d, scale, _ptr(out), _ptr(lse), _ptr(workspace),
+                                               ws_bytes, _stream(stream)),
            "mocap_chunk_attn_varlen")
 
 

@@ -32,7 +32,7 @@ SIGNATURES = {
                                          c_vp, c_vp, c_vp]),
     "mocap_chunk_attn_varlen": (c_i32, [c_vp, c_vp, c_vp, ctypes.POINTER(VarlenItem), c_i32,
                                         c_i64, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp, c_vp,
-                                        c_vp]),
+                                        c_vp, c_sz, c_vp]),
     "mocap_last_row_attn_workspace_size": (c_sz, [ctypes.POINTER(c_i64), c_i32, c_i32, c_i32,
                                                    c_i32]),
     "mocap_last_row_attn": (c_i32, [c_vp, c_vp, c_vp, ctypes.POINTER(c_i64), ctypes.POINTER(c_i64),

@@ -1099,10 +1099,13 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
   }
   if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
   if (sp.splits > 1) {
-    const int64_t len = items[0].len;
+    // the item's rows start at q_row of the packed out / lse (0 for a
+    // single-chunk call)
+    const int64_t len = items[0].len, q_row = items[0].q_row;
     const int64_t warps = len * sh.n_q_heads;
     attn_combine_kernel<D><<<static_cast<unsigned>((warps + 7) / 8), 256, 0, stream>>>(
-        prm.o_part, prm.lse_part, sp.splits, len, sh.n_q_heads, prm.out, lse, lse_stride, status);
+        prm.o_part, prm.lse_part, sp.splits, len, sh.n_q_heads,
+        prm.out + q_row * sh.n_q_heads * D, lse + q_row, lse_stride, status);
     if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
   }
   return MOCAP_OK;
@@ -1189,7 +1192,8 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
                                                 int64_t q_rows_total, int64_t kv_rows_total,
                                                 int32_t n_q_heads, int32_t n_kv_heads,
                                                 int32_t head_dim, float scale, void *out,
-                                                float *lse, mocap_stream_t stream) {
+                                                float *lse, void *workspace,
+                                                size_t workspace_bytes, mocap_stream_t stream) {
   const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
   const mocap_status st = mocap::check_shape(sh, scale);
   if (st != MOCAP_OK) return st;
@@ -1197,6 +1201,7 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
   if (n_items > 0 && items == nullptr) return MOCAP_EINVAL;
   if (q_rows_total < 0 || kv_rows_total < 0) return MOCAP_EINVAL;
   if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
+  if (workspace != nullptr && !mocap::aligned16(workspace)) return MOCAP_EINVAL;
   std::vector<HostItem> list;
   for (int i = 0; i < n_items; ++i) {
     const mocap_varlen_item &x = items[i];
@@ -1207,6 +1212,16 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
     if (x.len > 0) list.push_back({x.q_row, x.kv_row, x.prefix, x.len});
   }
   if (list.empty()) return MOCAP_OK;
+  if (list.size() == 1) {
+    // One item: the single-chunk plan, key-range split included when the
+    // caller's workspace holds its partials.
+    const HostItem &x = list[0];
+    mocap::SplitPlan sp = plan_for(x.prefix, x.len, n_q_heads, n_kv_heads, head_dim);
+    if (sp.splits > 1 && (workspace == nullptr || workspace_bytes < sp.bytes))
+      sp = mocap::SplitPlan();
+    return mocap::dispatch<1>(q, k_cache, v_cache, list, q_rows_total, sh, scale, out, lse,
+                              reinterpret_cast<cudaStream_t>(stream), sp, workspace);
+  }
   // Heaviest items first (their last row blocks see the most keys).
   std::stable_sort(list.begin(), list.end(), [](const HostItem &a, const HostItem &b) {
     return a.prefix + a.len > b.prefix + b.len;

@@ -69,13 +69,20 @@ class ChunkedPrefill:
         self.out = torch.empty((total, w.n_q_heads, w.head_dim), **kw)
         self.lse = torch.empty((w.n_q_heads * total,), device=self.device, dtype=torch.float32)
         self.single = len(w.seq_lens) == 1
-        # Split-KV scratch for the single-request path: the largest any chunk uses.
+        # Split-KV scratch: the largest any launch uses.  A single request
+        # splits any chunk that gains from it; several requests split only
+        # the steps left with one request's chunk (the tail of the longest
+        # request), since a launch of several items never splits.
         self.workspace = None
-        if self.single and split_kv:
-            b = self.bounds[0]
-            need = max(mocap_chunk_attn_workspace_size(b[i], b[i + 1] - b[i], w.n_q_heads,
-                                                       w.n_kv_heads, w.head_dim)
-                       for i in range(len(b) - 1))
+        if split_kv:
+            one = [(0, i) for i in range(len(self.bounds[0]) - 1)] if self.single else \
+                [step[0] for step in self.steps() if len(step) == 1]
+            need = 0
+            for r, c in one:
+                b = self.bounds[r]
+                need = max(need, mocap_chunk_attn_workspace_size(b[c], b[c + 1] - b[c],
+                                                                 w.n_q_heads, w.n_kv_heads,
+                                                                 w.head_dim))
             if need > 0:
                 self.workspace = torch.empty((need,), device=self.device, dtype=torch.uint8)
 
@@ -142,7 +149,8 @@ class ChunkedPrefill:
                 b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
                 items.append((self.cu[r] + b0, self.cu[r], b0, b1 - b0))
             mocap_chunk_attn_varlen(q, self.k_cache, self.v_cache, items, self.out,
-                                    self.lse_packed(), w.scale, stream=stream)
+                                    self.lse_packed(), w.scale, workspace=self.workspace,
+                                    stream=stream)
         if events is not None:
             events[2].record(stream)
 

@@ -152,7 +152,7 @@ def test_varlen_rejects_bad_items_before_launch(lib):
     def call(items, q_rows=1000, kv_rows=1000, n=None):
         arr = (VarlenItem * max(1, len(items)))(*[VarlenItem(*x) for x in items])
         return f(FAKE, FAKE, FAKE, arr, len(items) if n is None else n, q_rows, kv_rows, 8, 2, 128,
-                 0.1, FAKE, FAKE, None)
+                 0.1, FAKE, FAKE, None, 0, None)
 
     assert call([(0, 0, 0, 10)], q_rows=5) == 1          # q rows past the buffer
     assert call([(0, 0, 995, 10)]) == 1                  # kv rows past the cache

@@ -656,3 +656,48 @@ def test_random_varlen_sweep(m, monkeypatch, case):
                                          f64(v[kr:kr + pre + ln]), pre, rows, scale)
         assert_close(out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref, l_ref,
                      f"case {case} item {j}: prefix {pre} len {ln} heads {hq}/{hkv} d {d}")
+
+
+@pytest.mark.parametrize("forced", [None, "2", "3", "4"])
+def test_varlen_single_item_splits_like_the_chunk_call(m, monkeypatch, forced):
+    """A varlen launch with one item and a workspace takes the single-chunk
+    plan, key-range split included: bitwise equal to mocap_chunk_attn on the
+    item's rows, other rows of the packed buffers untouched."""
+    if forced is None:
+        monkeypatch.delenv("MOCAP_SPLIT_KV", raising=False)
+    else:
+        monkeypatch.setenv("MOCAP_SPLIT_KV", forced)
+    hq, hkv, d = 32, 8, 128
+    lens = [3000, 23168, 1500]           # the long request's late chunk is the item
+    cu = np.concatenate([[0], np.cumsum(lens)]).tolist()
+    t = cu[-1]
+    pre, ln = 17152, 1280
+    item = (cu[1] + pre, cu[1], pre, ln)
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(4321)
+    q, k, v = _randn((t, hq, d), gen, dev), _randn((t, hkv, d), gen, dev), _randn((t, hkv, d), gen, dev)
+    need = m.mocap_chunk_attn_workspace_size(pre, ln, hq, hkv, d)
+    assert need > 0, "shape chosen so that the plan splits"
+    ws = torch.full((need,), 0xFF, device=dev, dtype=torch.uint8)
+    out = torch.full((t, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+    lse = torch.full((hq, t), float("nan"), device=dev, dtype=torch.float32)
+    m.mocap_chunk_attn_varlen(q, k, v, [item], out, lse, 0.088, workspace=ws)
+    ws2 = torch.full((need,), 0x00, device=dev, dtype=torch.uint8)
+    o1 = torch.empty((ln, hq, d), device=dev, dtype=torch.bfloat16)
+    l1 = torch.empty((hq, ln), device=dev, dtype=torch.float32)
+    a = cu[1]
+    m.mocap_chunk_attn(q[a + pre:a + pre + ln], k[a:a + pre + ln], v[a:a + pre + ln], pre, o1, l1,
+                       0.088, workspace=ws2)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    rows = slice(a + pre, a + pre + ln)
+    assert torch.equal(out[rows], o1) and torch.equal(lse[:, rows], l1)
+    mask = torch.ones(t, dtype=torch.bool, device=dev)
+    mask[rows] = False
+    assert torch.isnan(out[mask].float()).all() and torch.isnan(lse[:, mask]).all()
+    sr = sample_rows(ln, every=97, seed=3)
+    idx = torch.as_tensor(sr + a + pre, device=dev)
+    o_ref, l_ref = chunk_rows_oracle(f64(q[idx]), f64(k[a:a + pre + ln]), f64(v[a:a + pre + ln]),
+                                     pre, sr, 0.088)
+    assert_close(out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref, l_ref,
+                 f"split {forced}")
