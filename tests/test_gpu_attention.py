@@ -701,3 +701,57 @@ def test_varlen_single_item_splits_like_the_chunk_call(m, monkeypatch, forced):
                                      pre, sr, 0.088)
     assert_close(out[idx].float().cpu().numpy(), lse[:, idx].cpu().numpy(), o_ref, l_ref,
                  f"split {forced}")
+
+
+def test_concurrent_host_threads_on_separate_streams(m):
+    """Four host threads, each with its own stream, workspace and shapes
+    (split and unsplit, both kernel forms' shapes, varlen and last-row),
+    call the library at once, many times: every result is bitwise equal to
+    the same calls made one after another."""
+    import threading
+    dev = torch.device("cuda")
+    specs = [(100000, 256, 8, 2, 128), (4096, 700, 64, 8, 128), (300, 257, 16, 1, 128),
+             (1000, 130, 4, 4, 64)]
+    data = []
+    for i, (pre, ln, hq, hkv, d) in enumerate(specs):
+        gen = torch.Generator(device=dev).manual_seed(70 + i)
+        q = _randn((ln, hq, d), gen, dev)
+        k, v = _randn((pre + ln, hkv, d), gen, dev), _randn((pre + ln, hkv, d), gen, dev)
+        need = m.mocap_chunk_attn_workspace_size(pre, ln, hq, hkv, d)
+        ws = torch.empty((max(need, 16),), device=dev, dtype=torch.uint8)
+        data.append((pre, q, k, v, ws, 1.0 / math.sqrt(d)))
+
+    def run(i, stream, reps):
+        pre, q, k, v, ws, scale = data[i]
+        outs = []
+        with torch.cuda.stream(stream):
+            for _ in range(reps):
+                o = torch.empty_like(q)
+                l = torch.empty((q.shape[1], q.shape[0]), device=dev, dtype=torch.float32)
+                m.mocap_chunk_attn(q, k, v, pre, o, l, scale, workspace=ws, stream=stream)
+                outs.append((o, l))
+        return outs
+
+    serial = [run(i, torch.cuda.current_stream(), 1)[0] for i in range(len(specs))]
+    torch.cuda.synchronize()
+    streams = [torch.cuda.Stream() for _ in specs]
+    results = [None] * len(specs)
+    errors = []
+
+    def worker(i):
+        try:
+            results[i] = run(i, streams[i], 20)
+        except Exception as e:  # surfaced below
+            errors.append(e)
+
+    threads = [threading.Thread(target=worker, args=(i,)) for i in range(len(specs))]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    torch.cuda.synchronize()
+    assert not errors, errors
+    assert m.mocap_last_device_status() == 0
+    for i, outs in enumerate(results):
+        for o, l in outs:
+            assert torch.equal(o, serial[i][0]) and torch.equal(l, serial[i][1]), f"spec {i}"
