@@ -1,6 +1,7 @@
 // status.cu -- per-device runtime state shared by the kernels' host code:
 // the status word for bounded-wait timeouts, the SM count, the tensor-map
 // encoder; status strings.
+#include <atomic>
 #include <mutex>
 
 #include "internal.h"
@@ -17,16 +18,17 @@ std::mutex g_status_mu;
 namespace mocap {
 
 int device_sm_count() {
-  static int cached[kMaxDevices] = {};
+  // atomics: threads may race to fill an entry (with the same value)
+  static std::atomic<int> cached[kMaxDevices] = {};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 152;
-  if (cached[dev] == 0) {
-    int n = 0;
+  int n = cached[dev].load(std::memory_order_relaxed);
+  if (n == 0) {
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
       n = 152;
-    cached[dev] = n;
+    cached[dev].store(n, std::memory_order_relaxed);
   }
-  return cached[dev];
+  return n;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
