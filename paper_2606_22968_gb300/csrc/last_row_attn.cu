@@ -219,26 +219,36 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) last_row_kernel(const __
   const uint32_t mma_bar = base + L::kBars + 8u * kStages;
   const int64_t prow = static_cast<int64_t>(split) * p.n_req + r;
 
-  __shared__ uint32_t abort_flag;
-  if (t == 0) abort_flag = *reinterpret_cast<volatile uint32_t *>(p.status);
-  __syncthreads();
-  if (abort_flag != 0u) return;
-  if (n <= 0) return;  // past the request's keys: this split takes no part
-  const int n_parts = (tiles + p.tiles_per_cta - 1) / p.tiles_per_cta;  // splits with keys
-
-  // Q_g (unscaled bf16) and a zeroed P tile, in the MMA's swizzled layout.
-  for (int i = t; i < kN * D; i += kThreads) {
-    const int h = i / D, c = i % D;
-    const __nv_bfloat16 v = h < G ? p.q[(static_cast<int64_t>(r) * p.n_q_heads + g * G + h) * D + c]
-                                  : __float2bfloat16(0.0f);
-    *reinterpret_cast<__nv_bfloat16 *>(sm + L::kQ + sw_off(h, c, kN)) = v;
-  }
-  for (int i = t; i < kN * kKeys / 8; i += kThreads)
-    reinterpret_cast<uint4 *>(sm + L::kP)[i] = make_uint4(0, 0, 0, 0);
+  // TMEM first: the SM starts its next CTA of this kernel only after this
+  // one has given up its allocation permit, so anything placed before the
+  // relinquish delays every later CTA on the SM.
   if (warp == 0) {
     tmem_alloc(base + L::kTmemSlot, kTmemCols);
     tmem_relinquish();
   }
+  __shared__ uint32_t abort_flag;
+  if (t == 0) abort_flag = *reinterpret_cast<volatile uint32_t *>(p.status);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  // an aborted launch, or a split past the request's keys, takes no part
+  if (abort_flag != 0u || n <= 0) {
+    if (warp == 0) tmem_dealloc(*reinterpret_cast<volatile uint32_t *>(sm + L::kTmemSlot), kTmemCols);
+    return;
+  }
+  const int n_parts = (tiles + p.tiles_per_cta - 1) / p.tiles_per_cta;  // splits with keys
+
+  // Q_g (unscaled bf16) and a zeroed P tile, in the MMA's swizzled layout;
+  // 16-byte pieces (8 dims of one head), which the swizzle keeps whole.
+  for (int i = t; i < kN * D / 8; i += kThreads) {
+    const int h = i / (D / 8), c = (i % (D / 8)) * 8;
+    const uint4 v = h < G ? *reinterpret_cast<const uint4 *>(
+                                p.q + (static_cast<int64_t>(r) * p.n_q_heads + g * G + h) * D + c)
+                          : make_uint4(0, 0, 0, 0);
+    *reinterpret_cast<uint4 *>(sm + L::kQ + sw_off(h, c, kN)) = v;
+  }
+  for (int i = t; i < kN * kKeys / 8; i += kThreads)
+    reinterpret_cast<uint4 *>(sm + L::kP)[i] = make_uint4(0, 0, 0, 0);
   if (t == 0) {
     for (int s = 0; s < kStages; ++s) mbar_init(full(s), 1);
     mbar_init(mma_bar, 1);
