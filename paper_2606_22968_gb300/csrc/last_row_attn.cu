@@ -219,9 +219,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) last_row_kernel(const __
   const uint32_t mma_bar = base + L::kBars + 8u * kStages;
   const int64_t prow = static_cast<int64_t>(split) * p.n_req + r;
 
-  // TMEM first: the SM starts its next CTA of this kernel only after this
-  // one has given up its allocation permit, so anything placed before the
-  // relinquish delays every later CTA on the SM.
+  // TMEM first.  Per-CTA timestamps on GB300 showed an SM starting its next
+  // CTA of this kernel only once the CTA before it had given up its TMEM
+  // allocation permit, so anything placed before the relinquish delays every
+  // later CTA on the SM (Q staging there cost the third CTA ~10 us).
   if (warp == 0) {
     tmem_alloc(base + L::kTmemSlot, kTmemCols);
     tmem_relinquish();
