@@ -12,6 +12,7 @@
  *
  *   mocap_lbcp_partition      chunk boundaries (host, exact integers)
  *   mocap_lbcp_partition_dp   boundaries from Algorithm 1's stage-1 DP (host)
+ *   mocap_lbcp_gemm_weight    the DP's GEMM-term weight from measured rates (host)
  *   mocap_kv_append           chunk K/V -> contiguous bf16 KV cache (device)
  *   mocap_qkv_rope_append     QKV projection + RoPE + KV append (device GEMM)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
@@ -110,15 +111,35 @@ typedef enum {
  * provided.
  *
  *   num_stages   N >= 1 pipeline stages
- *   gemm_weight  >= 0, weight of the linear term (same doubled units)
+ *   gemm_weight  0 .. 2^40, weight of the linear term (same doubled units)
  *   boundaries   HOST array of num_chunks + 1 int64, written on success
- * MOCAP_EINVAL for bad arguments; MOCAP_EUNSUPPORTED when M * U^2 > 4e9 (the
- * O(M U^2) host work would be too long; use a coarser granularity).
+ * MOCAP_EINVAL for bad arguments, including N (2 U^2 + gemm_weight U) >=
+ * 2^62 (the compared objective t_sum + (N - 1) t_max could leave int64);
+ * MOCAP_EUNSUPPORTED when M * U^2 > 4e9 (the O(M U^2) host work would be too
+ * long; use a coarser granularity).
  */
 mocap_status mocap_lbcp_partition_dp(int64_t seq_len, int32_t num_chunks,
                                      int32_t granularity, int32_t num_stages,
                                      mocap_cost_model model, int64_t gemm_weight,
                                      int64_t *boundaries);
+
+/*
+ * mocap_lbcp_gemm_weight -- the gemm_weight argument of
+ * mocap_lbcp_partition_dp for chunk stages whose measured cost is
+ * a * (causal query-key pairs) + b * (rows): Eq. 1's attention term plus its
+ * GEMM term (Sec. 3.2).  A chunk of k units of `granularity` g rows starting
+ * at unit s has about g^2 k (s + k/2) pairs and g k rows, so in the DP's
+ * doubled units its cost is proportional to k (2 s + k) + w k with
+ * w = 2 b / (g a), rounded half up.
+ *
+ *   attn_s_per_pair  a > 0 (seconds, or any unit shared with b)
+ *   gemm_s_per_row   b >= 0
+ *   weight           HOST int64, written on success
+ * MOCAP_EINVAL for a null pointer, granularity < 1, a <= 0, b < 0, NaN, or a
+ * weight above 2^40.  Pure host arithmetic.
+ */
+mocap_status mocap_lbcp_gemm_weight(double attn_s_per_pair, double gemm_s_per_row,
+                                    int32_t granularity, int64_t *weight);
 
 /*
  * mocap_kv_append -- write a chunk's K and V into the KV cache.

@@ -146,10 +146,17 @@ def evaluate_chunk(k: int, s: int, model: int, gemm_weight: int) -> int:
     return attn + gemm_weight * k
 
 
-def dp_boundaries(seq_len: int, num_chunks: int, granularity: int, num_stages: int,
-                  model: int = COST_CAUSAL, gemm_weight: int = 0) -> List[int]:
-    """Chunk boundaries from stage 1 of Algorithm 1 (exact integers)."""
-    units = _check(seq_len, num_chunks, granularity)
+def dp_tables(units: int, num_chunks: int, num_stages: int, model: int = COST_CAUSAL,
+              gemm_weight: int = 0):
+    """The three tables of Algorithm 1's stage-1 DP over ``units`` positions.
+
+    Returns dicts ``t_max``, ``t_sum`` and ``ss`` keyed by ``(m, s)`` (chunk
+    index m in 1..M, start position s); a state that no valid suffix reaches
+    has no key (its objective counts as +infinity).  The terminal state
+    ``(M + 1, units)`` has ``t_max = t_sum = 0``.
+    """
+    if units < num_chunks or num_chunks < 1:
+        raise ValueError("1 <= num_chunks <= units required")
     if num_stages < 1 or gemm_weight < 0:
         raise ValueError("num_stages >= 1 and gemm_weight >= 0 required")
     M, S, N = num_chunks, units, num_stages
@@ -169,8 +176,17 @@ def dp_boundaries(seq_len: int, num_chunks: int, granularity: int, num_stages: i
                 if cur not in t_max or \
                         tsum_new + (N - 1) * tmax_new < t_sum[cur] + (N - 1) * t_max[cur]:
                     t_max[cur], t_sum[cur], ss[cur] = tmax_new, tsum_new, k
+    return t_max, t_sum, ss
+
+
+def dp_boundaries(seq_len: int, num_chunks: int, granularity: int, num_stages: int,
+                  model: int = COST_CAUSAL, gemm_weight: int = 0) -> List[int]:
+    """Chunk boundaries from stage 1 of Algorithm 1 (exact integers): the
+    chunk slice scheme ``ss`` read forward from state (1, 0)."""
+    units = _check(seq_len, num_chunks, granularity)
+    _, _, ss = dp_tables(units, num_chunks, num_stages, model, gemm_weight)
     out, s = [0], 0
-    for m in range(1, M + 1):
+    for m in range(1, num_chunks + 1):
         s += ss[(m, s)]
         out.append(granularity * s)
     out[-1] = seq_len

@@ -75,6 +75,20 @@ def mocap_lbcp_partition_dp(seq_len: int, num_chunks: int, granularity: int = 12
     return list(out)
 
 
+def mocap_lbcp_gemm_weight(attn_s_per_pair: float, gemm_s_per_row: float,
+                           granularity: int = 128) -> int:
+    """The stage-1 DP's GEMM weight for chunk stages that cost
+    ``a * pairs + b * rows`` (a = attention seconds per causal pair, b =
+    projection seconds per row)."""
+    out = ctypes.c_int64(0)
+    st = _lib.load().mocap_lbcp_gemm_weight(float(attn_s_per_pair), float(gemm_s_per_row),
+                                            granularity, ctypes.byref(out))
+    if st == MOCAP_EINVAL:
+        raise ValueError("attn_s_per_pair > 0 and gemm_s_per_row >= 0 required")
+    _check(st, "mocap_lbcp_gemm_weight")
+    return out.value
+
+
 def mocap_kv_append(k_chunk, v_chunk, k_cache, v_cache, offset: int, stream=None):
     """Copy chunk K/V ([len, Hkv, d] bf16) into cache rows [offset, offset+len)."""
     length, n_kv, d = k_chunk.shape

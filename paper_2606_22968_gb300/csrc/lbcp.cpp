@@ -91,6 +91,17 @@ extern "C" mocap_status mocap_lbcp_partition_dp(int64_t seq_len, int32_t num_chu
   if (static_cast<double>(M) * static_cast<double>(U) * static_cast<double>(U) > 4e9)
     return MOCAP_EUNSUPPORTED;  // O(M U^2) host work; use a coarser granularity
   if (gemm_weight > (int64_t(1) << 40)) return MOCAP_EINVAL;
+  // Every chunk cost is at most 2 U^2 + gemm_weight U (Eq. 1's form with
+  // s + k <= U), so t_sum and t_max are too, and the compared objective
+  // t_sum + (N - 1) t_max is at most N (2 U^2 + gemm_weight U).  Refuse
+  // arguments for which that bound could leave int64.
+  {
+    const unsigned __int128 t_bound = static_cast<unsigned __int128>(2) * U * U +
+                                      static_cast<unsigned __int128>(gemm_weight) * U;
+    if (t_bound * static_cast<unsigned __int128>(num_stages) >=
+        (static_cast<unsigned __int128>(1) << 62))
+      return MOCAP_EINVAL;
+  }
   const int64_t nm1 = num_stages - 1;
   const size_t W = static_cast<size_t>(U + 1);
   auto at = [&](int64_t m, int64_t s) { return static_cast<size_t>(m) * W + static_cast<size_t>(s); };
@@ -125,5 +136,19 @@ extern "C" mocap_status mocap_lbcp_partition_dp(int64_t seq_len, int32_t num_chu
     boundaries[m] = granularity * s;
   }
   boundaries[M] = seq_len;
+  return MOCAP_OK;
+}
+
+// Eq. 1 with its GEMM term: a chunk stage costs a * (causal pairs) + b *
+// (rows).  In the DP's doubled units of g rows, a chunk of k units at unit s
+// has about g^2 k (s + k/2) pairs and g k rows, so its cost is proportional
+// to k (2 s + k) + w k with w = 2 b / (g a), rounded to the nearest integer.
+extern "C" mocap_status mocap_lbcp_gemm_weight(double attn_s_per_pair, double gemm_s_per_row,
+                                               int32_t granularity, int64_t *weight) {
+  if (weight == nullptr || granularity < 1) return MOCAP_EINVAL;
+  if (!(attn_s_per_pair > 0.0) || !(gemm_s_per_row >= 0.0)) return MOCAP_EINVAL;  // NaN too
+  const double w = 2.0 * gemm_s_per_row / (static_cast<double>(granularity) * attn_s_per_pair);
+  if (!(w <= static_cast<double>(int64_t(1) << 40))) return MOCAP_EINVAL;  // inf, too large
+  *weight = static_cast<int64_t>(w + 0.5);  // w >= 0: round half up
   return MOCAP_OK;
 }

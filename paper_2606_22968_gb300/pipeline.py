@@ -16,19 +16,17 @@ import torch
 
 from . import (MOCAP_COST_CAUSAL, MOCAP_PART_LBCP, MOCAP_PART_UNIFORM, mocap_chunk_attn,
                mocap_chunk_attn_varlen, mocap_chunk_attn_workspace_size, mocap_kv_append,
-               mocap_lbcp_partition, mocap_lbcp_partition_dp, mocap_qkv_rope_append)
+               mocap_lbcp_gemm_weight, mocap_lbcp_partition, mocap_lbcp_partition_dp,
+               mocap_qkv_rope_append)
 from .workloads import GRANULARITY, Workload, request_offsets
 
 
 def gemm_weight(attn_s_per_pair: float, gemm_s_per_row: float, granularity: int = 128) -> int:
     """The DP's GEMM weight for a chunk stage costing ``a * pairs + b * rows``
     (Eq. 1 with its GEMM term; a = attention seconds per causal (query, key)
-    pair, b = projection seconds per row).  In the DP's doubled units of
-    ``granularity`` rows, a chunk of k units at s costs k (2 s + k) + w k with
-    w = 2 b / (g a)."""
-    if attn_s_per_pair <= 0 or gemm_s_per_row < 0:
-        raise ValueError("attn_s_per_pair > 0 and gemm_s_per_row >= 0 required")
-    return max(0, int(round(2.0 * gemm_s_per_row / (granularity * attn_s_per_pair))))
+    pair, b = projection seconds per row), computed by the library
+    (``mocap_lbcp_gemm_weight``)."""
+    return mocap_lbcp_gemm_weight(attn_s_per_pair, gemm_s_per_row, granularity)
 
 
 def stage_balanced_bounds(seq_len: int, num_chunks: int, attn_s_per_pair: float,

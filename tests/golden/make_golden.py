@@ -1,7 +1,13 @@
-"""Writes partition_boundaries.txt from the oracle alone (oracle/partition.py).
+"""Writes the partition fixtures from the oracle alone (oracle/partition.py).
 
 Run from the repository root:  python tests/golden/make_golden.py
-The cases are the five workloads' (seq_len, chunks) pairs plus ragged extras.
+  partition_boundaries.txt  the closed-form split of the five workloads'
+                            (seq_len, chunks) pairs plus ragged extras
+  dp_boundaries.txt         Algorithm 1's stage-1 DP on the 32768-token /
+                            16-chunk and 131072-token / 32-chunk shapes
+                            (N = 16 stages; causal cost, Eq. 1's cost, and
+                            the causal cost with a GEMM weight of 90)
+The DP rows of the 131072-token shape take a few minutes of pure Python.
 """
 import os
 import sys
@@ -28,15 +34,34 @@ CASES = [
     (100000, 9, 64, P.LBCP),
 ]
 
+# (seq_len, chunks, granularity, stages, cost model, gemm weight)
+DP_CASES = [
+    (32768, 16, 128, 16, P.COST_CAUSAL, 0),
+    (32768, 16, 128, 16, P.COST_EQ1, 0),
+    (32768, 16, 128, 16, P.COST_CAUSAL, 90),
+    (131072, 32, 128, 16, P.COST_CAUSAL, 0),
+    (131072, 32, 128, 16, P.COST_EQ1, 0),
+    (131072, 32, 128, 16, P.COST_CAUSAL, 90),
+]
+
 
 def main():
-    out = os.path.join(os.path.dirname(os.path.abspath(__file__)), "partition_boundaries.txt")
-    with open(out, "w") as f:
+    here = os.path.dirname(os.path.abspath(__file__))
+    with open(os.path.join(here, "partition_boundaries.txt"), "w") as f:
         f.write("# seq_len chunks granularity mode(0=uniform,1=lbcp): b_0 .. b_M\n")
         f.write("# written by tests/golden/make_golden.py from oracle/partition.py\n")
         for s, m, g, mode in CASES:
             b = P.boundaries(s, m, g, mode)
             f.write(f"{s} {m} {g} {mode}: " + " ".join(str(x) for x in b) + "\n")
+    with open(os.path.join(here, "dp_boundaries.txt"), "w") as f:
+        f.write("# seq_len chunks granularity stages model(0=causal,1=eq1) gemm_weight: "
+                "b_0 .. b_M\n")
+        f.write("# written by tests/golden/make_golden.py from oracle/partition.py "
+                "(dp_boundaries)\n")
+        for s, m, g, n, model, gemm in DP_CASES:
+            b = P.dp_boundaries(s, m, g, n, model, gemm)
+            f.write(f"{s} {m} {g} {n} {model} {gemm}: " + " ".join(str(x) for x in b) + "\n")
+            f.flush()
 
 
 if __name__ == "__main__":

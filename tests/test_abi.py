@@ -233,3 +233,51 @@ def test_stage_balanced_bounds_weight_and_dp():
     for a, b in ((1.84e-11, 1.06e-7), (1e-11, 0.0)):
         got = stage_balanced_bounds(32768, 16, a, b)
         assert got == P.dp_boundaries(32768, 16, 128, 16, P.COST_CAUSAL, gemm_weight(a, b))
+
+
+def test_dp_hand_worked_tie_case_bit_exact(lib):
+    """Algorithm 1's tie rule (strict improvement, k ascending) on the case
+    worked by hand in tests/golden/dp_tie_case.txt."""
+    from tests.golden_utils import dp_tie_case
+    case, _, _, bounds = dp_tie_case()
+    out = (ctypes.c_int64 * (case["chunks"] + 1))()
+    assert lib.mocap_lbcp_partition_dp(case["seq_len"], case["chunks"], case["granularity"],
+                                       case["stages"], case["model"], case["gemm"], out) == 0
+    assert list(out) == bounds
+
+
+def test_dp_golden_rows_of_the_workload_shapes(lib):
+    """The DP on the 32768/16 and 131072/32 shapes against rows the oracle wrote."""
+    from tests.golden_utils import dp_boundary_rows
+    rows = dp_boundary_rows()
+    assert {r[0] for r in rows} == {32768, 131072}
+    for s, m, g, n, model, gemm, b in rows:
+        out = (ctypes.c_int64 * (m + 1))()
+        assert lib.mocap_lbcp_partition_dp(s, m, g, n, model, gemm, out) == 0
+        assert list(out) == b, (s, m, g, n, model, gemm)
+
+
+def test_dp_rejects_arguments_whose_objective_could_overflow(lib):
+    out = (ctypes.c_int64 * 40)()
+    big_n = 2 ** 31 - 1
+    # U = 1024: N (2 U^2 + w U) with w = 2^40 far beyond 2^62
+    assert lib.mocap_lbcp_partition_dp(131072, 32, 128, big_n, 0, 2 ** 40, out) == 1
+    assert lib.mocap_lbcp_partition_dp(131072, 32, 128, 2 ** 22, 0, 2 ** 40, out) == 1
+    assert lib.mocap_lbcp_partition_dp(131072, 32, 128, 16, 0, 2 ** 40, out) == 0  # 1.8e16
+    # U = 63245 (M U^2 < 4e9): 2 U^2 N with N = 2^31 - 1 is about 1.7e19 > 2^62
+    assert lib.mocap_lbcp_partition_dp(63245, 1, 1, big_n, 0, 0, out) == 1
+    # inside the bound: U = 1024 with the largest N, and a realistic weight
+    assert lib.mocap_lbcp_partition_dp(131072, 32, 128, big_n, 0, 0, out) == 0
+    assert lib.mocap_lbcp_partition_dp(131072, 32, 128, 16, 1, 90, out) == 0
+
+
+def test_gemm_weight_entry_point(lib):
+    w = ctypes.c_int64(-1)
+    assert lib.mocap_lbcp_gemm_weight(1.0, 64.0, 128, ctypes.byref(w)) == 0 and w.value == 1
+    assert lib.mocap_lbcp_gemm_weight(1.84e-11, 1.06e-7, 128, ctypes.byref(w)) == 0
+    assert w.value == 90
+    assert lib.mocap_lbcp_gemm_weight(1.0, 96.0, 128, ctypes.byref(w)) == 0 and w.value == 2
+    for bad in ((0.0, 1.0, 128), (1.0, -1.0, 128), (float("nan"), 1.0, 128), (1.0, 1.0, 0),
+                (1e-30, 1.0, 128)):
+        assert lib.mocap_lbcp_gemm_weight(*bad, ctypes.byref(w)) == 1, bad
+    assert lib.mocap_lbcp_gemm_weight(1.0, 1.0, 128, None) == 1

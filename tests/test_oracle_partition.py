@@ -267,3 +267,75 @@ def test_dp_beats_closed_form_objective_on_workload_shapes():
         dp = P.dp_boundaries(s, m, 128, 16)
         cf = P.boundaries(s, m, 128)
         assert P.dp_objective(dp, 128, 16) <= P.dp_objective(cf, 128, 16)
+
+
+# ---------------------------------------------------------------------------
+# Algorithm 1's exact output under ties (Sec. 4.2, stage 1): the table of a
+# case worked by hand from the algorithm's steps (tests/golden/dp_tie_case.txt)
+# fixes which of several equal-objective splits the DP keeps.
+from tests.golden_utils import dp_boundary_rows, dp_tie_case  # noqa: E402
+
+
+def test_dp_tables_match_the_hand_worked_tie_case():
+    case, states, terminal, bounds = dp_tie_case()
+    t_max, t_sum, ss = P.dp_tables(case["units"], case["chunks"], case["stages"],
+                                   case["model"], case["gemm"])
+    got = {key: (ss[key], t_max[key], t_sum[key]) for key in ss}
+    assert got == states
+    m_end, s_end, tmax_end, tsum_end = terminal
+    assert (t_max[(m_end, s_end)], t_sum[(m_end, s_end)]) == (tmax_end, tsum_end)
+    assert set(t_max) == set(states) | {(m_end, s_end)}  # no other state is reached
+    assert P.dp_boundaries(case["seq_len"], case["chunks"], case["granularity"], case["stages"],
+                           case["model"], case["gemm"]) == bounds
+
+
+def test_hand_worked_case_has_two_optima_brute_force():
+    # independent of the DP: the objective t_sum + (N - 1) t_max over every
+    # composition of 6 units into 3 chunks has two minimisers; the golden
+    # boundaries are one of them
+    case, _, _, bounds = dp_tie_case()
+    n = case["stages"]
+    objs = {}
+    for sizes in _compositions(case["units"], case["chunks"]):
+        costs = _chunk_costs(sizes, P.COST_CAUSAL, 0)
+        objs[sizes] = sum(costs) + (n - 1) * max(costs)
+    best = min(objs.values())
+    optima = sorted(s for s, v in objs.items() if v == best)
+    assert optima == [(3, 2, 1), (4, 1, 1)]
+    g = case["granularity"]
+    assert tuple((bounds[i + 1] - bounds[i]) // g for i in range(3)) == (3, 2, 1)
+
+
+def _mutant_dp(replace_from, replace_to):
+    """The oracle's dp_tables with one planted change, compiled on the CPU."""
+    import inspect
+    src = inspect.getsource(P.dp_tables)
+    assert src.count(replace_from) == 1, replace_from
+    ns = dict(P.__dict__)
+    exec(src.replace(replace_from, replace_to), ns)
+    return ns["dp_tables"]
+
+
+@pytest.mark.parametrize("mutation", [
+    ("tsum_new + (N - 1) * tmax_new < t_sum[cur]", "tsum_new + (N - 1) * tmax_new <= t_sum[cur]"),
+    ("range(1, S - s - (M - m) + 1)", "range(S - s - (M - m), 0, -1)"),
+])
+def test_reversed_tie_rule_fails_the_hand_worked_case(mutation):
+    # a "<=" comparison or k tried downward keeps the same objective values
+    # but a different split, which the golden table catches
+    case, states, _, _ = dp_tie_case()
+    dp = _mutant_dp(*mutation)
+    t_max, t_sum, ss = dp(case["units"], case["chunks"], case["stages"], case["model"],
+                          case["gemm"])
+    assert (t_max[(1, 0)], t_sum[(1, 0)]) == states[(1, 0)][1:]  # same objective ...
+    assert ss[(1, 0)] != states[(1, 0)][0]                      # ... other split
+
+
+def test_dp_golden_rows_of_the_32k_shape():
+    # the rows written by make_golden.py from the oracle alone; re-derived here
+    # for the 32768-token shape (the 131072-token rows take minutes in Python)
+    rows = [r for r in dp_boundary_rows() if r[0] == 32768]
+    assert len(rows) == 3
+    for s, m, g, n, model, gemm, b in rows:
+        assert P.dp_boundaries(s, m, g, n, model, gemm) == b
+        _check_invariants(b, s, m, g)
