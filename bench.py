@@ -58,6 +58,12 @@ def parse_args():
     ap.add_argument("--case", default=None,
                     help="profiling case 'prefix,len,Hq,Hkv,d': one chunk attention launch "
                          "repeated warmup+steps times (no JSON metric line)")
+    ap.add_argument("--case-split", choices=["none", "auto"], default="none",
+                    help="with --case: 'auto' passes the library's split-KV workspace, as "
+                         "the prompt pipeline does (the launch may split and add a combine)")
+    ap.add_argument("--case-append", default=None,
+                    help="profiling case 'rows,Hkv,d': one KV append launch repeated "
+                         "warmup+steps times")
     ap.add_argument("--case-qkv", default=None,
                     help="profiling case 'len,hidden,Hq,Hkv,d': one QKV projection launch "
                          "repeated warmup+steps times")
@@ -98,24 +104,70 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(workload_name):
-    """DRAM bytes per launch of the attention kernel from the committed ncu
-    summary, if it was taken on the current kernel source (else None)."""
+def attn_min_bytes(prefix, length, n_q_heads, n_kv_heads, head_dim):
+    """Algorithmic HBM bytes of one chunk attention launch: K and V of the
+    prefix plus the chunk read once, Q read, O written (bf16), LSE written
+    (fp32)."""
+    kv = 2 * (prefix + length) * n_kv_heads * head_dim * 2
+    return kv + 2 * length * n_q_heads * head_dim * 2 + 4 * length * n_q_heads
+
+
+def read_traffic_cases():
+    """Single-kernel ncu captures of chunk_attn_kernel (one launch each) from
+    the committed summary: {(prefix, len, Hq, Hkv, d): DRAM bytes}, or None
+    when the summary was not taken on the current kernel source."""
     path = os.path.join(ROOT, "profiles", "chunk_attn_dram_traffic.txt")
     try:
-        vals = {}
+        cases, src = {}, None
         with open(path) as f:
             for line in f:
-                if ":" in line and not line.startswith("#"):
-                    k, v = line.split(":", 1)
-                    vals[k.strip()] = v.strip()
-        if vals.get("kernel_source_sha256_16") != kernel_source_hash():
+                line = line.strip()
+                if not line or line.startswith("#"):
+                    continue
+                key, val = line.split(":", 1)
+                if key == "kernel_source_sha256_16":
+                    src = val.strip()
+                elif key == "case":
+                    fields = val.split()
+                    shape = tuple(int(x) for x in fields[:5])
+                    kv = dict(x.split("=") for x in fields[5:])
+                    cases[shape] = float(kv["dram_bytes"])
+        if src != kernel_source_hash() or not cases:
             return None
-        if vals.get("workload") != workload_name:
-            return None
-        return float(vals["dram_bytes_per_launch_full_workload"])
+        return cases
     except Exception:
         return None
+
+
+def ncu_traffic(bounds, n_q_heads, n_kv_heads, head_dim):
+    """DRAM bytes per attention launch of a single-request prompt, averaged
+    over its chunks.  Each chunk's bytes are its algorithmic minimum times the
+    measured ratio (DRAM bytes / minimum) of the captured shapes, linearly
+    interpolated in the chunk's key count prefix + len (captured shapes of
+    the same heads and head dimension; outside their range the nearest
+    ratio).  None without current captures of these heads."""
+    cases = read_traffic_cases()
+    if cases is None:
+        return None
+    pts = sorted((p + n, b / attn_min_bytes(p, n, hq, hkv, d))
+                 for (p, n, hq, hkv, d), b in cases.items()
+                 if (hq, hkv, d) == (n_q_heads, n_kv_heads, head_dim))
+    if not pts:
+        return None
+
+    def ratio(keys):
+        if keys <= pts[0][0]:
+            return pts[0][1]
+        for (x0, r0), (x1, r1) in zip(pts, pts[1:]):
+            if keys <= x1:
+                return r0 + (r1 - r0) * (keys - x0) / (x1 - x0)
+        return pts[-1][1]
+
+    alg = [attn_min_bytes(b0, b1 - b0, n_q_heads, n_kv_heads, head_dim)
+           for b0, b1 in zip(bounds[:-1], bounds[1:])]
+    est = [a * ratio(b1) for a, b1 in zip(alg, bounds[1:])]
+    return {"traffic": sum(est) / len(est), "algorithmic": sum(alg) / len(alg),
+            "captured_shapes": len(pts)}
 
 
 class ClockSampler:
@@ -406,7 +458,17 @@ def ours_arm(args, rank, world, local):
     peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAK_TFLOPS))
     attn_avg_ms = statistics.mean(attn_step_ms)
     achieved = total_flops / (attn_avg_ms * 1e-3) / 1e12
-    traffic_per_launch = ncu_traffic(w.name)
+    traffic = ncu_traffic(pf.bounds[0], w.n_q_heads, w.n_kv_heads, w.head_dim) \
+        if pf.single else None
+    alg_bytes = statistics.mean(
+        attn_min_bytes(b0, b1 - b0, w.n_q_heads, w.n_kv_heads, w.head_dim)
+        for bnd in pf.bounds for b0, b1 in zip(bnd[:-1], bnd[1:]))
+    # The sustained peak was measured at its own median SM clock; at the
+    # bench's median clock the same tensor pipe delivers peak * f / f_peak.
+    peak_mhz = (peaks.get("clocks_under_load") or {}).get("sm_mhz_median")
+    frac_clock = None
+    if peak_mhz and clk.get("sm_mhz"):
+        frac_clock = achieved / (peak * clk["sm_mhz"] / float(peak_mhz))
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     app_gbs = append_bytes / (statistics.mean(app_step_ms) * 1e-3) / 1e9
 
@@ -429,9 +491,19 @@ def ours_arm(args, rank, world, local):
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak,
                      "peak_source": f"bf16_tflops_sustained ({peak_src})",
+                     "frac_at_peak_clock": frac_clock,
+                     "clock_note": (f"achieved / (peak x bench median SM clock {clk.get('sm_mhz')}"
+                                    f" MHz / peak's median SM clock {peak_mhz} MHz)"),
                      "kernel": "chunk_attn_kernel",
-                     "traffic": traffic_per_launch,
-                     "traffic_unit": "bytes per launch (avg over the step's launches)"},
+                     "traffic": None if traffic is None else traffic["traffic"],
+                     "algorithmic_bytes": alg_bytes,
+                     "traffic_over_algorithmic": None if traffic is None else
+                     traffic["traffic"] / traffic["algorithmic"],
+                     "traffic_unit": "bytes per launch (avg over the step's launches)",
+                     "traffic_source": None if traffic is None else
+                     (f"single-launch ncu captures of {traffic['captured_shapes']} chunk shapes "
+                      "(profiles/chunk_attn_dram_traffic.txt), DRAM/minimum ratio "
+                      "interpolated in keys per chunk")},
         "clocks": clk,
         # our kernels per timed region: one append per (request, chunk), one
         # attention launch per step, one split-KV combine per split chunk
@@ -747,13 +819,40 @@ def profile_case(args):
     vc = torch.randn((prefix + length, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
     out = torch.empty_like(q)
     lse = torch.empty((hq, length), device=dev, dtype=torch.float32)
+    ws_bytes = 0
+    ws = None
+    if args.case_split == "auto":
+        ws_bytes = m.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d)
+        if ws_bytes:
+            ws = torch.empty((ws_bytes,), device=dev, dtype=torch.uint8)
     ms = _repeat_timed(args, lambda: m.mocap_chunk_attn(q, kc, vc, prefix, out, lse,
-                                                        1.0 / math.sqrt(d)))
+                                                        1.0 / math.sqrt(d), workspace=ws))
     if m.mocap_last_device_status() != m.MOCAP_OK:
         raise RuntimeError("device wait expired")
     flops = 4 * hq * d * (length * prefix + length * (length + 1) // 2)
     print(json.dumps({"case": args.case, "ms": ms, "tflops": flops / ms / 1e9,
-                      "kv_bytes": 2 * (prefix + length) * hkv * d * 2}), flush=True)
+                      "split_workspace_bytes": ws_bytes,
+                      "min_bytes": attn_min_bytes(prefix, length, hq, hkv, d)}), flush=True)
+    return 0
+
+
+def profile_case_append(args):
+    """One KV append shape, repeated (ncu probe): rows of K and V into a cache
+    of the same size."""
+    import torch
+    import paper_2606_22968_gb300 as m
+    rows, hkv, d = (int(x) for x in args.case_append.split(","))
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(13)
+    k = torch.randn((rows, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    v = torch.randn((rows, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    kc, vc = torch.empty_like(k), torch.empty_like(v)
+    ms = _repeat_timed(args, lambda: m.mocap_kv_append(k, v, kc, vc, 0))
+    if not (torch.equal(kc, k) and torch.equal(vc, v)):
+        raise RuntimeError("append probe: cache differs from the chunk")
+    byts = 2 * 2 * rows * hkv * d * 2
+    print(json.dumps({"case_append": args.case_append, "ms": ms, "bytes": byts,
+                      "gb_per_s": byts / ms / 1e6}), flush=True)
     return 0
 
 
@@ -821,6 +920,8 @@ def main():
     args = parse_args()
     if args.case:
         return profile_case(args)
+    if args.case_append:
+        return profile_case_append(args)
     if args.case_qkv:
         return profile_case_qkv(args)
     if args.case_last_row:

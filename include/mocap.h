@@ -266,16 +266,22 @@ size_t mocap_chunk_attn_workspace_size(int64_t prefix, int64_t len, int32_t n_q_
  * MOCAP_NOALLOC_SCRATCH_BYTES (32 MiB) array compiled into the library: it
  * calls no cudaMalloc, cudaFree or other allocating routine.
  *
- *   - Results: as mocap_chunk_attn with enough workspace (same split plan,
- *     same kernels).
- *   - Limit: if the split the library would use for this shape needs more
- *     than MOCAP_NOALLOC_SCRATCH_BYTES (see mocap_chunk_attn_workspace_size),
- *     the call returns MOCAP_EINVAL and enqueues nothing.  Shapes that need no
- *     split run the single-pass kernel and use no scratch.
+ *   - Results: bitwise those of mocap_chunk_attn given a workspace of
+ *     MOCAP_NOALLOC_SCRATCH_BYTES bytes (same split plan, same kernels).
+ *   - Limit: when the split the library would use for this shape needs more
+ *     than MOCAP_NOALLOC_SCRATCH_BYTES (see mocap_chunk_attn_workspace_size;
+ *     e.g. 2 splits of a 2048-row chunk with 64 query heads need 135 MB), the
+ *     call runs the single-pass kernel instead, as mocap_chunk_attn does with
+ *     too small a workspace: the same results up to fp32 rounding order, but
+ *     a late chunk's last wave may leave SMs idle.  Shapes that need no split
+ *     run the single-pass kernel too and use no scratch.
  *   - Every GPU that loads the library holds the array until the process
  *     exits.  The first call on a device looks up the array's device address
  *     (cudaGetSymbolAddress, once per device, that device current); make
- *     that first call before any stream capture.
+ *     that first call before any stream capture.  The address is kept per
+ *     device ordinal: the entry point assumes each device's primary context
+ *     (the one the CUDA runtime API uses), not a context the caller created
+ *     with the driver API.
  *   - All calls on a device share the array.  A call writes every scratch
  *     byte it reads, so nothing has to start at zero, but calls whose work
  *     overlaps on the GPU (e.g. on different streams) race on the array.

@@ -64,7 +64,7 @@ def _rows_for_head(q_rows, pos, k, v, scale):
     return o, lse
 
 
-def chunk_attention(q_chunk, k_cache, v_cache, prefix, scale, rows=None):
+def chunk_attention(q_chunk, k_cache, v_cache, prefix, scale, rows=None, heads=None):
     """Attention of one chunk against the KV prefix plus itself (Sec. 2.2).
 
     q_chunk  [len, Hq, d] float64 -- the chunk's queries, global rows
@@ -72,7 +72,10 @@ def chunk_attention(q_chunk, k_cache, v_cache, prefix, scale, rows=None):
     k_cache, v_cache [>= prefix+len, Hkv, d] float64 -- KV of all rows so far.
     rows     optional 1-D array of chunk-local row indices to evaluate
              (sampling); default all rows.
-    Returns (O [n, Hq, d], LSE [Hq, n]) for the n requested rows.
+    heads    optional list of query heads to evaluate (sampling); default
+             all Hq heads.  Each head is computed exactly as in the full call.
+    Returns (O [n, H, d], LSE [H, n]) for the n requested rows and the H
+    requested heads, in the order given.
     """
     length, n_q, d = q_chunk.shape
     n_kv = k_cache.shape[1]
@@ -84,16 +87,19 @@ def chunk_attention(q_chunk, k_cache, v_cache, prefix, scale, rows=None):
     rows = np.asarray(rows, dtype=np.int64)
     if k_cache.shape[0] < prefix + (int(rows.max()) + 1 if rows.size else 0):
         raise ValueError("cache shorter than prefix + rows")
-    out = np.zeros((rows.size, n_q, d), dtype=np.float64)
-    lse = np.zeros((n_q, rows.size), dtype=np.float64)
-    for h in range(n_q):
+    heads = list(range(n_q)) if heads is None else [int(h) for h in heads]
+    if any(h < 0 or h >= n_q for h in heads):
+        raise ValueError("head index out of range")
+    out = np.zeros((rows.size, len(heads), d), dtype=np.float64)
+    lse = np.zeros((len(heads), rows.size), dtype=np.float64)
+    for j, h in enumerate(heads):
         g = h // group
         for a in range(0, rows.size, _ROW_BLOCK):
             r = rows[a:a + _ROW_BLOCK]
             o_b, l_b = _rows_for_head(q_chunk[r, h, :], prefix + r,
                                       k_cache[:, g, :], v_cache[:, g, :], scale)
-            out[a:a + r.size, h, :] = o_b
-            lse[h, a:a + r.size] = l_b
+            out[a:a + r.size, j, :] = o_b
+            lse[j, a:a + r.size] = l_b
     return out, lse
 
 

@@ -1249,7 +1249,9 @@ std::mutex g_noalloc_mu;
 
 // Device address of g_noalloc_scratch on the current device.  The name is
 // only a host-side handle in host code, so the address is looked up once per
-// device (that device current) and cached; nullptr if the lookup fails.
+// device (that device current) and cached; nullptr if the lookup fails.  The
+// cache is keyed by device ordinal, i.e. it assumes the CUDA runtime's primary
+// context of each device (the context every runtime-API caller uses).
 uint8_t *noalloc_scratch() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
@@ -1274,8 +1276,10 @@ extern "C" mocap_status mocap_chunk_attn_noalloc(const void *q, const void *k_ca
   if (prefix < 0 || len < 0 || prefix > mocap::kMaxRows - len) return MOCAP_EINVAL;
   if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
   if (len == 0) return MOCAP_OK;
-  const mocap::SplitPlan sp = plan_for(prefix, len, n_q_heads, n_kv_heads, head_dim);
-  if (sp.bytes > MOCAP_NOALLOC_SCRATCH_BYTES) return MOCAP_EINVAL;  // beyond the fixed scratch
+  // Exactly mocap_chunk_attn with a workspace of MOCAP_NOALLOC_SCRATCH_BYTES:
+  // a split whose partials do not fit runs as the single-pass kernel.
+  mocap::SplitPlan sp = plan_for(prefix, len, n_q_heads, n_kv_heads, head_dim);
+  if (sp.splits > 1 && sp.bytes > MOCAP_NOALLOC_SCRATCH_BYTES) sp = mocap::SplitPlan();
   void *ws = nullptr;
   if (sp.splits > 1) {
     ws = noalloc_scratch();

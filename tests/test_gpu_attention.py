@@ -191,7 +191,7 @@ def test_varlen_equals_single_launches_bitwise(m):
 
 
 # ---------------------------------------------------------------- workloads --
-def _workload_parity(m, index, rows_fn, chunks=None):
+def _workload_parity(m, index, rows_fn, chunks=None, heads_fn=None):
     from paper_2606_22968_gb300 import workloads
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
     w = workloads.get(index)
@@ -203,7 +203,7 @@ def _workload_parity(m, index, rows_fn, chunks=None):
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == 0
     assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
-    return check_single_request(pf, q, k, v, rows_fn=rows_fn, chunks=chunks)
+    return check_single_request(pf, q, k, v, rows_fn=rows_fn, chunks=chunks, heads_fn=heads_fn)
 
 
 def test_workload1_tiny_all_elements(m):
@@ -224,10 +224,15 @@ def test_workload4_128k_lbcp_sampled(m):
                      chunks=[0, 1, 15, 29, 30, 31])
 
 
-def test_workload4_every_chunk_first_and_last_row(m):
-    # all 32 chunks at full size: each chunk's first row and its last row,
-    # which attends to the whole prefix plus the whole chunk
-    _workload_parity(m, 4, lambda n, i: np.array([0, n - 1]))
+def test_workload4_every_chunk_at_every_tile_edge(m):
+    # all 32 chunks at full size, element by element on: both sides of every
+    # 128-row tile edge, the first and last two rows (the last sees the whole
+    # prefix and the whole chunk), a 2000-row stride and random rows; four
+    # heads per chunk, rotating so the 32 chunks cover all 64 heads, every KV
+    # group and both head slots of both CTAs of a pair
+    from tests.parity_utils import rotating_heads
+    _workload_parity(m, 4, lambda n, i: sample_rows(n, every=2000, edge=2, seed=i),
+                     heads_fn=rotating_heads(64))
 
 
 def test_workload5_varlen_sampled(m):
@@ -350,6 +355,67 @@ def test_graph_replay_matches_eager_run(m, index):
         assert m.mocap_last_device_status() == 0
         assert torch.equal(pf.out, out_ref) and torch.equal(pf.lse, lse_ref)
         assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
+
+
+def _check_varlen_every_chunk(pf, q, k, v, rows_fn, heads_fn=None):
+    """Oracle check of a multi-request ChunkedPrefill on the rows
+    ``rows_fn(len, (request, chunk))`` of every chunk of every request."""
+    w = pf.w
+    lse = pf.lse_packed()
+    for r in range(len(w.seq_lens)):
+        a = pf.cu[r]
+        kf, vf = f64(k[a:a + w.seq_lens[r]]), f64(v[a:a + w.seq_lens[r]])
+        b = pf.bounds[r]
+        for i in range(len(b) - 1):
+            rows = rows_fn(b[i + 1] - b[i], (r, i))
+            heads = None if heads_fn is None else list(heads_fn(r * 64 + i))
+            idx = torch.as_tensor(rows + a + b[i], device=q.device)
+            o_ref, l_ref = chunk_rows_oracle(f64(q[idx]), kf[:b[i + 1]], vf[:b[i + 1]], b[i],
+                                             rows, w.scale, heads)
+            o_gpu, l_gpu = pf.out[idx], lse[:, idx]
+            if heads is not None:
+                o_gpu, l_gpu = o_gpu[:, heads], l_gpu[heads]
+            assert_close(o_gpu.float().cpu().numpy(), l_gpu.cpu().numpy(), o_ref, l_ref,
+                         f"request {r} chunk {i}")
+
+
+@pytest.mark.parametrize("index", [3, 4, 5])
+def test_graph_replay_against_oracle(m, index):
+    """The prompt replayed from one CUDA graph (outputs, caches and LSE
+    poisoned with NaN first) against the oracle on sampled rows of every
+    chunk, and bitwise against the eager run."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    from tests.parity_utils import rotating_heads
+    w = workloads.get(index)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev)
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    out_ref, lse_ref = pf.out.clone(), pf.lse.clone()
+    graph = pf.capture(q, k, v)
+    for t in (pf.out, pf.lse, pf.k_cache, pf.v_cache):
+        t.fill_(float("nan"))
+    graph.replay()
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
+    assert torch.equal(pf.out, out_ref) and torch.equal(pf.lse, lse_ref)
+    heads = rotating_heads(w.n_q_heads)
+    if index == 3:
+        check_single_request(pf, q, k, v, rows_fn=lambda n, i: sample_rows(n, every=509, edge=2,
+                                                                          seed=100 + i),
+                             heads_fn=heads)
+    elif index == 4:
+        check_single_request(pf, q, k, v,
+                             rows_fn=lambda n, i: np.array([0, 127, 128, n // 2, n - 1]),
+                             heads_fn=heads)
+    else:
+        _check_varlen_every_chunk(pf, q, k, v,
+                                  lambda n, ri: sample_rows(n, every=509, edge=2, seed=ri[0]),
+                                  heads_fn=heads)
+    del graph
 
 
 PAIR_CASES = [

@@ -81,6 +81,22 @@ def test_sampled_rows_equal_full_rows():
     assert np.max(np.abs(ls_ - lse[:, rows])) < 1e-13
 
 
+def test_sampled_heads_equal_full_heads():
+    # head sampling selects heads; against the brute-force definition too
+    q = _rand((40, 8, 6), 21)
+    k = _rand((40, 2, 6), 22)
+    v = _rand((40, 2, 6), 23)
+    o, lse = A.chunk_attention(q[10:], k, v, 10, 0.4)
+    heads = [7, 0, 4]
+    oh, lh = A.chunk_attention(q[10:], k, v, 10, 0.4, rows=[0, 5, 29], heads=heads)
+    assert np.max(np.abs(oh - o[[0, 5, 29]][:, heads])) < 1e-13
+    assert np.max(np.abs(lh - lse[heads][:, [0, 5, 29]])) < 1e-13
+    ob, lb = _brute(q[10:], k, v, 0.4, 10)
+    assert np.max(np.abs(oh - ob[[0, 5, 29]][:, heads])) < 1e-12
+    with pytest.raises(ValueError):
+        A.chunk_attention(q[10:], k, v, 10, 0.4, heads=[8])
+
+
 def test_chunked_equals_unchunked_random_boundaries():
     rnd = random.Random(11)
     s, hq, hkv, d = 611, 4, 2, 16

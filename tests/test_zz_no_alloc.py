@@ -2,9 +2,11 @@
 allocate device memory (a host program whose own pool owns the GPU's memory,
 or a serving loop that cannot afford cudaMalloc / cudaFree).  It keeps its
 split-KV partials in a fixed scratch array inside the library, so these tests
-check that, called twice in a row through the C ABI, it gives the results of
-mocap_chunk_attn with a caller-provided workspace, and that it refuses a
-shape whose partials would not fit the array.
+check that, called twice in a row through the C ABI, it gives bitwise the
+results of mocap_chunk_attn with a caller-provided workspace, and that a
+shape whose partials would not fit the array runs the single-pass kernel
+(bitwise mocap_chunk_attn without a workspace, and within the parity
+tolerances of the oracle).
 
 Kept in a file of its own that pytest collects last; it passes alone in a
 fresh process and after the other tests.
@@ -80,27 +82,47 @@ def test_noalloc_matches_workspace_entry_two_calls(lib, monkeypatch):
         assert st == 0
         torch.cuda.synchronize()
         assert lib.mocap_last_device_status(torch.cuda.current_stream().cuda_stream) == 0
-        # same results as the workspace entry point, within the parity tolerances
-        assert_close(out_n.float().cpu().numpy(), lse_n.cpu().numpy(),
-                     out_w.double().cpu().numpy(), lse_w.double().cpu().numpy(),
-                     f"call {i}: noalloc vs workspace")
+        # same split plan and kernels as the workspace entry point: bitwise equal
+        assert torch.equal(out_n, out_w), f"call {i}: noalloc vs workspace (O)"
+        assert torch.equal(lse_n, lse_w), f"call {i}: noalloc vs workspace (LSE)"
         # and against the float64 oracle
         o_ref, l_ref = A.chunk_attention(f64(q), f64(k), f64(v), prefix, scale)
         assert_close(out_n.float().cpu().numpy(), lse_n.cpu().numpy(), o_ref, l_ref,
                      f"call {i}: noalloc vs oracle")
 
 
-def test_noalloc_rejects_split_beyond_scratch(lib, monkeypatch):
-    # 2 splits x 2048 rows x 64 heads x (128 + 1) fp32 = 135 MB > 32 MiB
+def test_noalloc_runs_single_pass_when_the_split_exceeds_the_scratch(lib, monkeypatch):
+    # A late chunk of the 131072-token Llama-3-70B shape (64 query heads, 8 KV
+    # heads): the library splits its key range in two, whose partials
+    # (2 x 2048 rows x 64 heads x (128 + 1) fp32 = 135 MB) exceed the 32 MiB
+    # array, so the call runs the single-pass kernel: bitwise mocap_chunk_attn
+    # without a workspace, and the oracle on sampled rows and heads.
     monkeypatch.setenv("MOCAP_SPLIT_KV", "2")
-    prefix, length, hq, hkv, d = 4096, 2048, 64, 8, 128
+    prefix, length, hq, hkv, d = 129024 - 2048 + 77, 2048, 64, 8, 128
     assert lib.mocap_chunk_attn_workspace_size(prefix, length, hq, hkv, d) > SCRATCH_BYTES
     q, k, v = _inputs(prefix, length, hq, hkv, d, seed=7)
-    out = torch.zeros((length, hq, d), device=q.device, dtype=torch.bfloat16)
-    lse = torch.zeros((hq, length), device=q.device, dtype=torch.float32)
-    assert _call_noalloc(lib, q, k, v, prefix, out, lse, 0.088) == 1  # MOCAP_EINVAL
+    scale = 1.0 / math.sqrt(d)
+    stream = torch.cuda.current_stream().cuda_stream
+    out_n = torch.full((length, hq, d), float("nan"), device=q.device, dtype=torch.bfloat16)
+    lse_n = torch.full((hq, length), float("nan"), device=q.device, dtype=torch.float32)
+    assert _call_noalloc(lib, q, k, v, prefix, out_n, lse_n, scale) == 0
+    out_1 = torch.empty_like(out_n)
+    lse_1 = torch.empty_like(lse_n)
+    assert lib.mocap_chunk_attn(q.data_ptr(), k.data_ptr(), v.data_ptr(), prefix, length, hq,
+                                hkv, d, scale, out_1.data_ptr(), lse_1.data_ptr(), None, 0,
+                                stream) == 0
     torch.cuda.synchronize()
-    assert torch.count_nonzero(out).item() == 0  # nothing was enqueued
+    assert lib.mocap_last_device_status(stream) == 0
+    assert torch.equal(out_n, out_1) and torch.equal(lse_n, lse_1)
+    rows = np.array([0, 1, 127, 128, 1023, 1024, 1919, 2047])
+    heads = [0, 9, 18, 27, 36, 45, 54, 63]  # every KV group, every head slot of a pair
+    idx = torch.as_tensor(rows, device=q.device)
+    kf, vf = f64(k), f64(v)
+    q_rows = np.zeros((length, hq, d))
+    q_rows[rows] = f64(q[idx])
+    o_ref, l_ref = A.chunk_attention(q_rows, kf, vf, prefix, scale, rows=rows, heads=heads)
+    assert_close(out_n[idx][:, heads].float().cpu().numpy(), lse_n[heads][:, idx].cpu().numpy(),
+                 o_ref, l_ref, "noalloc single pass vs oracle")
 
 
 def test_python_binding_noalloc_equals_c_call(lib, monkeypatch):
