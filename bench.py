@@ -407,7 +407,15 @@ def ours_arm(args, rank, world, local):
     # per step (chunk index k): attention FLOP of every (request, k)
     step_flops = [sum(flops_chunks[r][c] for r, c in st) for st in steps_plan]
     total_flops = sum(step_flops)
-    append_bytes = 2 * 2 * w.total_tokens * w.n_kv_heads * w.head_dim * 2  # K,V x (rd+wr)
+    row_bytes = w.n_kv_heads * w.head_dim * 2
+
+    def rows_of(step):
+        return sum(pf.bounds[r][c + 1] - pf.bounds[r][c] for r, c in step)
+
+    append_bytes = 2 * 2 * w.total_tokens * row_bytes  # K, V x (read + write)
+    # with fused appends only step 0's chunks are appended by a launch of
+    # their own; the attention launches' idle warps append the rest
+    standalone_bytes = 2 * 2 * rows_of(steps_plan[0]) * row_bytes
 
     def one_step(ev=None):
         pf.partition()
@@ -470,7 +478,7 @@ def ours_arm(args, rank, world, local):
     if peak_mhz and clk.get("sm_mhz"):
         frac_clock = achieved / (peak * clk["sm_mhz"] / float(peak_mhz))
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
-    app_gbs = append_bytes / (statistics.mean(app_step_ms) * 1e-3) / 1e9
+    app_gbs = standalone_bytes / (statistics.mean(app_step_ms) * 1e-3) / 1e9
 
     line = {
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
@@ -486,8 +494,14 @@ def ours_arm(args, rank, world, local):
         "attn_frac_of_peak": achieved / peak,
         "per_chunk_attn_ms": {"min": min(per_chunk), "max": max(per_chunk),
                               "max_over_min": max(per_chunk) / min(per_chunk), "cv": cv},
-        "append": {"gb_per_s": app_gbs, "frac_of_hbm": app_gbs / hbm,
-                   "ms_per_step": statistics.mean(app_step_ms)},
+        "append": {"bytes_per_step": append_bytes,
+                   "standalone_bytes_per_step": standalone_bytes,
+                   "fused_bytes_per_step": append_bytes - standalone_bytes,
+                   "gb_per_s": app_gbs, "frac_of_hbm": app_gbs / hbm,
+                   "ms_per_step": statistics.mean(app_step_ms),
+                   "note": "gb_per_s: the step's standalone appends (step 0's chunks) between "
+                           "events in the timed steps; the other chunks' K/V are appended by "
+                           "the attention launch of the step before (mocap_chunk_attn_append)"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak,
                      "peak_source": f"bf16_tflops_sustained ({peak_src})",
@@ -505,9 +519,10 @@ def ours_arm(args, rank, world, local):
                       "(profiles/chunk_attn_dram_traffic.txt), DRAM/minimum ratio "
                       "interpolated in keys per chunk")},
         "clocks": clk,
-        # our kernels per timed region: one append per (request, chunk), one
-        # attention launch per step, one split-KV combine per split chunk
-        "gpu_launches": args.steps * (sum(1 + len(st) for st in steps_plan) + n_combines),
+        # our kernels per timed region: step 0's appends (one per request),
+        # one attention launch per step (carrying the next step's appends),
+        # one split-KV combine per split chunk
+        "gpu_launches": args.steps * (len(steps_plan[0]) + len(steps_plan) + n_combines),
     }
 
     if not args.no_e2e:
@@ -515,7 +530,8 @@ def ours_arm(args, rank, world, local):
         # thermal state of the GPU (the auxiliary measurements below add
         # about a minute of load first)
         line["e2e"] = measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world)
-    line["append"].update(measure_append_graph(m, w, pf, k, v, dev, append_bytes, hbm))
+    line["append"].update(measure_append_graph(m, w, pf, k, v, dev, hbm))
+    line["append"].update(measure_fusion(args, pf, w, q, k, v, dev, stream, total_flops))
     if not args.no_graph:
         line["graph_replay"] = measure_graph(args, pf, q, k, v, dev, stream, total_flops,
                                              w.total_tokens, world)
@@ -549,47 +565,90 @@ def ours_arm(args, rank, world, local):
     return 0
 
 
-def measure_append_graph(m, w, pf, k, v, dev, append_bytes, hbm, reps=5):
-    """Device time of the step's appends alone: all of them captured in one
-    CUDA graph and replayed back to back (no launch gaps, no attention in
-    between), so the figure is the append kernel's own bandwidth."""
+def measure_append_graph(m, w, pf, k, v, dev, hbm, reps=5):
+    """Device time of the append kernel alone, replayed from CUDA graphs (no
+    launch gaps, no attention in between): the step's standalone appends
+    (step 0's chunks) and, for comparison, every chunk's append as the
+    unfused pipeline launches them."""
     import torch
-    side = torch.cuda.Stream(dev)
-    side.wait_stream(torch.cuda.current_stream(dev))
-    graph = torch.cuda.CUDAGraph()
+    row_bytes = w.n_kv_heads * w.head_dim * 2
 
-    def appends(stream):
-        for step in pf.steps():
-            for r, c in step:
+    def timed(pairs):
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(torch.cuda.current_stream(dev))
+        graph = torch.cuda.CUDAGraph()
+
+        def appends(stream):
+            for r, c in pairs:
                 b0, b1 = pf.bounds[r][c], pf.bounds[r][c + 1]
                 base = pf.cu[r]
-                m.mocap_kv_append(k[base + b0:base + b1], v[base + b0:base + b1],
-                                  pf.k_cache[base:base + w.seq_lens[r]],
-                                  pf.v_cache[base:base + w.seq_lens[r]], b0, stream=stream)
+                m.mocap_kv_append(k[base + b0:base + b1], v[base + b0:base + b1], pf.k_cache,
+                                  pf.v_cache, base + b0, stream=stream)
 
-    with torch.cuda.stream(side):
-        appends(side)  # outside the capture: one-time set-up
-        with torch.cuda.graph(graph, stream=side):
-            appends(side)
-    torch.cuda.current_stream(dev).wait_stream(side)
-    graph.replay()
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(reps):
+        with torch.cuda.stream(side):
+            appends(side)  # outside the capture: one-time set-up
+            with torch.cuda.graph(graph, stream=side):
+                appends(side)
+        torch.cuda.current_stream(dev).wait_stream(side)
         graph.replay()
-    e1.record()
-    torch.cuda.synchronize(dev)
-    ms = e0.elapsed_time(e1) / reps
-    gbs = append_bytes / (ms * 1e-3) / 1e9
-    return {"kernel_ms_per_step": ms, "kernel_gb_per_s": gbs, "kernel_frac_of_hbm": gbs / hbm,
-            "kernel_note": "the step's appends replayed as one CUDA graph"}
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            graph.replay()
+        e1.record()
+        torch.cuda.synchronize(dev)
+        ms = e0.elapsed_time(e1) / reps
+        byts = sum(4 * (pf.bounds[r][c + 1] - pf.bounds[r][c]) * row_bytes for r, c in pairs)
+        return ms, byts / (ms * 1e-3) / 1e9
+
+    steps = pf.steps()
+    ms0, gbs0 = timed(steps[0])
+    ms_all, gbs_all = timed([rc for st in steps for rc in st])
+    return {"kernel_ms_per_step": ms0, "kernel_gb_per_s": gbs0, "kernel_frac_of_hbm": gbs0 / hbm,
+            "kernel_note": "the step's standalone appends (step 0's chunks) replayed as one "
+                           "CUDA graph",
+            "unfused_kernel_ms_per_step": ms_all, "unfused_kernel_gb_per_s": gbs_all,
+            "unfused_kernel_frac_of_hbm": gbs_all / hbm,
+            "unfused_note": "every chunk's append as its own launch, replayed as one graph"}
+
+
+def measure_fusion(args, pf, w, q, k, v, dev, stream, total_flops, reps=3):
+    """What carrying the next chunk's append in the attention launch costs:
+    the same prompt with fused appends and with one append launch per chunk
+    (ChunkedPrefill(fuse_appends=False)), each replayed from one CUDA graph,
+    interleaved, median of `reps` (no host gaps in either)."""
+    import torch
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    pu = ChunkedPrefill(w, dev, fuse_appends=False)
+    pu.workspace = pf.workspace  # same split plans and scratch
+    pu.k_cache, pu.v_cache, pu.out, pu.lse = pf.k_cache, pf.v_cache, pf.out, pf.lse
+    pu.run(q, k, v, stream)
+    g_f, g_u = pf.capture(q, k, v), pu.capture(q, k, v)
+    times = {"fused": [], "unfused": []}
+    for _ in range(reps):
+        for name, g in (("fused", g_f), ("unfused", g_u)):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            g.replay()
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            times[name].append(e0.elapsed_time(e1))
+    f, u = statistics.median(times["fused"]), statistics.median(times["unfused"])
+    del g_f, g_u, pu
+    return {"graph_fused_ms_per_step": f, "graph_unfused_ms_per_step": u,
+            "fusion_saves_ms_per_step": u - f,
+            "fusion_note": "whole prompt replayed from one CUDA graph: appends fused into the "
+                           "attention launches vs one append launch per chunk"}
 
 
 def measure_graph(args, pf, q, k, v, dev, stream, total_flops, tokens, world):
     """The same step replayed as one captured CUDA graph (every append,
     attention launch and combine of the prompt): no per-launch host work and
-    no gaps between launches.  Timed like the main region, after it."""
+    no gaps between launches.  Timed like the main region, after it.  Then
+    the per-chunk latency under replay: one graph per chunk step, replayed in
+    order with events between them (median over `steps` passes)."""
     import torch
     graph = pf.capture(q, k, v)
     for _ in range(args.warmup):
@@ -608,8 +667,30 @@ def measure_graph(args, pf, q, k, v, dev, stream, total_flops, tokens, world):
     barrier(world)
     ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world, dev)
     del graph
+    graphs = pf.capture_steps(q, k, v)
+    n = len(graphs)
+    per = [[] for _ in range(n)]
+    for rep in range(max(3, args.steps)):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+        ev[0].record(stream)
+        for i, g in enumerate(graphs):
+            g.replay()
+            ev[i + 1].record(stream)
+        torch.cuda.synchronize(dev)
+        for i in range(n):
+            per[i].append(ev[i].elapsed_time(ev[i + 1]))
+    pc = [statistics.median(x) for x in per]
+    del graphs
+    # step 0 also carries the prompt's one standalone append; steps 1.. are
+    # one attention launch (plus a split-KV combine) each
+    spread = pc[1:] if len(pc) > 2 else pc
     return {"ms_per_step": ms, "value": replica_throughput(total_flops, ms, world) / 1e12,
-            "unit": "TFLOP/s", "prefill_tokens_per_s": replica_throughput(tokens, ms, world)}
+            "unit": "TFLOP/s", "prefill_tokens_per_s": replica_throughput(tokens, ms, world),
+            "per_chunk_ms": {"min": min(pc), "max": max(pc), "max_over_min": max(pc) / min(pc),
+                             "cv": statistics.pstdev(pc) / statistics.mean(pc),
+                             "max_over_min_steps_1_on": max(spread) / min(spread),
+                             "note": "one graph per chunk step, replayed in order, events "
+                                     "between replays"}}
 
 
 def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):

@@ -17,6 +17,8 @@
  *   mocap_qkv_rope_append     QKV projection + RoPE + KV append (device GEMM)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
+ *   mocap_chunk_attn_append, mocap_chunk_attn_varlen_append
+ *                             the same with the next chunk's KV append in the launch
  *   mocap_last_row_attn       each request's last row only (prefill-only output)
  *   mocap_last_device_status  bounded-wait timeouts reported by the kernels
  *   mocap_selftest_bounded_wait  drives that timeout path on purpose (tests)
@@ -339,6 +341,69 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
                                      float scale, void *out, float *lse,
                                      void *workspace, size_t workspace_bytes,
                                      mocap_stream_t stream);
+
+/*
+ * One KV append that an attention launch carries out (see
+ * mocap_chunk_attn_append): rows [0, rows) of k_src / v_src (bf16
+ * [rows, n_kv_heads, head_dim], 16-byte aligned, device) are written to cache
+ * rows [dst_row, dst_row + rows), as mocap_kv_append would.
+ */
+typedef struct {
+  const void *k_src;
+  const void *v_src;
+  int64_t dst_row;
+  int64_t rows;
+} mocap_kv_append_item;
+
+#define MOCAP_FUSED_APPEND_MAX 64
+
+/*
+ * mocap_chunk_attn_append -- mocap_chunk_attn plus KV appends done in the same
+ * launch: the chunked prefill walks its chunks in order (Sec. 2.2), and
+ * chunk i + 1's K/V rows, which chunk i's attention never reads, are written
+ * to the cache by warps of chunk i's attention kernel that would otherwise
+ * idle.  The copy's HBM traffic overlaps tensor-bound work, and a prompt of
+ * M chunks needs M attention launches plus one append (chunk 0's) instead of
+ * M of each.
+ *
+ * Attention arguments and results as mocap_chunk_attn (split-KV workspace
+ * included).  Then:
+ *   appends        HOST array of n_appends descriptors (read during the call)
+ *   n_appends      0 .. MOCAP_FUSED_APPEND_MAX
+ *   cache_capacity rows of k_cache / v_cache (>= prefix + len)
+ * Each append must lie inside the cache and write only rows outside
+ * [0, prefix + len) (the rows this call reads) and outside the other
+ * appends' rows; sources must not overlap the cache rows written.  Else
+ * MOCAP_EINVAL, with nothing enqueued.  The appended rows are complete, like
+ * the outputs, when work queued after the call on `stream` starts.  With
+ * len == 0 the appends run as plain append launches.  After an expired
+ * bounded wait (see mocap_last_device_status) the call does nothing, appends
+ * included.
+ */
+mocap_status mocap_chunk_attn_append(const void *q, const void *k_cache, const void *v_cache,
+                                     int64_t prefix, int64_t len,
+                                     int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
+                                     float scale, void *out, float *lse,
+                                     void *workspace, size_t workspace_bytes,
+                                     const mocap_kv_append_item *appends, int32_t n_appends,
+                                     int64_t cache_capacity, mocap_stream_t stream);
+
+/*
+ * mocap_chunk_attn_varlen_append -- mocap_chunk_attn_varlen plus KV appends
+ * done in the same launch (e.g. chunk k + 1 of every request while chunk k
+ * of every request attends).  Appends as in mocap_chunk_attn_append, with
+ * destination rows in the packed caches (kv_rows_total rows): each must
+ * avoid every item's rows [kv_row, kv_row + prefix + len).
+ */
+mocap_status mocap_chunk_attn_varlen_append(const void *q, const void *k_cache,
+                                            const void *v_cache,
+                                            const mocap_varlen_item *items, int32_t n_items,
+                                            int64_t q_rows_total, int64_t kv_rows_total,
+                                            int32_t n_q_heads, int32_t n_kv_heads,
+                                            int32_t head_dim, float scale, void *out, float *lse,
+                                            void *workspace, size_t workspace_bytes,
+                                            const mocap_kv_append_item *appends,
+                                            int32_t n_appends, mocap_stream_t stream);
 
 /*
  * mocap_last_row_attn -- attention of each request's last prompt row only.

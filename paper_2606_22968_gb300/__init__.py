@@ -13,11 +13,12 @@ import ctypes
 from typing import List, Sequence
 
 from . import _lib
-from ._lib import VarlenItem
+from ._lib import AppendItem, VarlenItem
 
 MOCAP_OK, MOCAP_EINVAL, MOCAP_ECUDA, MOCAP_EUNSUPPORTED, MOCAP_ETIMEOUT = 0, 1, 2, 3, 4
 MOCAP_PART_UNIFORM, MOCAP_PART_LBCP = 0, 1
 MOCAP_VARLEN_MAX_ITEMS = 64
+MOCAP_FUSED_APPEND_MAX = 64
 
 
 class MocapError(RuntimeError):
@@ -165,6 +166,53 @@ def mocap_chunk_attn_varlen(q, k_cache, v_cache, items: Sequence[tuple], out, ls
                                                d, scale, _ptr(out), _ptr(lse), _ptr(workspace),
                                                ws_bytes, _stream(stream)),
            "mocap_chunk_attn_varlen")
+
+
+def _append_array(appends):
+    """(k_src, v_src, dst_row) triples -> the C descriptor array; the sources
+    are [rows, Hkv, d] tensors (contiguous, on the device)."""
+    arr = (AppendItem * max(1, len(appends)))()
+    for i, (k_src, v_src, dst_row) in enumerate(appends):
+        if k_src.shape != v_src.shape:
+            raise ValueError("K and V sources of an append must have the same shape")
+        arr[i] = AppendItem(_ptr(k_src), _ptr(v_src), dst_row, k_src.shape[0])
+    return arr
+
+
+def mocap_chunk_attn_append(q, k_cache, v_cache, prefix: int, out, lse, scale: float,
+                            appends: Sequence[tuple] = (), workspace=None, stream=None):
+    """mocap_chunk_attn that also writes ``appends`` -- (k_src, v_src, dst_row)
+    with sources [rows, Hkv, d] -- into cache rows [dst_row, dst_row + rows)
+    in the same launch (rows outside [0, prefix + len))."""
+    length, n_q, d = q.shape
+    n_kv = k_cache.shape[1]
+    if workspace is not None and not workspace.is_contiguous():
+        raise ValueError("workspace must be contiguous")
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(_lib.load().mocap_chunk_attn_append(_ptr(q), _ptr(k_cache), _ptr(v_cache), prefix,
+                                               length, n_q, n_kv, d, scale, _ptr(out), _ptr(lse),
+                                               _ptr(workspace), ws_bytes, _append_array(appends),
+                                               len(appends), k_cache.shape[0], _stream(stream)),
+           "mocap_chunk_attn_append")
+
+
+def mocap_chunk_attn_varlen_append(q, k_cache, v_cache, items: Sequence[tuple], out, lse,
+                                   scale: float, appends: Sequence[tuple] = (), workspace=None,
+                                   stream=None):
+    """mocap_chunk_attn_varlen that also writes ``appends`` (as in
+    mocap_chunk_attn_append, rows of the packed caches) in the same launch."""
+    q_rows, n_q, d = q.shape
+    n_kv = k_cache.shape[1]
+    arr = (VarlenItem * max(1, len(items)))()
+    for i, (q_row, kv_row, prefix, length) in enumerate(items):
+        arr[i] = VarlenItem(q_row, kv_row, prefix, length)
+    if workspace is not None and not workspace.is_contiguous():
+        raise ValueError("workspace must be contiguous")
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(_lib.load().mocap_chunk_attn_varlen_append(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), arr, len(items), q_rows, k_cache.shape[0], n_q,
+        n_kv, d, scale, _ptr(out), _ptr(lse), _ptr(workspace), ws_bytes, _append_array(appends),
+        len(appends), _stream(stream)), "mocap_chunk_attn_varlen_append")
 
 
 def mocap_last_row_attn_workspace_size(kv_len, n_q_heads: int, n_kv_heads: int,

@@ -18,6 +18,10 @@ class VarlenItem(ctypes.Structure):
     _fields_ = [("q_row", c_i64), ("kv_row", c_i64), ("prefix", c_i64), ("len", c_i64)]
 
 
+class AppendItem(ctypes.Structure):
+    _fields_ = [("k_src", c_vp), ("v_src", c_vp), ("dst_row", c_i64), ("rows", c_i64)]
+
+
 SIGNATURES = {
     "mocap_lbcp_partition": (c_i32, [c_i64, c_i32, c_i32, c_i32, ctypes.POINTER(c_i64)]),
     "mocap_lbcp_partition_dp": (c_i32, [c_i64, c_i32, c_i32, c_i32, c_i32, c_i64,
@@ -35,6 +39,13 @@ SIGNATURES = {
     "mocap_chunk_attn_varlen": (c_i32, [c_vp, c_vp, c_vp, ctypes.POINTER(VarlenItem), c_i32,
                                         c_i64, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp, c_vp,
                                         c_vp, c_sz, c_vp]),
+    "mocap_chunk_attn_append": (c_i32, [c_vp, c_vp, c_vp, c_i64, c_i64, c_i32, c_i32, c_i32, c_f32,
+                                        c_vp, c_vp, c_vp, c_sz, ctypes.POINTER(AppendItem), c_i32,
+                                        c_i64, c_vp]),
+    "mocap_chunk_attn_varlen_append": (c_i32, [c_vp, c_vp, c_vp, ctypes.POINTER(VarlenItem), c_i32,
+                                               c_i64, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp,
+                                               c_vp, c_vp, c_sz, ctypes.POINTER(AppendItem),
+                                               c_i32, c_vp]),
     "mocap_last_row_attn_workspace_size": (c_sz, [ctypes.POINTER(c_i64), c_i32, c_i32, c_i32,
                                                    c_i32]),
     "mocap_last_row_attn": (c_i32, [c_vp, c_vp, c_vp, ctypes.POINTER(c_i64), ctypes.POINTER(c_i64),

@@ -82,6 +82,19 @@ constexpr uint32_t kTmemCols = 512;
 constexpr float kMaxGrowthLog2 = 8.0f;  // rescale O only past a 2^8 max increase
 constexpr uint64_t kDrainLimitNs = 20000000ull;  // 20 ms for in-flight copies
 
+// One KV append carried by an attention launch (16-byte vectors): the K
+// source's n_vec vectors go to k_cache + dst_vec, the V source's to
+// v_cache + dst_vec.  `begin` is the segment's first index in the launch's
+// flattened list of 2 * sum(n_vec) vectors, which the CTAs share out evenly.
+struct AppendSeg {
+  const uint4 *k_src;
+  const uint4 *v_src;
+  int64_t dst_vec;
+  int64_t n_vec;
+  int64_t begin;
+};
+constexpr int kMaxAppends = MOCAP_FUSED_APPEND_MAX;
+
 struct ItemDesc {
   int64_t q_row;      // first packed Q/O row of the item
   int32_t prefix;     // keys before the chunk
@@ -113,7 +126,17 @@ struct AttnParams {
   float *o_part;
   float *lse_part;
   int32_t splits;
+  // KV appends done by this launch's otherwise idle warps 2-3 (cache rows no
+  // CTA of the launch reads): n_app segments, app_total vectors in all.
+  uint4 *k_cache_vec;
+  uint4 *v_cache_vec;
+  int64_t app_total;
+  int32_t n_app;
+  AppendSeg app[kMaxAppends];
 };
+
+// Kernel parameters are limited to 32764 bytes (__grid_constant__ block).
+static_assert(sizeof(AttnParams<MOCAP_VARLEN_MAX_ITEMS>) <= 32764, "kernel parameter space");
 
 // Shared memory of one CTA.  Single-CTA form: two Q tiles and a ring of four
 // stages, each holding one K or one V tile.  CTA-pair form (PAIR): each CTA
@@ -212,8 +235,57 @@ __device__ __forceinline__ float row_max(const float (&x)[128]) {
   return fmax3(a, b, fmaxf(m[6], m[7]));
 }
 
+__device__ __forceinline__ uint4 ld_stream_v4(const uint4 *ptr) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(ptr));
+  return v;
+}
+
+// This CTA's share of the launch's KV appends: vectors [lo, hi) of the
+// flattened list, lo = cta * total / ctas, copied by `nthreads` threads
+// (tid 0 .. nthreads-1) with four 16-byte loads in flight per thread.  The
+// destination rows are never read by this launch, so the copy needs no
+// ordering with the attention work; kernel completion publishes it to later
+// work on the stream.
+template <int MAXI>
+__device__ __forceinline__ void append_share(const AttnParams<MAXI> &p, int tid, int nthreads) {
+  if (p.n_app == 0) return;
+  const int64_t ctas = gridDim.x;
+  const int64_t cta = blockIdx.x;
+  const int64_t lo = cta * p.app_total / ctas;
+  const int64_t hi = (cta + 1) * p.app_total / ctas;
+  constexpr int kInFlight = 4;
+  for (int a = 0; a < p.n_app; ++a) {
+    const AppendSeg &sg = p.app[a];
+    const int64_t b = max(lo, sg.begin);
+    const int64_t e = min(hi, sg.begin + 2 * sg.n_vec);
+    for (int64_t i0 = b + tid; i0 < e; i0 += static_cast<int64_t>(kInFlight) * nthreads) {
+      uint4 v[kInFlight];
+#pragma unroll
+      for (int u = 0; u < kInFlight; ++u) {
+        const int64_t off = i0 + static_cast<int64_t>(u) * nthreads - sg.begin;
+        if (off < e - sg.begin)
+          v[u] = ld_stream_v4(off < sg.n_vec ? sg.k_src + off : sg.v_src + (off - sg.n_vec));
+      }
+#pragma unroll
+      for (int u = 0; u < kInFlight; ++u) {
+        const int64_t off = i0 + static_cast<int64_t>(u) * nthreads - sg.begin;
+        if (off < e - sg.begin) {
+          if (off < sg.n_vec) {
+            p.k_cache_vec[sg.dst_vec + off] = v[u];
+          } else {
+            p.v_cache_vec[sg.dst_vec + (off - sg.n_vec)] = v[u];
+          }
+        }
+      }
+    }
+  }
+}
+
 // Warpgroup 0: warp 0 is the TMA producer, warp 1 the MMA issuer (one lane
-// each); warps 2-3 only take part in the barriers.
+// each); warps 2-3 copy this CTA's share of the launch's KV appends, if any.
 template <int D, int MAXI>
 __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_t base,
                                               uint32_t bars, uint32_t tmem, uint32_t warp,
@@ -342,6 +414,8 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
       mbar_wait(bar(L::kBarDrain), 0, p.status, kDrainLimitNs, false);
     }
     __syncwarp();
+  } else {
+    append_share(p, static_cast<int>(threadIdx.x) - 64, 64);  // warps 2-3
   }
 }
 
@@ -504,6 +578,8 @@ __device__ __forceinline__ void control_roles_pair(const AttnParams<MAXI> &p, ui
       mbar_wait(bar(L::kBarDrain), 0, p.status, kDrainLimitNs, false);
     }
     __syncwarp();
+  } else if (warp >= 2) {
+    append_share(p, static_cast<int>(threadIdx.x) - 64, 64);  // warps 2-3
   }
 }
 
@@ -725,7 +801,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (n_kv <= 0) {
     // No key tile in this split (the host never schedules one): an empty
-    // partial, weight 0 in the combine.
+    // partial, weight 0 in the combine, and this CTA's share of the appends.
+    if (warp == 2 || warp == 3) append_share(p, static_cast<int>(threadIdx.x) - 64, 64);
     if (p.splits > 1 && warp >= 4) {
       const int sl = static_cast<int>(warp - 4) / 4;
       const int row = static_cast<int>((warp & 3u) * 32 + lane);
@@ -905,6 +982,13 @@ struct HostItem {
   int64_t q_row, kv_row, prefix, len;
 };
 
+// KV appends a launch carries (validated by the entry points): K/V sources
+// of `rows` rows each, written to cache rows [dst_row, dst_row + rows).
+struct HostAppend {
+  const void *k_src, *v_src;
+  int64_t dst_row, rows;
+};
+
 // Split-KV scratch (single item): o_part [splits, len, Hq, D] fp32 followed by
 // lse_part [splits, Hq, len] fp32, the latter 256-byte aligned.
 struct SplitPlan {
@@ -998,7 +1082,8 @@ template <int D, int MAXI>
 mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
                     const std::vector<HostItem> &items, int64_t lse_stride, const Shape &sh,
                     float scale, void *out, float *lse, cudaStream_t stream,
-                    const SplitPlan &sp = SplitPlan(), void *workspace = nullptr) {
+                    const SplitPlan &sp = SplitPlan(), void *workspace = nullptr,
+                    const std::vector<HostAppend> &apps = {}) {
   using L = Layout<D>;
   static AttnParams<MAXI> prm;  // large: build in static storage, guarded below
   static std::mutex mu;
@@ -1049,6 +1134,20 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     if (n != 1 || workspace == nullptr || sp.splits > kMaxSplits) return MOCAP_EINVAL;
     prm.o_part = static_cast<float *>(workspace);
     prm.lse_part = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + sp.lse_off);
+  }
+  if (apps.size() > static_cast<size_t>(kMaxAppends)) return MOCAP_EINVAL;
+  prm.k_cache_vec = static_cast<uint4 *>(const_cast<void *>(k_cache));
+  prm.v_cache_vec = static_cast<uint4 *>(const_cast<void *>(v_cache));
+  const int64_t row_vec = static_cast<int64_t>(sh.n_kv_heads) * D / 8;  // 16-byte vectors per row
+  for (const HostAppend &a : apps) {
+    if (a.rows <= 0) continue;
+    AppendSeg &g = prm.app[prm.n_app++];
+    g.k_src = static_cast<const uint4 *>(a.k_src);
+    g.v_src = static_cast<const uint4 *>(a.v_src);
+    g.dst_vec = a.dst_row * row_vec;
+    g.n_vec = a.rows * row_vec;
+    g.begin = prm.app_total;
+    prm.app_total += 2 * g.n_vec;
   }
 
   int dev = 0;
@@ -1115,12 +1214,38 @@ template <int MAXI>
 mocap_status dispatch(const void *q, const void *k_cache, const void *v_cache,
                       const std::vector<HostItem> &items, int64_t lse_stride, const Shape &sh,
                       float scale, void *out, float *lse, cudaStream_t stream,
-                      const SplitPlan &sp = SplitPlan(), void *workspace = nullptr) {
+                      const SplitPlan &sp = SplitPlan(), void *workspace = nullptr,
+                      const std::vector<HostAppend> &apps = {}) {
   if (sh.head_dim == 128)
     return launch<128, MAXI>(q, k_cache, v_cache, items, lse_stride, sh, scale, out, lse, stream,
-                             sp, workspace);
+                             sp, workspace, apps);
   return launch<64, MAXI>(q, k_cache, v_cache, items, lse_stride, sh, scale, out, lse, stream, sp,
-                          workspace);
+                          workspace, apps);
+}
+
+// Validates the KV appends an attention launch is to carry and converts
+// them: each must fit the cache (kv_rows_total rows), have 16-byte aligned
+// sources, and write only rows that no item of the launch reads (item r
+// reads cache rows [kv_row, kv_row + prefix + len)).  Appends must not write
+// overlapping rows either.
+mocap_status check_appends(const mocap_kv_append_item *appends, int32_t n_appends,
+                           int64_t kv_rows_total, const std::vector<HostItem> &items,
+                           std::vector<HostAppend> *out) {
+  if (n_appends < 0 || n_appends > kMaxAppends) return MOCAP_EINVAL;
+  if (n_appends > 0 && appends == nullptr) return MOCAP_EINVAL;
+  for (int i = 0; i < n_appends; ++i) {
+    const mocap_kv_append_item &a = appends[i];
+    if (a.rows < 0 || a.dst_row < 0 || a.dst_row > kv_rows_total - a.rows) return MOCAP_EINVAL;
+    if (a.rows == 0) continue;
+    if (!a.k_src || !a.v_src || !aligned16(a.k_src) || !aligned16(a.v_src)) return MOCAP_EINVAL;
+    const int64_t lo = a.dst_row, hi = a.dst_row + a.rows;
+    for (const HostItem &it : items)
+      if (lo < it.kv_row + it.prefix + it.len && it.kv_row < hi) return MOCAP_EINVAL;
+    for (const HostAppend &b : *out)
+      if (lo < b.dst_row + b.rows && b.dst_row < hi) return MOCAP_EINVAL;
+    out->push_back({a.k_src, a.v_src, a.dst_row, a.rows});
+  }
+  return MOCAP_OK;
 }
 
 bool pointers_ok(const void *q, const void *k, const void *v, const void *out, const float *lse) {
@@ -1166,34 +1291,52 @@ extern "C" size_t mocap_chunk_attn_workspace_size(int64_t prefix, int64_t len, i
   return plan_for(prefix, len, n_q_heads, n_kv_heads, head_dim).bytes;
 }
 
-extern "C" mocap_status mocap_chunk_attn(const void *q, const void *k_cache, const void *v_cache,
-                                         int64_t prefix, int64_t len, int32_t n_q_heads,
-                                         int32_t n_kv_heads, int32_t head_dim, float scale,
-                                         void *out, float *lse, void *workspace,
-                                         size_t workspace_bytes, mocap_stream_t stream) {
+namespace {
+// mocap_chunk_attn, optionally carrying KV appends (checked by the caller).
+mocap_status chunk_attn_impl(const void *q, const void *k_cache, const void *v_cache,
+                             int64_t prefix, int64_t len, int32_t n_q_heads, int32_t n_kv_heads,
+                             int32_t head_dim, float scale, void *out, float *lse,
+                             void *workspace, size_t workspace_bytes, mocap_stream_t stream,
+                             bool with_appends = false,
+                             const mocap_kv_append_item *appends = nullptr,
+                             int32_t n_appends = 0, int64_t cache_rows = 0) {
   const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
   const mocap_status st = mocap::check_shape(sh, scale);
   if (st != MOCAP_OK) return st;
   if (prefix < 0 || len < 0 || prefix > mocap::kMaxRows - len) return MOCAP_EINVAL;
   if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
   if (workspace != nullptr && !mocap::aligned16(workspace)) return MOCAP_EINVAL;
-  if (len == 0) return MOCAP_OK;
+  std::vector<HostItem> items{{0, 0, prefix, len}};
+  std::vector<mocap::HostAppend> apps;
+  if (with_appends) {
+    if (cache_rows < prefix + len) return MOCAP_EINVAL;
+    const mocap_status sa = mocap::check_appends(appends, n_appends, cache_rows, items, &apps);
+    if (sa != MOCAP_OK) return sa;
+  }
+  if (len == 0) {
+    // no attention work: the appends run as plain append launches
+    for (const mocap::HostAppend &a : apps) {
+      const mocap_status sa = mocap_kv_append(a.k_src, a.v_src, const_cast<void *>(k_cache),
+                                              const_cast<void *>(v_cache), cache_rows, a.dst_row,
+                                              a.rows, n_kv_heads, head_dim, stream);
+      if (sa != MOCAP_OK) return sa;
+    }
+    return MOCAP_OK;
+  }
   // Split the key range only when the caller's scratch holds the partials.
   mocap::SplitPlan sp = plan_for(prefix, len, n_q_heads, n_kv_heads, head_dim);
   if (sp.splits > 1 && (workspace == nullptr || workspace_bytes < sp.bytes)) sp = mocap::SplitPlan();
-  std::vector<HostItem> items{{0, 0, prefix, len}};
   return mocap::dispatch<1>(q, k_cache, v_cache, items, len, sh, scale, out, lse,
-                            reinterpret_cast<cudaStream_t>(stream), sp, workspace);
+                            reinterpret_cast<cudaStream_t>(stream), sp, workspace, apps);
 }
 
-extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache,
-                                                const void *v_cache,
-                                                const mocap_varlen_item *items, int32_t n_items,
-                                                int64_t q_rows_total, int64_t kv_rows_total,
-                                                int32_t n_q_heads, int32_t n_kv_heads,
-                                                int32_t head_dim, float scale, void *out,
-                                                float *lse, void *workspace,
-                                                size_t workspace_bytes, mocap_stream_t stream) {
+// mocap_chunk_attn_varlen, optionally carrying KV appends.
+mocap_status varlen_impl(const void *q, const void *k_cache, const void *v_cache,
+                         const mocap_varlen_item *items, int32_t n_items, int64_t q_rows_total,
+                         int64_t kv_rows_total, int32_t n_q_heads, int32_t n_kv_heads,
+                         int32_t head_dim, float scale, void *out, float *lse, void *workspace,
+                         size_t workspace_bytes, mocap_stream_t stream,
+                         const mocap_kv_append_item *appends = nullptr, int32_t n_appends = 0) {
   const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
   const mocap_status st = mocap::check_shape(sh, scale);
   if (st != MOCAP_OK) return st;
@@ -1211,7 +1354,18 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
     if (x.kv_row > kv_rows_total - (x.prefix + x.len)) return MOCAP_EINVAL;
     if (x.len > 0) list.push_back({x.q_row, x.kv_row, x.prefix, x.len});
   }
-  if (list.empty()) return MOCAP_OK;
+  std::vector<mocap::HostAppend> apps;
+  const mocap_status sa = mocap::check_appends(appends, n_appends, kv_rows_total, list, &apps);
+  if (sa != MOCAP_OK) return sa;
+  if (list.empty()) {
+    for (const mocap::HostAppend &a : apps) {
+      const mocap_status sk = mocap_kv_append(a.k_src, a.v_src, const_cast<void *>(k_cache),
+                                              const_cast<void *>(v_cache), kv_rows_total,
+                                              a.dst_row, a.rows, n_kv_heads, head_dim, stream);
+      if (sk != MOCAP_OK) return sk;
+    }
+    return MOCAP_OK;
+  }
   if (list.size() == 1) {
     // One item: the single-chunk plan, key-range split included when the
     // caller's workspace holds its partials.
@@ -1220,7 +1374,7 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
     if (sp.splits > 1 && (workspace == nullptr || workspace_bytes < sp.bytes))
       sp = mocap::SplitPlan();
     return mocap::dispatch<1>(q, k_cache, v_cache, list, q_rows_total, sh, scale, out, lse,
-                              reinterpret_cast<cudaStream_t>(stream), sp, workspace);
+                              reinterpret_cast<cudaStream_t>(stream), sp, workspace, apps);
   }
   // Heaviest items first (their last row blocks see the most keys).
   std::stable_sort(list.begin(), list.end(), [](const HostItem &a, const HostItem &b) {
@@ -1228,7 +1382,51 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
   });
   return mocap::dispatch<MOCAP_VARLEN_MAX_ITEMS>(q, k_cache, v_cache, list, q_rows_total, sh,
                                                  scale, out, lse,
-                                                 reinterpret_cast<cudaStream_t>(stream));
+                                                 reinterpret_cast<cudaStream_t>(stream),
+                                                 mocap::SplitPlan(), nullptr, apps);
+}
+}  // namespace
+
+extern "C" mocap_status mocap_chunk_attn(const void *q, const void *k_cache, const void *v_cache,
+                                         int64_t prefix, int64_t len, int32_t n_q_heads,
+                                         int32_t n_kv_heads, int32_t head_dim, float scale,
+                                         void *out, float *lse, void *workspace,
+                                         size_t workspace_bytes, mocap_stream_t stream) {
+  return chunk_attn_impl(q, k_cache, v_cache, prefix, len, n_q_heads, n_kv_heads, head_dim, scale,
+                         out, lse, workspace, workspace_bytes, stream);
+}
+
+extern "C" mocap_status mocap_chunk_attn_append(
+    const void *q, const void *k_cache, const void *v_cache, int64_t prefix, int64_t len,
+    int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim, float scale, void *out, float *lse,
+    void *workspace, size_t workspace_bytes, const mocap_kv_append_item *appends,
+    int32_t n_appends, int64_t cache_capacity, mocap_stream_t stream) {
+  return chunk_attn_impl(q, k_cache, v_cache, prefix, len, n_q_heads, n_kv_heads, head_dim, scale,
+                         out, lse, workspace, workspace_bytes, stream, true, appends, n_appends,
+                         cache_capacity);
+}
+
+extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache,
+                                                const void *v_cache,
+                                                const mocap_varlen_item *items, int32_t n_items,
+                                                int64_t q_rows_total, int64_t kv_rows_total,
+                                                int32_t n_q_heads, int32_t n_kv_heads,
+                                                int32_t head_dim, float scale, void *out,
+                                                float *lse, void *workspace,
+                                                size_t workspace_bytes, mocap_stream_t stream) {
+  return varlen_impl(q, k_cache, v_cache, items, n_items, q_rows_total, kv_rows_total, n_q_heads,
+                     n_kv_heads, head_dim, scale, out, lse, workspace, workspace_bytes, stream);
+}
+
+extern "C" mocap_status mocap_chunk_attn_varlen_append(
+    const void *q, const void *k_cache, const void *v_cache, const mocap_varlen_item *items,
+    int32_t n_items, int64_t q_rows_total, int64_t kv_rows_total, int32_t n_q_heads,
+    int32_t n_kv_heads, int32_t head_dim, float scale, void *out, float *lse, void *workspace,
+    size_t workspace_bytes, const mocap_kv_append_item *appends, int32_t n_appends,
+    mocap_stream_t stream) {
+  return varlen_impl(q, k_cache, v_cache, items, n_items, q_rows_total, kv_rows_total, n_q_heads,
+                     n_kv_heads, head_dim, scale, out, lse, workspace, workspace_bytes, stream,
+                     appends, n_appends);
 }
 
 // ---------------------------------------------------------------------------

@@ -15,7 +15,8 @@ from typing import List, Optional
 import torch
 
 from . import (MOCAP_COST_CAUSAL, MOCAP_PART_LBCP, MOCAP_PART_UNIFORM, mocap_chunk_attn,
-               mocap_chunk_attn_varlen, mocap_chunk_attn_workspace_size, mocap_kv_append,
+               mocap_chunk_attn_append, mocap_chunk_attn_varlen, mocap_chunk_attn_varlen_append,
+               mocap_chunk_attn_workspace_size, mocap_kv_append,
                mocap_lbcp_gemm_weight, mocap_lbcp_partition, mocap_lbcp_partition_dp,
                mocap_qkv_rope_append)
 from .workloads import GRANULARITY, Workload, request_offsets
@@ -50,10 +51,14 @@ class ChunkedPrefill:
     """
 
     def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True,
-                 bounds: Optional[List[List[int]]] = None):
+                 bounds: Optional[List[List[int]]] = None, fuse_appends: bool = True):
         """``bounds`` (one boundary list per request) replaces the workload's
-        partition rule, e.g. with the Algorithm 1 stage-1 DP's split."""
+        partition rule, e.g. with the Algorithm 1 stage-1 DP's split.
+        ``fuse_appends`` lets each attention launch append the next step's
+        chunks (mocap_chunk_attn_append); False launches one append per chunk
+        before its attention (mocap_kv_append)."""
         self.w = w
+        self.fuse_appends = fuse_appends
         self.device = torch.device(device)
         self.mode = w.mode if mode is None else mode
         self.fixed_bounds = None if bounds is None else [list(b) for b in bounds]
@@ -112,52 +117,74 @@ class ChunkedPrefill:
         return self.lse.view(self.w.n_q_heads, self.w.total_tokens)
 
     # -- execution ----------------------------------------------------------------
-    def run_step(self, q, k, v, step, stream=None, events=None):
-        """Append + attention for one step (one chunk index).  ``events`` is
-        an optional triple of CUDA events recorded before the appends, between
-        appends and attention, and after the attention.  With MOCAP_NVTX=1 in
-        the environment each step is an NVTX range ("mocap chunk <index>")
-        for timeline profilers."""
+    def run_step(self, q, k, v, i, stream=None, events=None):
+        """Step ``i`` of ``steps()`` (one chunk index of every request that has
+        it).  With fused appends (the default) step 0 first appends its own
+        chunks, and every step's attention launch also appends the next step's
+        chunks (rows it never reads); otherwise each step appends its own
+        chunks, then attends.  ``events`` is an optional triple of CUDA events
+        recorded before the step's own appends (step 0 only when fused),
+        before the attention launch, and after it.  With MOCAP_NVTX=1 in the
+        environment each step is an NVTX range ("mocap chunk <index>") for
+        timeline profilers."""
         if os.environ.get("MOCAP_NVTX", "0") != "0":
-            with torch.cuda.nvtx.range(f"mocap chunk {step[0][1]}"):
-                return self._run_step(q, k, v, step, stream, events)
-        return self._run_step(q, k, v, step, stream, events)
+            with torch.cuda.nvtx.range(f"mocap chunk {i}"):
+                return self._run_step(q, k, v, i, stream, events)
+        return self._run_step(q, k, v, i, stream, events)
 
-    def _run_step(self, q, k, v, step, stream=None, events=None):
+    def _append_rows(self, k, v, r, c):
+        """(K rows, V rows, destination cache row) of chunk c of request r."""
+        b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
+        base = self.cu[r]
+        return k[base + b0:base + b1], v[base + b0:base + b1], base + b0
+
+    def _run_step(self, q, k, v, i, stream=None, events=None):
         w = self.w
+        steps = self.steps()
+        step = steps[i]
         if events is not None:
             events[0].record(stream)
-        for r, c in step:
-            b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
-            base = self.cu[r]
-            mocap_kv_append(k[base + b0:base + b1], v[base + b0:base + b1],
-                            self.k_cache[base:base + w.seq_lens[r]],
-                            self.v_cache[base:base + w.seq_lens[r]], b0, stream=stream)
+        if not self.fuse_appends or i == 0:
+            for r, c in step:
+                kr, vr, dst = self._append_rows(k, v, r, c)
+                mocap_kv_append(kr, vr, self.k_cache, self.v_cache, dst, stream=stream)
+        nxt = []
+        if self.fuse_appends and i + 1 < len(steps):
+            nxt = [self._append_rows(k, v, r, c) for r, c in steps[i + 1]]
         if events is not None:
             events[1].record(stream)
         if self.single:
             (_, c), = step
             b0, b1 = self.bounds[0][c], self.bounds[0][c + 1]
-            mocap_chunk_attn(q[b0:b1], self.k_cache, self.v_cache, b0, self.out[b0:b1],
-                             self.chunk_lse(c), w.scale, workspace=self.workspace,
-                             stream=stream)
+            if self.fuse_appends:
+                mocap_chunk_attn_append(q[b0:b1], self.k_cache, self.v_cache, b0,
+                                        self.out[b0:b1], self.chunk_lse(c), w.scale, nxt,
+                                        workspace=self.workspace, stream=stream)
+            else:
+                mocap_chunk_attn(q[b0:b1], self.k_cache, self.v_cache, b0, self.out[b0:b1],
+                                 self.chunk_lse(c), w.scale, workspace=self.workspace,
+                                 stream=stream)
         else:
             items = []
             for r, c in step:
                 b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
                 items.append((self.cu[r] + b0, self.cu[r], b0, b1 - b0))
-            mocap_chunk_attn_varlen(q, self.k_cache, self.v_cache, items, self.out,
-                                    self.lse_packed(), w.scale, workspace=self.workspace,
-                                    stream=stream)
+            if self.fuse_appends:
+                mocap_chunk_attn_varlen_append(q, self.k_cache, self.v_cache, items, self.out,
+                                               self.lse_packed(), w.scale, nxt,
+                                               workspace=self.workspace, stream=stream)
+            else:
+                mocap_chunk_attn_varlen(q, self.k_cache, self.v_cache, items, self.out,
+                                        self.lse_packed(), w.scale, workspace=self.workspace,
+                                        stream=stream)
         if events is not None:
             events[2].record(stream)
 
     def run(self, q, k, v, stream=None, chunk_events=None):
         """The whole prompt: every step in order.  ``chunk_events`` optionally
         holds one event triple per step (see run_step)."""
-        for i, step in enumerate(self.steps()):
-            self.run_step(q, k, v, step, stream,
-                          None if chunk_events is None else chunk_events[i])
+        for i in range(len(self.steps())):
+            self.run_step(q, k, v, i, stream, None if chunk_events is None else chunk_events[i])
 
     def run_stage(self, x, w_qkv, q_buf, stream=None, rope_theta: float = 500000.0,
                   chunk_events=None):
@@ -193,7 +220,8 @@ class ChunkedPrefill:
 
         Every chunk's Q/K/V rows are copied into the device buffers ``q, k, v``
         on a copy stream, in chunk order; the compute stream starts chunk i as
-        soon as its rows have landed, and a third stream copies chunk i's O
+        soon as its rows (and, with fused appends, chunk i + 1's, which its
+        launch appends) have landed, and a third stream copies chunk i's O
         and LSE back to ``host_out`` / ``host_lse`` (shaped like ``self.out``
         and ``self.lse``) as soon as its attention is done.  With several
         requests a chunk's LSE columns are strided in the ``[Hq, T]`` array, so
@@ -220,7 +248,9 @@ class ChunkedPrefill:
         d2h.wait_stream(compute)
         for i, step in enumerate(steps):
             compute.wait_event(landed[i])
-            self.run_step(q, k, v, step, compute)
+            if self.fuse_appends and i + 1 < len(steps):
+                compute.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
+            self.run_step(q, k, v, i, compute)
             done = torch.cuda.Event()
             done.record(compute)
             d2h.wait_event(done)
@@ -294,7 +324,9 @@ class ChunkedPrefill:
                 compute.wait_event(outputs_gone)
             for i, step in enumerate(steps):
                 compute.wait_event(landed[p][i])
-                self.run_step(q, k, v, step, compute)
+                if self.fuse_appends and i + 1 < len(steps):
+                    compute.wait_event(landed[p][i + 1])  # appended by this launch
+                self.run_step(q, k, v, i, compute)
                 done = torch.cuda.Event()
                 done.record(compute)
                 d2h.wait_event(done)
@@ -319,6 +351,23 @@ class ChunkedPrefill:
         compute.wait_stream(h2d)
 
     # -- CUDA graph ------------------------------------------------------------------
+    def capture_steps(self, q, k, v, stream=None):
+        """One CUDA graph per step (its launches as ``run_step`` enqueues them);
+        replaying them in order is the whole prompt, and events recorded
+        between the replays time each chunk step without host gaps inside
+        it.  Same preconditions as ``capture``."""
+        graphs = []
+        side = torch.cuda.Stream(self.device) if stream is None else stream
+        side.wait_stream(torch.cuda.current_stream(self.device))
+        with torch.cuda.stream(side):
+            for i in range(len(self.steps())):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=side):
+                    self.run_step(q, k, v, i, side)
+                graphs.append(g)
+        torch.cuda.current_stream(self.device).wait_stream(side)
+        return graphs
+
     def capture(self, q, k, v, stream=None):
         """Record the whole prompt's launch sequence (every append, attention
         launch and split-KV combine) into one CUDA graph.  Replaying it runs

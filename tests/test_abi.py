@@ -281,3 +281,33 @@ def test_gemm_weight_entry_point(lib):
                 (1e-30, 1.0, 128)):
         assert lib.mocap_lbcp_gemm_weight(*bad, ctypes.byref(w)) == 1, bad
     assert lib.mocap_lbcp_gemm_weight(1.0, 1.0, 128, None) == 1
+
+
+def test_fused_append_argument_checks(lib):
+    """mocap_chunk_attn_append / _varlen_append refuse appends that overlap
+    the rows the launch reads, each other, or the cache end (nothing is
+    launched, so no GPU is needed)."""
+    from paper_2606_22968_gb300._lib import AppendItem, VarlenItem
+    f = lib.mocap_chunk_attn_append
+
+    def call(apps, prefix=100, length=50, cap=1000, n=None):
+        arr = (AppendItem * max(1, len(apps)))(*[AppendItem(*a) for a in apps])
+        return f(FAKE, FAKE, FAKE, prefix, length, 8, 2, 128, 0.1, FAKE, FAKE, None, 0,
+                 arr if apps or n else None, len(apps) if n is None else n, cap, None)
+
+    assert call([(FAKE, FAKE, 149, 10)]) == 1            # overlaps the chunk's own rows
+    assert call([(FAKE, FAKE, 0, 10)]) == 1              # overlaps the prefix
+    assert call([(FAKE, FAKE, 995, 10)]) == 1            # past the cache
+    assert call([(FAKE, FAKE, -1, 10)]) == 1
+    assert call([(FAKE, FAKE, 200, -1)]) == 1
+    assert call([(FAKE + 8, FAKE, 200, 10)]) == 1        # misaligned source
+    assert call([(None, FAKE, 200, 10)]) == 1
+    assert call([(FAKE, FAKE, 200, 10), (FAKE, FAKE, 205, 10)]) == 1  # appends overlap
+    assert call([(FAKE, FAKE, 200, 10)] * 65) == 1       # too many
+    assert call([], n=3) == 1                            # count without an array
+    assert call([(FAKE, FAKE, 200, 10)], cap=120) == 1   # cache shorter than prefix + len
+    g = lib.mocap_chunk_attn_varlen_append
+    items = (VarlenItem * 2)(VarlenItem(0, 0, 0, 10), VarlenItem(10, 500, 20, 10))
+    arr = (AppendItem * 1)(AppendItem(FAKE, FAKE, 515, 4))  # inside item 1's rows [500, 530)
+    assert g(FAKE, FAKE, FAKE, items, 2, 100, 1000, 8, 2, 128, 0.1, FAKE, FAKE, None, 0, arr, 1,
+             None) == 1
