@@ -41,6 +41,9 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", type=int, default=4)
+    ap.add_argument("--append-mode", choices=["serial", "fused", "overlap"], default="overlap",
+                    help="how chunk K/V reach the cache in the timed steps "
+                         "(ChunkedPrefill append_mode)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
@@ -391,7 +394,7 @@ def ours_arm(args, rank, world, local):
     torch.cuda.set_device(dev)
     w = workloads.get(args.workload)
     q, k, v = workloads.make_qkv(w, dev)
-    pf = ChunkedPrefill(w, dev)
+    pf = ChunkedPrefill(w, dev, append_mode=args.append_mode)
     steps_plan = pf.steps()
     n_chunks = len(steps_plan)
     stream = torch.cuda.current_stream(dev)
@@ -413,9 +416,12 @@ def ours_arm(args, rank, world, local):
         return sum(pf.bounds[r][c + 1] - pf.bounds[r][c] for r, c in step)
 
     append_bytes = 2 * 2 * w.total_tokens * row_bytes  # K, V x (read + write)
-    # with fused appends only step 0's chunks are appended by a launch of
-    # their own; the attention launches' idle warps append the rest
+    # only step 0's chunks are appended on the compute stream before their
+    # attention; the rest go to the cache beside the attention launches
+    # (second stream, or inside the launch; ChunkedPrefill.append_mode)
     standalone_bytes = 2 * 2 * rows_of(steps_plan[0]) * row_bytes
+    if pf.append_mode == "serial":
+        standalone_bytes = append_bytes
 
     def one_step(ev=None):
         pf.partition()
@@ -499,9 +505,9 @@ def ours_arm(args, rank, world, local):
                    "fused_bytes_per_step": append_bytes - standalone_bytes,
                    "gb_per_s": app_gbs, "frac_of_hbm": app_gbs / hbm,
                    "ms_per_step": statistics.mean(app_step_ms),
-                   "note": "gb_per_s: the step's standalone appends (step 0's chunks) between "
-                           "events in the timed steps; the other chunks' K/V are appended by "
-                           "the attention launch of the step before (mocap_chunk_attn_append)"},
+                   "note": "gb_per_s: the appends on the compute stream (step 0's chunks "
+                           "unless append_mode is serial) between events in the timed steps; "
+                           f"append_mode {pf.append_mode}"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak,
                      "peak_source": f"bf16_tflops_sustained ({peak_src})",
@@ -519,10 +525,13 @@ def ours_arm(args, rank, world, local):
                       "(profiles/chunk_attn_dram_traffic.txt), DRAM/minimum ratio "
                       "interpolated in keys per chunk")},
         "clocks": clk,
-        # our kernels per timed region: step 0's appends (one per request),
-        # one attention launch per step (carrying the next step's appends),
-        # one split-KV combine per split chunk
-        "gpu_launches": args.steps * (len(steps_plan[0]) + len(steps_plan) + n_combines),
+        # our kernels per timed region: one append per (request, chunk) (in
+        # fused mode only step 0's; the others ride in the attention
+        # launches), one attention launch per step, one split-KV combine per
+        # split chunk
+        "gpu_launches": args.steps * (
+            (len(steps_plan[0]) if pf.append_mode == "fused" else
+             sum(len(st) for st in steps_plan)) + len(steps_plan) + n_combines),
     }
 
     if not args.no_e2e:
@@ -614,41 +623,49 @@ def measure_append_graph(m, w, pf, k, v, dev, hbm, reps=5):
 
 
 def measure_fusion(args, pf, w, q, k, v, dev, stream, total_flops, reps=3):
-    """What carrying the next chunk's append in the attention launch costs:
-    the same prompt with fused appends and with one append launch per chunk
-    (ChunkedPrefill(fuse_appends=False)), each replayed from one CUDA graph,
-    interleaved, median of `reps` (no host gaps in either)."""
+    """The three ways the prompt's chunk K/V reach the cache (ChunkedPrefill
+    append_mode): one append launch per chunk before its attention
+    ("serial"), the next chunk's append inside the attention launch
+    ("fused"), or appends on a second stream beside the attention launches
+    ("overlap").  Each prompt is replayed from one CUDA graph, interleaved,
+    median of `reps` (no host gaps in any)."""
     import torch
-    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
-    pu = ChunkedPrefill(w, dev, fuse_appends=False)
-    pu.workspace = pf.workspace  # same split plans and scratch
-    pu.k_cache, pu.v_cache, pu.out, pu.lse = pf.k_cache, pf.v_cache, pf.out, pf.lse
-    pu.run(q, k, v, stream)
-    g_f, g_u = pf.capture(q, k, v), pu.capture(q, k, v)
-    times = {"fused": [], "unfused": []}
+    from paper_2606_22968_gb300.pipeline import APPEND_MODES, ChunkedPrefill
+    times, graphs, keep = {}, {}, []
+    for mode in APPEND_MODES:
+        px = ChunkedPrefill(w, dev, append_mode=mode)
+        px.workspace = pf.workspace  # same split plans and scratch
+        px.k_cache, px.v_cache, px.out, px.lse = pf.k_cache, pf.v_cache, pf.out, pf.lse
+        px.run(q, k, v, stream)
+        graphs[mode] = px.capture(q, k, v)
+        times[mode] = []
+        keep.append(px)
     for _ in range(reps):
-        for name, g in (("fused", g_f), ("unfused", g_u)):
+        for mode, g in graphs.items():
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             g.replay()
             e0.record(stream)
             g.replay()
             e1.record(stream)
             torch.cuda.synchronize(dev)
-            times[name].append(e0.elapsed_time(e1))
-    f, u = statistics.median(times["fused"]), statistics.median(times["unfused"])
-    del g_f, g_u, pu
-    return {"graph_fused_ms_per_step": f, "graph_unfused_ms_per_step": u,
-            "fusion_saves_ms_per_step": u - f,
-            "fusion_note": "whole prompt replayed from one CUDA graph: appends fused into the "
-                           "attention launches vs one append launch per chunk"}
+            times[mode].append(e0.elapsed_time(e1))
+    del graphs, keep
+    med = {mode: statistics.median(t) for mode, t in times.items()}
+    return {"graph_ms_per_step_by_append_mode": med,
+            "append_mode_used": pf.append_mode,
+            "append_mode_note": "whole prompt replayed from one CUDA graph: serial = one append "
+                                "launch per chunk before its attention; fused = the next chunk's "
+                                "append inside the attention launch; overlap = appends on a "
+                                "second stream beside the attention launches"}
 
 
 def measure_graph(args, pf, q, k, v, dev, stream, total_flops, tokens, world):
     """The same step replayed as one captured CUDA graph (every append,
     attention launch and combine of the prompt): no per-launch host work and
     no gaps between launches.  Timed like the main region, after it.  Then
-    the per-chunk latency under replay: one graph per chunk step, replayed in
-    order with events between them (median over `steps` passes)."""
+    the per-chunk latency under replay: each step's attention launch (and
+    combine) as its own graph, replayed in order with events between them
+    (median over `steps` passes)."""
     import torch
     graph = pf.capture(q, k, v)
     for _ in range(args.warmup):
@@ -681,16 +698,12 @@ def measure_graph(args, pf, q, k, v, dev, stream, total_flops, tokens, world):
             per[i].append(ev[i].elapsed_time(ev[i + 1]))
     pc = [statistics.median(x) for x in per]
     del graphs
-    # step 0 also carries the prompt's one standalone append; steps 1.. are
-    # one attention launch (plus a split-KV combine) each
-    spread = pc[1:] if len(pc) > 2 else pc
     return {"ms_per_step": ms, "value": replica_throughput(total_flops, ms, world) / 1e12,
             "unit": "TFLOP/s", "prefill_tokens_per_s": replica_throughput(tokens, ms, world),
             "per_chunk_ms": {"min": min(pc), "max": max(pc), "max_over_min": max(pc) / min(pc),
                              "cv": statistics.pstdev(pc) / statistics.mean(pc),
-                             "max_over_min_steps_1_on": max(spread) / min(spread),
-                             "note": "one graph per chunk step, replayed in order, events "
-                                     "between replays"}}
+                             "note": "each step's attention launch (and split-KV combine) as "
+                                     "its own graph, replayed in order, events between replays"}}
 
 
 def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):

@@ -14,6 +14,7 @@
  *   mocap_lbcp_partition_dp   boundaries from Algorithm 1's stage-1 DP (host)
  *   mocap_lbcp_gemm_weight    the DP's GEMM-term weight from measured rates (host)
  *   mocap_kv_append           chunk K/V -> contiguous bf16 KV cache (device)
+ *   mocap_kv_append_overlap   the same, sized to run beside an attention launch
  *   mocap_qkv_rope_append     QKV projection + RoPE + KV append (device GEMM)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
@@ -161,6 +162,24 @@ mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk,
                              int64_t cache_capacity, int64_t offset, int64_t len,
                              int32_t n_kv_heads, int32_t head_dim,
                              mocap_stream_t stream);
+
+/*
+ * mocap_kv_append_overlap -- mocap_kv_append with a kernel sized to run
+ * beside a concurrently running attention launch (Sec. 2.2: chunk i + 1's
+ * K/V can be written while chunk i attends, since chunk i never reads those
+ * rows).  Its CTAs are one warp of at most 32 registers per thread and use
+ * no shared memory: that fits in what an attention CTA (384 threads x 168
+ * registers) leaves free on an SM, so the copy proceeds on every SM while
+ * the attention runs instead of waiting for SMs to drain.  Meant for a
+ * second stream whose work is joined (event) before the attention that
+ * reads the rows.  Same arguments, checks and results as mocap_kv_append;
+ * its own bandwidth is lower (a few TB/s at most), by design.
+ */
+mocap_status mocap_kv_append_overlap(const void *k_chunk, const void *v_chunk,
+                                     void *k_cache, void *v_cache,
+                                     int64_t cache_capacity, int64_t offset, int64_t len,
+                                     int32_t n_kv_heads, int32_t head_dim,
+                                     mocap_stream_t stream);
 
 /*
  * mocap_qkv_rope_append -- a chunk's QKV projection, rotary embedding and KV

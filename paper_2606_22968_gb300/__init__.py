@@ -98,6 +98,16 @@ def mocap_kv_append(k_chunk, v_chunk, k_cache, v_cache, offset: int, stream=None
                                        _stream(stream)), "mocap_kv_append")
 
 
+def mocap_kv_append_overlap(k_chunk, v_chunk, k_cache, v_cache, offset: int, stream=None):
+    """mocap_kv_append with a kernel that runs beside a concurrent attention
+    launch (for a second stream)."""
+    length, n_kv, d = k_chunk.shape
+    _check(_lib.load().mocap_kv_append_overlap(_ptr(k_chunk), _ptr(v_chunk), _ptr(k_cache),
+                                               _ptr(v_cache), k_cache.shape[0], offset, length,
+                                               n_kv, d, _stream(stream)),
+           "mocap_kv_append_overlap")
+
+
 def mocap_qkv_rope_append(x, w_qkv, q_out, k_cache, v_cache, offset: int,
                           rope_theta: float = 500000.0, stream=None):
     """[Q|K|V] = x w_qkv^T, RoPE on Q/K at positions offset + r, Q -> q_out,

@@ -29,6 +29,8 @@ SIGNATURES = {
     "mocap_lbcp_gemm_weight": (c_i32, [ctypes.c_double, ctypes.c_double, c_i32,
                                        ctypes.POINTER(c_i64)]),
     "mocap_kv_append": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32, c_i32, c_vp]),
+    "mocap_kv_append_overlap": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32, c_i32,
+                                        c_vp]),
     "mocap_qkv_rope_append": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32,
                                       c_i32, c_i32, c_i32, c_f32, c_vp]),
     "mocap_chunk_attn": (c_i32, [c_vp, c_vp, c_vp, c_i64, c_i64, c_i32, c_i32, c_i32, c_f32,

@@ -249,8 +249,11 @@ __device__ __forceinline__ uint4 ld_stream_v4(const uint4 *ptr) {
 // destination rows are never read by this launch, so the copy needs no
 // ordering with the attention work; kernel completion publishes it to later
 // work on the stream.
+// Kept out of line: inlined into the attention kernel it changed the
+// register allocation of the whole kernel and cost about 12 % of its speed
+// (out of line, about 1.4 %, measured on GB300).
 template <int MAXI>
-__device__ __forceinline__ void append_share(const AttnParams<MAXI> &p, int tid, int nthreads) {
+__device__ __noinline__ void append_share(const AttnParams<MAXI> &p, int tid, int nthreads) {
   if (p.n_app == 0) return;
   const int64_t ctas = gridDim.x;
   const int64_t cta = blockIdx.x;
@@ -286,7 +289,7 @@ __device__ __forceinline__ void append_share(const AttnParams<MAXI> &p, int tid,
 
 // Warpgroup 0: warp 0 is the TMA producer, warp 1 the MMA issuer (one lane
 // each); warps 2-3 copy this CTA's share of the launch's KV appends, if any.
-template <int D, int MAXI>
+template <int D, int MAXI, bool APPEND>
 __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_t base,
                                               uint32_t bars, uint32_t tmem, uint32_t warp,
                                               uint32_t lane, int item, int g, int h0, int r0,
@@ -414,7 +417,7 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
       mbar_wait(bar(L::kBarDrain), 0, p.status, kDrainLimitNs, false);
     }
     __syncwarp();
-  } else {
+  } else if constexpr (APPEND) {
     append_share(p, static_cast<int>(threadIdx.x) - 64, 64);  // warps 2-3
   }
 }
@@ -428,7 +431,7 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
 //   O_s += P_s V    M = 256 (P in each CTA's TMEM), N = 128 dims
 // and its commits arrive on both CTAs' barriers.  Both CTAs' copies count on
 // the first CTA's barriers, and so do both CTAs' P arrivals.
-template <int MAXI>
+template <int MAXI, bool APPEND>
 __device__ __forceinline__ void control_roles_pair(const AttnParams<MAXI> &p, uint32_t base,
                                                    uint32_t bars, uint32_t tmem, uint32_t warp,
                                                    uint32_t lane, uint32_t rank, int item, int g,
@@ -579,7 +582,7 @@ __device__ __forceinline__ void control_roles_pair(const AttnParams<MAXI> &p, ui
     }
     __syncwarp();
   } else if (warp >= 2) {
-    append_share(p, static_cast<int>(threadIdx.x) - 64, 64);  // warps 2-3
+    if constexpr (APPEND) append_share(p, static_cast<int>(threadIdx.x) - 64, 64);  // warps 2-3
   }
 }
 
@@ -748,7 +751,10 @@ __device__ __forceinline__ void cta_barrier() {
   asm volatile("barrier.sync 1, %0;" ::"n"(kThreads) : "memory");
 }
 
-template <int D, int MAXI, bool PAIR = false>
+// APPEND: the launch carries KV appends (warps 2-3 copy them).  A separate
+// instantiation, so launches without appends run exactly the code they
+// would without this feature.
+template <int D, int MAXI, bool PAIR = false, bool APPEND = false>
 __global__ void __launch_bounds__(kThreads, 1)
     chunk_attn_kernel(const __grid_constant__ AttnParams<MAXI> p) {
   using L = Layout<D, PAIR>;
@@ -802,7 +808,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (n_kv <= 0) {
     // No key tile in this split (the host never schedules one): an empty
     // partial, weight 0 in the combine, and this CTA's share of the appends.
-    if (warp == 2 || warp == 3) append_share(p, static_cast<int>(threadIdx.x) - 64, 64);
+    if constexpr (APPEND)
+      if (warp == 2 || warp == 3) append_share(p, static_cast<int>(threadIdx.x) - 64, 64);
     if (p.splits > 1 && warp >= 4) {
       const int sl = static_cast<int>(warp - 4) / 4;
       const int row = static_cast<int>((warp & 3u) * 32 + lane);
@@ -856,7 +863,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (run) {
       if (warp < 4) {
         setmaxnreg_dec<kRegsControl>();
-        control_roles_pair<MAXI>(p, base, bar(0), tmem, warp, lane, rank, item, g, h0, r0, nslots,
+        control_roles_pair<MAXI, APPEND>(p, base, bar(0), tmem, warp, lane, rank, item, g, h0, r0, nslots,
                                  t0, n_kv);
       } else {
         setmaxnreg_inc<kRegsSoftmax>();
@@ -874,7 +881,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     if (warp < 4) {
       setmaxnreg_dec<kRegsControl>();
-      control_roles<D, MAXI>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, t0,
+      control_roles<D, MAXI, APPEND>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, t0,
                              n_kv);
       tc_fence_before();
       cta_barrier();
@@ -1164,38 +1171,51 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     done[dev] = true;
     return MOCAP_OK;
   };
+  // the CTA-pair or single-CTA form, each with or without the append copy
+  auto launch_form = [&](auto kern, bool as_pair, int smem, bool *done) -> mocap_status {
+    const mocap_status st = prepare(kern, smem, done);
+    if (st != MOCAP_OK) return st;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(ctas));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = as_pair ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, prm) == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+  };
+  const bool append = prm.n_app > 0;
+  mocap_status lst = MOCAP_OK;
   bool launched = false;
   if constexpr (D == 128) {
     if (pair) {
       if (ctas % 2 != 0) return MOCAP_EINVAL;  // whole pairs by construction
-      using LP = Layout<D, true>;
-      auto kern = chunk_attn_kernel<D, MAXI, true>;
-      static bool done[64] = {};
-      const mocap_status st = prepare(kern, LP::kBytes, done);
-      if (st != MOCAP_OK) return st;
-      cudaLaunchConfig_t cfg = {};
-      cfg.gridDim = dim3(static_cast<unsigned>(ctas));
-      cfg.blockDim = dim3(kThreads);
-      cfg.dynamicSmemBytes = LP::kBytes;
-      cfg.stream = stream;
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = 2;
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = 1;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      if (cudaLaunchKernelEx(&cfg, kern, prm) != cudaSuccess) return MOCAP_ECUDA;
+      constexpr int kSmem = Layout<D, true>::kBytes;
+      if (append) {
+        static bool done[64] = {};
+        lst = launch_form(chunk_attn_kernel<D, MAXI, true, true>, true, kSmem, done);
+      } else {
+        static bool done[64] = {};
+        lst = launch_form(chunk_attn_kernel<D, MAXI, true, false>, true, kSmem, done);
+      }
       launched = true;
     }
   }
   if (!launched) {
-    auto kern = chunk_attn_kernel<D, MAXI>;
-    static bool done[64] = {};
-    const mocap_status st = prepare(kern, L::kBytes, done);
-    if (st != MOCAP_OK) return st;
-    kern<<<static_cast<unsigned>(ctas), kThreads, L::kBytes, stream>>>(prm);
+    if (append) {
+      static bool done[64] = {};
+      lst = launch_form(chunk_attn_kernel<D, MAXI, false, true>, false, L::kBytes, done);
+    } else {
+      static bool done[64] = {};
+      lst = launch_form(chunk_attn_kernel<D, MAXI, false, false>, false, L::kBytes, done);
+    }
   }
+  if (lst != MOCAP_OK) return lst;
   if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
   if (sp.splits > 1) {
     // the item's rows start at q_row of the packed out / lse (0 for a

@@ -16,7 +16,7 @@ import torch
 
 from . import (MOCAP_COST_CAUSAL, MOCAP_PART_LBCP, MOCAP_PART_UNIFORM, mocap_chunk_attn,
                mocap_chunk_attn_append, mocap_chunk_attn_varlen, mocap_chunk_attn_varlen_append,
-               mocap_chunk_attn_workspace_size, mocap_kv_append,
+               mocap_chunk_attn_workspace_size, mocap_kv_append, mocap_kv_append_overlap,
                mocap_lbcp_gemm_weight, mocap_lbcp_partition, mocap_lbcp_partition_dp,
                mocap_qkv_rope_append)
 from .workloads import GRANULARITY, Workload, request_offsets
@@ -40,6 +40,9 @@ def stage_balanced_bounds(seq_len: int, num_chunks: int, attn_s_per_pair: float,
                                    gemm_weight(attn_s_per_pair, gemm_s_per_row, granularity))
 
 
+APPEND_MODES = ("serial", "fused", "overlap")
+
+
 class ChunkedPrefill:
     """Buffers and launch sequence for one workload on one device.
 
@@ -51,14 +54,24 @@ class ChunkedPrefill:
     """
 
     def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True,
-                 bounds: Optional[List[List[int]]] = None, fuse_appends: bool = True):
+                 bounds: Optional[List[List[int]]] = None, append_mode: str = "overlap"):
         """``bounds`` (one boundary list per request) replaces the workload's
         partition rule, e.g. with the Algorithm 1 stage-1 DP's split.
-        ``fuse_appends`` lets each attention launch append the next step's
-        chunks (mocap_chunk_attn_append); False launches one append per chunk
-        before its attention (mocap_kv_append)."""
+
+        ``append_mode`` says how chunk K/V reach the cache (step 0's chunks
+        are always appended by a launch of their own before its attention):
+          "serial"   each step appends its chunks (mocap_kv_append), then
+                     attends, all on one stream;
+          "fused"    each step's attention launch also appends the next
+                     step's chunks (mocap_chunk_attn_append);
+          "overlap"  a second stream appends steps 1.. in order
+                     (mocap_kv_append_overlap, a kernel that fits beside the
+                     attention CTAs), and step i's attention waits for its
+                     own chunks' event only."""
+        if append_mode not in APPEND_MODES:
+            raise ValueError(f"append_mode must be one of {APPEND_MODES}")
         self.w = w
-        self.fuse_appends = fuse_appends
+        self.append_mode = append_mode
         self.device = torch.device(device)
         self.mode = w.mode if mode is None else mode
         self.fixed_bounds = None if bounds is None else [list(b) for b in bounds]
@@ -117,20 +130,20 @@ class ChunkedPrefill:
         return self.lse.view(self.w.n_q_heads, self.w.total_tokens)
 
     # -- execution ----------------------------------------------------------------
-    def run_step(self, q, k, v, i, stream=None, events=None):
+    def run_step(self, q, k, v, i, stream=None, events=None, ready=None, attention_only=False):
         """Step ``i`` of ``steps()`` (one chunk index of every request that has
-        it).  With fused appends (the default) step 0 first appends its own
-        chunks, and every step's attention launch also appends the next step's
-        chunks (rows it never reads); otherwise each step appends its own
-        chunks, then attends.  ``events`` is an optional triple of CUDA events
-        recorded before the step's own appends (step 0 only when fused),
-        before the attention launch, and after it.  With MOCAP_NVTX=1 in the
-        environment each step is an NVTX range ("mocap chunk <index>") for
-        timeline profilers."""
+        it), as ``append_mode`` says.  ``ready`` is the event after which step
+        i's chunks are in the cache (overlap mode, from ``launch_appends``);
+        without one, step i appends its own chunks first.  ``attention_only``
+        skips every append (the caches already hold the rows).  ``events`` is
+        an optional triple of CUDA events recorded before the step's own
+        appends, before the attention launch, and after it.  With MOCAP_NVTX=1
+        in the environment each step is an NVTX range ("mocap chunk <index>")
+        for timeline profilers."""
         if os.environ.get("MOCAP_NVTX", "0") != "0":
             with torch.cuda.nvtx.range(f"mocap chunk {i}"):
-                return self._run_step(q, k, v, i, stream, events)
-        return self._run_step(q, k, v, i, stream, events)
+                return self._run_step(q, k, v, i, stream, events, ready, attention_only)
+        return self._run_step(q, k, v, i, stream, events, ready, attention_only)
 
     def _append_rows(self, k, v, r, c):
         """(K rows, V rows, destination cache row) of chunk c of request r."""
@@ -138,25 +151,54 @@ class ChunkedPrefill:
         base = self.cu[r]
         return k[base + b0:base + b1], v[base + b0:base + b1], base + b0
 
-    def _run_step(self, q, k, v, i, stream=None, events=None):
+    def launch_appends(self, k, v, stream=None, landed=None):
+        """Overlap mode: on a second stream, the appends of steps 1.. in step
+        order (each after ``landed[i]`` if given, e.g. its host upload), each
+        step followed by an event.  The second stream starts after the work
+        queued so far on ``stream``.  Returns the per-step events (None for
+        step 0, which run_step appends itself) and the second stream."""
+        main = torch.cuda.current_stream(self.device) if stream is None else stream
+        side = torch.cuda.Stream(self.device)
+        side.wait_stream(main)
+        ready = [None]
+        with torch.cuda.stream(side):
+            for i, step in enumerate(self.steps()):
+                if i == 0:
+                    continue
+                if landed is not None:
+                    side.wait_event(landed[i])
+                for r, c in step:
+                    kr, vr, dst = self._append_rows(k, v, r, c)
+                    mocap_kv_append_overlap(kr, vr, self.k_cache, self.v_cache, dst, stream=side)
+                ev = torch.cuda.Event()
+                ev.record(side)
+                ready.append(ev)
+        return ready, side
+
+    def _run_step(self, q, k, v, i, stream=None, events=None, ready=None, attention_only=False):
         w = self.w
+        mode = self.append_mode
         steps = self.steps()
         step = steps[i]
         if events is not None:
             events[0].record(stream)
-        if not self.fuse_appends or i == 0:
-            for r, c in step:
-                kr, vr, dst = self._append_rows(k, v, r, c)
-                mocap_kv_append(kr, vr, self.k_cache, self.v_cache, dst, stream=stream)
+        if not attention_only:
+            if ready is not None:
+                (torch.cuda.current_stream(self.device) if stream is None else stream).wait_event(
+                    ready)
+            elif mode != "fused" or i == 0:
+                for r, c in step:
+                    kr, vr, dst = self._append_rows(k, v, r, c)
+                    mocap_kv_append(kr, vr, self.k_cache, self.v_cache, dst, stream=stream)
         nxt = []
-        if self.fuse_appends and i + 1 < len(steps):
+        if mode == "fused" and not attention_only and i + 1 < len(steps):
             nxt = [self._append_rows(k, v, r, c) for r, c in steps[i + 1]]
         if events is not None:
             events[1].record(stream)
         if self.single:
             (_, c), = step
             b0, b1 = self.bounds[0][c], self.bounds[0][c + 1]
-            if self.fuse_appends:
+            if nxt:
                 mocap_chunk_attn_append(q[b0:b1], self.k_cache, self.v_cache, b0,
                                         self.out[b0:b1], self.chunk_lse(c), w.scale, nxt,
                                         workspace=self.workspace, stream=stream)
@@ -169,7 +211,7 @@ class ChunkedPrefill:
             for r, c in step:
                 b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
                 items.append((self.cu[r] + b0, self.cu[r], b0, b1 - b0))
-            if self.fuse_appends:
+            if nxt:
                 mocap_chunk_attn_varlen_append(q, self.k_cache, self.v_cache, items, self.out,
                                                self.lse_packed(), w.scale, nxt,
                                                workspace=self.workspace, stream=stream)
@@ -180,11 +222,24 @@ class ChunkedPrefill:
         if events is not None:
             events[2].record(stream)
 
-    def run(self, q, k, v, stream=None, chunk_events=None):
+    def run(self, q, k, v, stream=None, chunk_events=None, landed=None):
         """The whole prompt: every step in order.  ``chunk_events`` optionally
-        holds one event triple per step (see run_step)."""
-        for i in range(len(self.steps())):
-            self.run_step(q, k, v, i, stream, None if chunk_events is None else chunk_events[i])
+        holds one event triple per step (see run_step); ``landed`` optionally
+        one event per step after which its inputs are in q, k, v."""
+        main = torch.cuda.current_stream(self.device) if stream is None else stream
+        n = len(self.steps())
+        ready, side = [None] * n, None
+        if self.append_mode == "overlap" and n > 1:
+            ready, side = self.launch_appends(k, v, main, landed)
+        for i in range(n):
+            if landed is not None:
+                main.wait_event(landed[i])
+                if self.append_mode == "fused" and i + 1 < n:
+                    main.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
+            self.run_step(q, k, v, i, stream, None if chunk_events is None else chunk_events[i],
+                          ready[i])
+        if side is not None:
+            main.wait_stream(side)
 
     def run_stage(self, x, w_qkv, q_buf, stream=None, rope_theta: float = 500000.0,
                   chunk_events=None):
@@ -213,6 +268,34 @@ class ChunkedPrefill:
     def _rows(self, r, c):
         b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
         return slice(self.cu[r] + b0, self.cu[r] + b1), b0, b1
+
+    def _compute_and_return(self, q, k, v, compute, d2h, landed, host_out, host_lse):
+        """Every step on ``compute`` once its inputs have landed (events
+        ``landed``), each step's O (and a single request's LSE block) copied
+        back on ``d2h`` as soon as that step is done."""
+        steps = self.steps()
+        hq = self.w.n_q_heads
+        n = len(steps)
+        ready, side = [None] * n, None
+        if self.append_mode == "overlap" and n > 1:
+            ready, side = self.launch_appends(k, v, compute, landed)
+        for i, step in enumerate(steps):
+            compute.wait_event(landed[i])
+            if self.append_mode == "fused" and i + 1 < n:
+                compute.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
+            self.run_step(q, k, v, i, compute, ready=ready[i])
+            done = torch.cuda.Event()
+            done.record(compute)
+            d2h.wait_event(done)
+            with torch.cuda.stream(d2h):
+                for r, c in step:
+                    rows, b0, b1 = self._rows(r, c)
+                    host_out[rows].copy_(self.out[rows], non_blocking=True)
+                    if self.single:
+                        host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
+                                                        non_blocking=True)
+        if side is not None:
+            compute.wait_stream(side)
 
     def run_from_host(self, host_q, host_k, host_v, host_out, host_lse, q, k, v):
         """The whole prompt from (pinned) host memory, overlapping transfers
@@ -246,21 +329,7 @@ class ChunkedPrefill:
                 ev.record(h2d)
                 landed.append(ev)
         d2h.wait_stream(compute)
-        for i, step in enumerate(steps):
-            compute.wait_event(landed[i])
-            if self.fuse_appends and i + 1 < len(steps):
-                compute.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
-            self.run_step(q, k, v, i, compute)
-            done = torch.cuda.Event()
-            done.record(compute)
-            d2h.wait_event(done)
-            with torch.cuda.stream(d2h):
-                for r, c in step:
-                    rows, b0, b1 = self._rows(r, c)
-                    host_out[rows].copy_(self.out[rows], non_blocking=True)
-                    if self.single:
-                        host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
-                                                        non_blocking=True)
+        self._compute_and_return(q, k, v, compute, d2h, landed, host_out, host_lse)
         if not self.single:
             d2h.wait_stream(compute)
             with torch.cuda.stream(d2h):
@@ -322,21 +391,7 @@ class ChunkedPrefill:
             host_out, host_lse = prompts[p][3], prompts[p][4]
             if outputs_gone is not None:
                 compute.wait_event(outputs_gone)
-            for i, step in enumerate(steps):
-                compute.wait_event(landed[p][i])
-                if self.fuse_appends and i + 1 < len(steps):
-                    compute.wait_event(landed[p][i + 1])  # appended by this launch
-                self.run_step(q, k, v, i, compute)
-                done = torch.cuda.Event()
-                done.record(compute)
-                d2h.wait_event(done)
-                with torch.cuda.stream(d2h):
-                    for r, c in step:
-                        rows, b0, b1 = self._rows(r, c)
-                        host_out[rows].copy_(self.out[rows], non_blocking=True)
-                        if self.single:
-                            host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
-                                                            non_blocking=True)
+            self._compute_and_return(q, k, v, compute, d2h, landed[p], host_out, host_lse)
             end = torch.cuda.Event()
             end.record(compute)
             computed[p % 2] = end
@@ -352,9 +407,10 @@ class ChunkedPrefill:
 
     # -- CUDA graph ------------------------------------------------------------------
     def capture_steps(self, q, k, v, stream=None):
-        """One CUDA graph per step (its launches as ``run_step`` enqueues them);
-        replaying them in order is the whole prompt, and events recorded
-        between the replays time each chunk step without host gaps inside
+        """One CUDA graph per step holding that step's attention launch (and
+        split-KV combine) only; the caches must already hold the prompt's
+        K/V (e.g. from ``run``).  Replaying them in order with events between
+        the replays times each chunk's attention without host gaps inside
         it.  Same preconditions as ``capture``."""
         graphs = []
         side = torch.cuda.Stream(self.device) if stream is None else stream
@@ -363,7 +419,7 @@ class ChunkedPrefill:
             for i in range(len(self.steps())):
                 g = torch.cuda.CUDAGraph()
                 with torch.cuda.graph(g, stream=side):
-                    self.run_step(q, k, v, i, side)
+                    self.run_step(q, k, v, i, side, attention_only=True)
                 graphs.append(g)
         torch.cuda.current_stream(self.device).wait_stream(side)
         return graphs

@@ -79,8 +79,21 @@ def test_fused_append_bitwise(m, monkeypatch, prefix, length, hq, hkv, d, app_ro
                        dtype=torch.bfloat16)[:length]
     lse_f = torch.full((hq, max(length, 1)), float("nan"), device=dev,
                        dtype=torch.float32)[:, :length]
-    m.mocap_chunk_attn_append(q, k_cache, v_cache, prefix, out_f, lse_f, scale, appends,
-                              workspace=ws)
+    if length > 0:
+        m.mocap_chunk_attn_append(q, k_cache, v_cache, prefix, out_f, lse_f, scale, appends,
+                                  workspace=ws)
+    else:
+        # torch reports a null data pointer for empty tensors, so the C ABI is
+        # called directly with the (unused) one-row buffers behind them
+        from paper_2606_22968_gb300._lib import AppendItem
+        arr = (AppendItem * len(appends))(*[AppendItem(ks.data_ptr(), vs.data_ptr(), r0,
+                                                       ks.shape[0]) for ks, vs, r0 in appends])
+        base_q = q.untyped_storage().data_ptr()
+        base_o = out_f.untyped_storage().data_ptr()
+        base_l = lse_f.untyped_storage().data_ptr()
+        assert m._lib.load().mocap_chunk_attn_append(
+            base_q, k_cache.data_ptr(), v_cache.data_ptr(), prefix, 0, hq, hkv, d, scale, base_o,
+            base_l, None, 0, arr, len(appends), cap, torch.cuda.current_stream().cuda_stream) == 0
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == 0
     # appended rows bitwise, every other row untouched
@@ -148,20 +161,21 @@ def test_varlen_fused_append_bitwise(m):
                      lse_f[:, a:a + cut[r]].cpu().numpy(), o_ref, l_ref, f"request {r}")
 
 
+@pytest.mark.parametrize("mode", ["fused", "overlap"])
 @pytest.mark.parametrize("index", [1, 2, 3, 5])
-def test_fused_pipeline_equals_unfused_pipeline(m, index):
-    """The prompt with each next chunk's append in the attention launch gives
-    bitwise the results of one append launch per chunk, eager and replayed
-    from a CUDA graph."""
+def test_append_modes_equal_serial_pipeline(m, index, mode):
+    """The prompt with each next chunk's append in the attention launch
+    ("fused") or on a second stream beside it ("overlap") gives bitwise the
+    results of one append launch per chunk on one stream ("serial"), eager
+    and replayed from a CUDA graph, caches poisoned with NaN first."""
     from paper_2606_22968_gb300 import workloads
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
     w = workloads.get(index)
     dev = torch.device("cuda")
     q, k, v = workloads.make_qkv(w, dev)
-    pu = ChunkedPrefill(w, dev, fuse_appends=False)
+    pu = ChunkedPrefill(w, dev, append_mode="serial")
     pu.run(q, k, v)
-    pf = ChunkedPrefill(w, dev)
-    assert pf.fuse_appends
+    pf = ChunkedPrefill(w, dev, append_mode=mode)
     for t in (pf.out, pf.lse, pf.k_cache, pf.v_cache):
         t.fill_(float("nan"))
     pf.run(q, k, v)
@@ -170,39 +184,75 @@ def test_fused_pipeline_equals_unfused_pipeline(m, index):
     assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
     assert torch.equal(pf.out, pu.out) and torch.equal(pf.lse, pu.lse)
     graph = pf.capture(q, k, v)
-    for t in (pf.out, pf.lse, pf.k_cache, pf.v_cache):
-        t.fill_(float("nan"))
-    graph.replay()
-    torch.cuda.synchronize()
-    assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
-    assert torch.equal(pf.out, pu.out) and torch.equal(pf.lse, pu.lse)
+    for _ in range(2):
+        for t in (pf.out, pf.lse, pf.k_cache, pf.v_cache):
+            t.fill_(float("nan"))
+        graph.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
+        assert torch.equal(pf.out, pu.out) and torch.equal(pf.lse, pu.lse)
     del graph
 
 
-def test_fused_step_graphs_against_oracle(m):
-    """The 131072-token workload replayed as one CUDA graph per chunk step
-    (each step's attention launch appending the next chunk), caches and
-    outputs poisoned first: caches bitwise, every chunk against the oracle
-    on its first, tile-edge, middle and last rows (four rotating heads)."""
+def test_overlap_pipeline_and_step_graphs_against_oracle(m):
+    """The 131072-token workload with its appends on a second stream (caches
+    and outputs poisoned first): caches bitwise, every chunk against the
+    oracle on its first, tile-edge, middle and last rows (four rotating
+    heads); then its per-step attention graphs replayed in order give the
+    same bits."""
     from paper_2606_22968_gb300 import workloads
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
     from tests.parity_utils import rotating_heads
     w = workloads.get(4)
     dev = torch.device("cuda")
     q, k, v = workloads.make_qkv(w, dev)
-    pf = ChunkedPrefill(w, dev)
-    pf.run(q, k, v)
-    graphs = pf.capture_steps(q, k, v)
+    pf = ChunkedPrefill(w, dev, append_mode="overlap")
     for t in (pf.out, pf.lse, pf.k_cache, pf.v_cache):
         t.fill_(float("nan"))
-    for g in graphs:
-        g.replay()
+    pf.run(q, k, v)
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == 0
     assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
     check_single_request(pf, q, k, v, rows_fn=lambda n, i: np.array([0, 127, 128, n // 2, n - 1]),
                          heads_fn=rotating_heads(64))
+    out_ref, lse_ref = pf.out.clone(), pf.lse.clone()
+    graphs = pf.capture_steps(q, k, v)
+    pf.out.fill_(float("nan"))
+    pf.lse.fill_(float("nan"))
+    for g in graphs:
+        g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(pf.out, out_ref) and torch.equal(pf.lse, lse_ref)
     del graphs
+
+
+@pytest.mark.parametrize("index", [3, 5])
+def test_overlap_mode_from_host_matches_device_run(m, index):
+    """Host-streamed prompts with overlapped appends (the second stream waits
+    for each step's upload) give bitwise the device-resident results."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(index)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev, append_mode="overlap")
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    out_ref, lse_ref = pf.out.clone(), pf.lse.clone()
+    hq, hk, hv = (t.cpu().pin_memory() for t in (q, k, v))
+    outs = []
+    for _ in range(3):
+        ho = torch.full(pf.out.shape, float("nan"), dtype=pf.out.dtype).pin_memory()
+        hl = torch.full(pf.lse.shape, float("nan"), dtype=pf.lse.dtype).pin_memory()
+        outs.append((hq, hk, hv, ho, hl))
+    bufs = [tuple(torch.full_like(t, float("nan")) for t in (q, k, v)) for _ in range(2)]
+    pf.k_cache.fill_(float("nan"))
+    pf.v_cache.fill_(float("nan"))
+    pf.run_prompts_from_host(outs, bufs)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    for _, _, _, ho, hl in outs:
+        assert torch.equal(ho, out_ref.cpu()) and torch.equal(hl, lse_ref.cpu())
 
 
 def test_fused_launch_after_expired_wait_does_nothing(m):
