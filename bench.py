@@ -67,6 +67,9 @@ def parse_args():
     ap.add_argument("--case-append", default=None,
                     help="profiling case 'rows,Hkv,d': one KV append launch repeated "
                          "warmup+steps times")
+    ap.add_argument("--case-append-overlap", action="store_true",
+                    help="with --case-append: time mocap_kv_append_overlap (the one-warp "
+                         "kernel meant to run beside attention) instead of mocap_kv_append")
     ap.add_argument("--case-qkv", default=None,
                     help="profiling case 'len,hidden,Hq,Hkv,d': one QKV projection launch "
                          "repeated warmup+steps times")
@@ -100,8 +103,10 @@ def load_peaks():
 
 
 def kernel_source_hash():
+    """Hash of the attention kernel's device source (the kernel header and the
+    PTX wrappers it uses), which the committed DRAM captures were taken on."""
     h = hashlib.sha256()
-    for f in ("chunk_attn.cu", "sm103_ptx.cuh"):
+    for f in ("attn_kernel.cuh", "sm103_ptx.cuh"):
         with open(os.path.join(ROOT, "paper_2606_22968_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -941,11 +946,13 @@ def profile_case_append(args):
     k = torch.randn((rows, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
     v = torch.randn((rows, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
     kc, vc = torch.empty_like(k), torch.empty_like(v)
-    ms = _repeat_timed(args, lambda: m.mocap_kv_append(k, v, kc, vc, 0))
+    fn = m.mocap_kv_append_overlap if args.case_append_overlap else m.mocap_kv_append
+    ms = _repeat_timed(args, lambda: fn(k, v, kc, vc, 0))
     if not (torch.equal(kc, k) and torch.equal(vc, v)):
         raise RuntimeError("append probe: cache differs from the chunk")
     byts = 2 * 2 * rows * hkv * d * 2
-    print(json.dumps({"case_append": args.case_append, "ms": ms, "bytes": byts,
+    print(json.dumps({"case_append": args.case_append, "overlap_kernel": args.case_append_overlap,
+                      "ms": ms, "bytes": byts,
                       "gb_per_s": byts / ms / 1e6}), flush=True)
     return 0
 

@@ -1,0 +1,94 @@
+// attn_combine.cuh -- the split-KV combine kernel (device code) on sm_103a.
+#pragma once
+
+#include <cmath>
+#include <cuda_bf16.h>
+
+#include "attn_kernel.cuh"
+
+namespace mocap {
+namespace {
+
+// Split-KV combine: the softmax over the union of disjoint key ranges weighs
+// each range's normalised output by exp(LSE_k - LSE), LSE = ln sum_k exp(LSE_k).
+// One warp per (row, head); each lane owns D/32 consecutive columns.  The
+// partial outputs are loaded before the range LSEs (they do not depend on
+// the weights), so both DRAM round trips overlap.  Like the attention launch
+// before it, it does nothing once a bounded wait has expired (the status
+// word is set), so the outputs keep their contents.
+template <int D>
+__global__ void __launch_bounds__(256) attn_combine_kernel(
+    const float *__restrict__ o_part, const float *__restrict__ lse_part, int splits,
+    int64_t len, int n_q_heads, __nv_bfloat16 *__restrict__ out, float *__restrict__ lse,
+    int64_t lse_stride, const uint32_t *status) {
+  constexpr int kPer = D / 32;
+  if (*reinterpret_cast<const volatile uint32_t *>(status) != 0u) return;
+  const int64_t idx = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (idx >= len * n_q_heads) return;
+  const int lane = threadIdx.x & 31;
+  const int64_t row = idx / n_q_heads;
+  const int h = static_cast<int>(idx % n_q_heads);
+  float o[kMaxSplits][kPer];
+#pragma unroll
+  for (int k = 0; k < kMaxSplits; ++k) {
+    if (k < splits) {
+      const float *src =
+          o_part + ((static_cast<int64_t>(k) * len + row) * n_q_heads + h) * D + lane * kPer;
+      if constexpr (kPer == 4) {
+        const float4 v = __ldcs(reinterpret_cast<const float4 *>(src));
+        o[k][0] = v.x;
+        o[k][1] = v.y;
+        o[k][2] = v.z;
+        o[k][3] = v.w;
+      } else {
+        const float2 v = __ldcs(reinterpret_cast<const float2 *>(src));
+        o[k][0] = v.x;
+        o[k][1] = v.y;
+      }
+    }
+  }
+  float lk[kMaxSplits];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int k = 0; k < kMaxSplits; ++k) {
+    if (k < splits) {
+      lk[k] = __ldcs(lse_part + (static_cast<int64_t>(k) * n_q_heads + h) * len + row);
+      mx = fmaxf(mx, lk[k]);
+    }
+  }
+  float wsum = 0.0f;
+#pragma unroll
+  for (int k = 0; k < kMaxSplits; ++k) {
+    if (k < splits) {
+      lk[k] = lk[k] > -INFINITY ? expf(lk[k] - mx) : 0.0f;
+      wsum += lk[k];
+    }
+  }
+  const float inv = 1.0f / wsum;
+  float acc[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) acc[e] = 0.0f;
+#pragma unroll
+  for (int k = 0; k < kMaxSplits; ++k) {
+    if (k < splits) {
+      const float wk = lk[k] * inv;
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) acc[e] += wk * o[k][e];
+    }
+  }
+  __nv_bfloat16 *dst = out + (row * n_q_heads + h) * D + lane * kPer;
+  if constexpr (kPer == 4) {
+    const __nv_bfloat162 a = __floats2bfloat162_rn(acc[0], acc[1]);
+    const __nv_bfloat162 b = __floats2bfloat162_rn(acc[2], acc[3]);
+    uint2 pk;
+    pk.x = *reinterpret_cast<const uint32_t *>(&a);
+    pk.y = *reinterpret_cast<const uint32_t *>(&b);
+    *reinterpret_cast<uint2 *>(dst) = pk;
+  } else {
+    *reinterpret_cast<__nv_bfloat162 *>(dst) = __floats2bfloat162_rn(acc[0], acc[1]);
+  }
+  if (lane == 0) lse[static_cast<int64_t>(h) * lse_stride + row] = mx + logf(wsum);
+}
+
+}  // namespace
+}  // namespace mocap
