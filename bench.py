@@ -53,6 +53,9 @@ def parse_args():
                     help="skip the QKV projection + RoPE + append measurement")
     ap.add_argument("--hidden", type=int, default=8192,
                     help="hidden size for the projection measurement (Llama-3-70B: 8192)")
+    ap.add_argument("--no-append-modes", action="store_true",
+                    help="skip the append measurements after the timed region (the append "
+                         "graphs and the comparison of the three append modes)")
     ap.add_argument("--no-last-row", action="store_true",
                     help="skip the last-row-only attention measurement")
     ap.add_argument("--no-uniform", action="store_true",
@@ -544,8 +547,9 @@ def ours_arm(args, rank, world, local):
         # thermal state of the GPU (the auxiliary measurements below add
         # about a minute of load first)
         line["e2e"] = measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world)
-    line["append"].update(measure_append_graph(m, w, pf, k, v, dev, hbm))
-    line["append"].update(measure_fusion(args, pf, w, q, k, v, dev, stream, total_flops))
+    if not args.no_append_modes:
+        line["append"].update(measure_append_graph(m, w, pf, k, v, dev, hbm))
+        line["append"].update(measure_fusion(args, pf, w, q, k, v, dev, stream, total_flops))
     if not args.no_graph:
         line["graph_replay"] = measure_graph(args, pf, q, k, v, dev, stream, total_flops,
                                              w.total_tokens, world)

@@ -11,7 +11,8 @@ namespace {
 
 // Split-KV combine: the softmax over the union of disjoint key ranges weighs
 // each range's normalised output by exp(LSE_k - LSE), LSE = ln sum_k exp(LSE_k).
-// One warp per (row, head); each lane owns D/32 consecutive columns.  The
+// One warp per (row, head): block (row, g) holds heads 8g .. 8g + 7, so no
+// index division is needed; each lane owns D/32 consecutive columns.  The
 // partial outputs are loaded before the range LSEs (they do not depend on
 // the weights), so both DRAM round trips overlap.  Like the attention launch
 // before it, it does nothing once a bounded wait has expired (the status
@@ -23,11 +24,10 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(
     int64_t lse_stride, const uint32_t *status) {
   constexpr int kPer = D / 32;
   if (*reinterpret_cast<const volatile uint32_t *>(status) != 0u) return;
-  const int64_t idx = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
-  if (idx >= len * n_q_heads) return;
+  const int64_t row = blockIdx.x;
+  const int h = static_cast<int>(blockIdx.y) * 8 + static_cast<int>(threadIdx.x >> 5);
+  if (row >= len || h >= n_q_heads) return;
   const int lane = threadIdx.x & 31;
-  const int64_t row = idx / n_q_heads;
-  const int h = static_cast<int>(idx % n_q_heads);
   float o[kMaxSplits][kPer];
 #pragma unroll
   for (int k = 0; k < kMaxSplits; ++k) {
