@@ -553,6 +553,9 @@ def ours_arm(args, rank, world, local):
     if not args.no_graph:
         line["graph_replay"] = measure_graph(args, pf, q, k, v, dev, stream, total_flops,
                                              w.total_tokens, world)
+        if pf.append_mode == "overlap" and len(steps_plan) > 1:
+            line["chunk_streams"] = measure_chunk_streams(args, pf, w, q, k, v, dev, stream,
+                                                          total_flops)
     if pf.single and not args.no_projection:
         line["qkv_projection"] = measure_projection(args, m, w, pf, q, dev, stream, total_flops,
                                                     peak)
@@ -666,6 +669,36 @@ def measure_fusion(args, pf, w, q, k, v, dev, stream, total_flops, reps=3):
                                 "launch per chunk before its attention; fused = the next chunk's "
                                 "append inside the attention launch; overlap = appends on a "
                                 "second stream beside the attention launches"}
+
+
+def measure_chunk_streams(args, pf, w, q, k, v, dev, stream, total_flops, reps=3):
+    """The prompt with its attention launches on one compute stream and
+    alternating between two (ChunkedPrefill chunk_streams = 2: step i + 1 may
+    use SMs that step i's last wave leaves idle), each replayed from one CUDA
+    graph, interleaved, median of `reps`."""
+    import torch
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    p2 = ChunkedPrefill(w, dev, chunk_streams=2)
+    p2.k_cache, p2.v_cache, p2.out, p2.lse = pf.k_cache, pf.v_cache, pf.out, pf.lse
+    p2.run(q, k, v, stream)
+    graphs = {1: pf.capture(q, k, v), 2: p2.capture(q, k, v)}
+    times = {1: [], 2: []}
+    for _ in range(reps):
+        for n, g in graphs.items():
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            g.replay()
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            times[n].append(e0.elapsed_time(e1))
+    del graphs, p2
+    one, two = statistics.median(times[1]), statistics.median(times[2])
+    return {"graph_ms_per_step_one_stream": one, "graph_ms_per_step_two_streams": two,
+            "two_streams_value": total_flops / (two * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "note": "attention launches alternating between two compute streams "
+                    "(ChunkedPrefill chunk_streams=2), appends beside them; whole prompt "
+                    "replayed from one CUDA graph"}
 
 
 def measure_graph(args, pf, q, k, v, dev, stream, total_flops, tokens, world):

@@ -12,10 +12,8 @@
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kUnroll = 4;        // 16-byte vectors in flight per thread (overlap kernel)
-constexpr int kBigUnroll = 8;     // the same for the standalone kernel
-constexpr int kCtasPerSm = 4;     // standalone grid cap: 1024 threads per SM, each
-                                  // looping with 8 x 16 B in flight (128 KB per SM)
+constexpr int kUnroll = 4;        // 16-byte vectors in flight per thread
+constexpr int kCtasPerSm = 32;    // grid cap; the loop strides over the rest
 
 __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
   uint4 v;
@@ -26,25 +24,23 @@ __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
 }
 
 // Vectors [0, n) come from k_src -> k_dst, vectors [n, 2n) from v_src -> v_dst.
-// A persistent grid (a few CTAs per SM) strides over both ranges, each thread
-// keeping eight 16-byte loads in flight.
 __global__ void __launch_bounds__(kThreads) kv_append_kernel(const uint4 *__restrict__ k_src,
                                                              const uint4 *__restrict__ v_src,
                                                              uint4 *__restrict__ k_dst,
                                                              uint4 *__restrict__ v_dst,
                                                              int64_t n) {
   const int64_t total = 2 * n;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads * kBigUnroll;
-  for (int64_t base = static_cast<int64_t>(blockIdx.x) * kThreads * kBigUnroll + threadIdx.x;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads * kUnroll;
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * kThreads * kUnroll + threadIdx.x;
        base < total; base += stride) {
-    uint4 v[kBigUnroll];
+    uint4 v[kUnroll];
 #pragma unroll
-    for (int u = 0; u < kBigUnroll; ++u) {
+    for (int u = 0; u < kUnroll; ++u) {
       const int64_t i = base + static_cast<int64_t>(u) * kThreads;
       if (i < total) v[u] = ld_stream(i < n ? k_src + i : v_src + (i - n));
     }
 #pragma unroll
-    for (int u = 0; u < kBigUnroll; ++u) {
+    for (int u = 0; u < kUnroll; ++u) {
       const int64_t i = base + static_cast<int64_t>(u) * kThreads;
       if (i < total) {
         if (i < n) k_dst[i] = v[u];
@@ -130,7 +126,7 @@ extern "C" mocap_status mocap_kv_append(const void *k_chunk, const void *v_chunk
   const mocap_status st = check_append(k_chunk, v_chunk, k_cache, v_cache, cache_capacity,
                                        offset, len, n_kv_heads, head_dim, &n, &dst_off);
   if (st != MOCAP_OK || len == 0) return st;
-  const int64_t want = (2 * n + kThreads * kBigUnroll - 1) / (kThreads * kBigUnroll);
+  const int64_t want = (2 * n + kThreads * kUnroll - 1) / (kThreads * kUnroll);
   const int64_t cap = static_cast<int64_t>(mocap::device_sm_count()) * kCtasPerSm;
   const int blocks = static_cast<int>(std::max<int64_t>(1, std::min(want, cap)));
   kv_append_kernel<<<blocks, kThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(

@@ -54,7 +54,8 @@ class ChunkedPrefill:
     """
 
     def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True,
-                 bounds: Optional[List[List[int]]] = None, append_mode: str = "overlap"):
+                 bounds: Optional[List[List[int]]] = None, append_mode: str = "overlap",
+                 chunk_streams: int = 1):
         """``bounds`` (one boundary list per request) replaces the workload's
         partition rule, e.g. with the Algorithm 1 stage-1 DP's split.
 
@@ -67,11 +68,25 @@ class ChunkedPrefill:
           "overlap"  a second stream appends steps 1.. in order
                      (mocap_kv_append_overlap, a kernel that fits beside the
                      attention CTAs), and step i's attention waits for its
-                     own chunks' event only."""
+                     own chunks' event only.
+
+        ``chunk_streams`` = 2 issues the steps' attention launches alternately
+        on the caller's stream and a second compute stream (``run`` only):
+        step i + 1 reads no output of step i, only K/V rows already appended,
+        so its CTAs may take SMs that step i's last wave leaves idle.  Each
+        compute stream has its own split-KV workspace.  Steps are still
+        issued in order; per-step events then time overlapping launches.
+        Needs append_mode "overlap": every step then waits for an event that
+        says its rows (and all earlier rows) are in the cache."""
         if append_mode not in APPEND_MODES:
             raise ValueError(f"append_mode must be one of {APPEND_MODES}")
+        if chunk_streams not in (1, 2):
+            raise ValueError("chunk_streams must be 1 or 2")
+        if chunk_streams == 2 and append_mode != "overlap":
+            raise ValueError("chunk_streams = 2 needs append_mode 'overlap'")
         self.w = w
         self.append_mode = append_mode
+        self.chunk_streams = chunk_streams
         self.device = torch.device(device)
         self.mode = w.mode if mode is None else mode
         self.fixed_bounds = None if bounds is None else [list(b) for b in bounds]
@@ -101,6 +116,10 @@ class ChunkedPrefill:
                                                                  w.head_dim))
             if need > 0:
                 self.workspace = torch.empty((need,), device=self.device, dtype=torch.uint8)
+        # the second compute stream's own split-KV scratch
+        self.workspace2 = None
+        if chunk_streams == 2 and self.workspace is not None:
+            self.workspace2 = torch.empty_like(self.workspace)
 
     def partition(self):
         """Chunk boundaries of every request (host call into the library)."""
@@ -130,7 +149,8 @@ class ChunkedPrefill:
         return self.lse.view(self.w.n_q_heads, self.w.total_tokens)
 
     # -- execution ----------------------------------------------------------------
-    def run_step(self, q, k, v, i, stream=None, events=None, ready=None, attention_only=False):
+    def run_step(self, q, k, v, i, stream=None, events=None, ready=None, attention_only=False,
+                 workspace=None):
         """Step ``i`` of ``steps()`` (one chunk index of every request that has
         it), as ``append_mode`` says.  ``ready`` is the event after which step
         i's chunks are in the cache (overlap mode, from ``launch_appends``);
@@ -139,11 +159,13 @@ class ChunkedPrefill:
         an optional triple of CUDA events recorded before the step's own
         appends, before the attention launch, and after it.  With MOCAP_NVTX=1
         in the environment each step is an NVTX range ("mocap chunk <index>")
-        for timeline profilers."""
+        for timeline profilers.  ``workspace`` replaces the split-KV scratch
+        (default: the prefill's own)."""
         if os.environ.get("MOCAP_NVTX", "0") != "0":
             with torch.cuda.nvtx.range(f"mocap chunk {i}"):
-                return self._run_step(q, k, v, i, stream, events, ready, attention_only)
-        return self._run_step(q, k, v, i, stream, events, ready, attention_only)
+                return self._run_step(q, k, v, i, stream, events, ready, attention_only,
+                                      workspace)
+        return self._run_step(q, k, v, i, stream, events, ready, attention_only, workspace)
 
     def _append_rows(self, k, v, r, c):
         """(K rows, V rows, destination cache row) of chunk c of request r."""
@@ -175,8 +197,10 @@ class ChunkedPrefill:
                 ready.append(ev)
         return ready, side
 
-    def _run_step(self, q, k, v, i, stream=None, events=None, ready=None, attention_only=False):
+    def _run_step(self, q, k, v, i, stream=None, events=None, ready=None, attention_only=False,
+                  workspace=None):
         w = self.w
+        workspace = self.workspace if workspace is None else workspace
         mode = self.append_mode
         steps = self.steps()
         step = steps[i]
@@ -201,10 +225,10 @@ class ChunkedPrefill:
             if nxt:
                 mocap_chunk_attn_append(q[b0:b1], self.k_cache, self.v_cache, b0,
                                         self.out[b0:b1], self.chunk_lse(c), w.scale, nxt,
-                                        workspace=self.workspace, stream=stream)
+                                        workspace=workspace, stream=stream)
             else:
                 mocap_chunk_attn(q[b0:b1], self.k_cache, self.v_cache, b0, self.out[b0:b1],
-                                 self.chunk_lse(c), w.scale, workspace=self.workspace,
+                                 self.chunk_lse(c), w.scale, workspace=workspace,
                                  stream=stream)
         else:
             items = []
@@ -214,10 +238,10 @@ class ChunkedPrefill:
             if nxt:
                 mocap_chunk_attn_varlen_append(q, self.k_cache, self.v_cache, items, self.out,
                                                self.lse_packed(), w.scale, nxt,
-                                               workspace=self.workspace, stream=stream)
+                                               workspace=workspace, stream=stream)
             else:
                 mocap_chunk_attn_varlen(q, self.k_cache, self.v_cache, items, self.out,
-                                        self.lse_packed(), w.scale, workspace=self.workspace,
+                                        self.lse_packed(), w.scale, workspace=workspace,
                                         stream=stream)
         if events is not None:
             events[2].record(stream)
@@ -231,13 +255,30 @@ class ChunkedPrefill:
         ready, side = [None] * n, None
         if self.append_mode == "overlap" and n > 1:
             ready, side = self.launch_appends(k, v, main, landed)
-        for i in range(n):
+        second = None
+        if self.chunk_streams == 2 and n > 1:
+            # step 0's chunks go to the cache first, on the caller's stream;
+            # the second stream starts after them (and after earlier work)
             if landed is not None:
-                main.wait_event(landed[i])
+                main.wait_event(landed[0])
+            for r, c in self.steps()[0]:
+                kr, vr, dst = self._append_rows(k, v, r, c)
+                mocap_kv_append(kr, vr, self.k_cache, self.v_cache, dst, stream=main)
+            ready[0] = torch.cuda.Event()
+            ready[0].record(main)
+            second = torch.cuda.Stream(self.device)
+            second.wait_stream(main)
+        for i in range(n):
+            st, ws = (second, self.workspace2) if (second is not None and i % 2) else (main, None)
+            if landed is not None:
+                st.wait_event(landed[i])
                 if self.append_mode == "fused" and i + 1 < n:
-                    main.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
-            self.run_step(q, k, v, i, stream, None if chunk_events is None else chunk_events[i],
-                          ready[i])
+                    st.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
+            with torch.cuda.stream(st):
+                self.run_step(q, k, v, i, st, None if chunk_events is None else chunk_events[i],
+                              ready[i], workspace=ws)
+        if second is not None:
+            main.wait_stream(second)
         if side is not None:
             main.wait_stream(side)
 

@@ -276,3 +276,43 @@ def test_fused_launch_after_expired_wait_does_nothing(m):
     assert m.mocap_last_device_status() == m.MOCAP_OK
     assert torch.equal(kc[400:600], ks) and torch.equal(vc[400:600], vs)
     assert not torch.isnan(out.float()).any()
+
+
+@pytest.mark.parametrize("index", [1, 2, 3, 5])
+def test_two_chunk_streams_equal_one(m, index):
+    """Attention launches alternating between two compute streams (each with
+    its own split-KV scratch; appends on a third) give bitwise the results
+    of one stream, eager and replayed from a CUDA graph."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(index)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    p1 = ChunkedPrefill(w, dev)
+    p1.run(q, k, v)
+    p2 = ChunkedPrefill(w, dev, chunk_streams=2)
+    for _ in range(2):
+        for t in (p2.out, p2.lse, p2.k_cache, p2.v_cache):
+            t.fill_(float("nan"))
+        p2.run(q, k, v)
+        torch.cuda.synchronize()
+        assert m.mocap_last_device_status() == 0
+        assert torch.equal(p2.k_cache, k) and torch.equal(p2.v_cache, v)
+        assert torch.equal(p2.out, p1.out) and torch.equal(p2.lse, p1.lse)
+    graph = p2.capture(q, k, v)
+    for t in (p2.out, p2.lse, p2.k_cache, p2.v_cache):
+        t.fill_(float("nan"))
+    graph.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(p2.k_cache, k) and torch.equal(p2.v_cache, v)
+    assert torch.equal(p2.out, p1.out) and torch.equal(p2.lse, p1.lse)
+    del graph
+
+
+def test_two_chunk_streams_need_overlapped_appends():
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    for mode in ("serial", "fused"):
+        with pytest.raises(ValueError):
+            ChunkedPrefill(workloads.get(1), torch.device("cuda"), append_mode=mode,
+                           chunk_streams=2)
