@@ -55,7 +55,7 @@ class ChunkedPrefill:
 
     def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True,
                  bounds: Optional[List[List[int]]] = None, append_mode: str = "overlap",
-                 chunk_streams: int = 1):
+                 chunk_streams: Optional[int] = None):
         """``bounds`` (one boundary list per request) replaces the workload's
         partition rule, e.g. with the Algorithm 1 stage-1 DP's split.
 
@@ -70,7 +70,8 @@ class ChunkedPrefill:
                      attention CTAs), and step i's attention waits for its
                      own chunks' event only.
 
-        ``chunk_streams`` = 2 issues the steps' attention launches alternately
+        ``chunk_streams`` = 2 (the default with overlapped appends, else 1)
+        issues the steps' attention launches alternately
         on the caller's stream and a second compute stream (``run`` only):
         step i + 1 reads no output of step i, only K/V rows already appended,
         so its CTAs may take SMs that step i's last wave leaves idle.  Each
@@ -80,6 +81,8 @@ class ChunkedPrefill:
         says its rows (and all earlier rows) are in the cache."""
         if append_mode not in APPEND_MODES:
             raise ValueError(f"append_mode must be one of {APPEND_MODES}")
+        if chunk_streams is None:
+            chunk_streams = 2 if append_mode == "overlap" else 1
         if chunk_streams not in (1, 2):
             raise ValueError("chunk_streams must be 1 or 2")
         if chunk_streams == 2 and append_mode != "overlap":
@@ -320,13 +323,26 @@ class ChunkedPrefill:
         ready, side = [None] * n, None
         if self.append_mode == "overlap" and n > 1:
             ready, side = self.launch_appends(k, v, compute, landed)
+        second = None
+        if self.chunk_streams == 2 and n > 1:
+            # as in run: step 0's chunks first, then two compute streams
+            compute.wait_event(landed[0])
+            for r, c in steps[0]:
+                kr, vr, dst = self._append_rows(k, v, r, c)
+                mocap_kv_append(kr, vr, self.k_cache, self.v_cache, dst, stream=compute)
+            ready[0] = torch.cuda.Event()
+            ready[0].record(compute)
+            second = torch.cuda.Stream(self.device)
+            second.wait_stream(compute)
         for i, step in enumerate(steps):
-            compute.wait_event(landed[i])
+            st, ws = (second, self.workspace2) if (second is not None and i % 2) else (compute, None)
+            st.wait_event(landed[i])
             if self.append_mode == "fused" and i + 1 < n:
-                compute.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
-            self.run_step(q, k, v, i, compute, ready=ready[i])
+                st.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
+            with torch.cuda.stream(st):
+                self.run_step(q, k, v, i, st, ready=ready[i], workspace=ws)
             done = torch.cuda.Event()
-            done.record(compute)
+            done.record(st)
             d2h.wait_event(done)
             with torch.cuda.stream(d2h):
                 for r, c in step:
@@ -335,6 +351,8 @@ class ChunkedPrefill:
                     if self.single:
                         host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
                                                         non_blocking=True)
+        if second is not None:
+            compute.wait_stream(second)
         if side is not None:
             compute.wait_stream(side)
 

@@ -293,7 +293,7 @@ def test_fused_append_argument_checks(lib):
     def call(apps, prefix=100, length=50, cap=1000, n=None):
         arr = (AppendItem * max(1, len(apps)))(*[AppendItem(*a) for a in apps])
         return f(FAKE, FAKE, FAKE, prefix, length, 8, 2, 128, 0.1, FAKE, FAKE, None, 0,
-                 arr if apps or n else None, len(apps) if n is None else n, cap, None)
+                 arr if apps else None, len(apps) if n is None else n, cap, None)
 
     assert call([(FAKE, FAKE, 149, 10)]) == 1            # overlaps the chunk's own rows
     assert call([(FAKE, FAKE, 0, 10)]) == 1              # overlaps the prefix
@@ -304,7 +304,7 @@ def test_fused_append_argument_checks(lib):
     assert call([(None, FAKE, 200, 10)]) == 1
     assert call([(FAKE, FAKE, 200, 10), (FAKE, FAKE, 205, 10)]) == 1  # appends overlap
     assert call([(FAKE, FAKE, 200, 10)] * 65) == 1       # too many
-    assert call([], n=3) == 1                            # count without an array
+    assert call([], n=3) == 1                            # a count with a null array
     assert call([(FAKE, FAKE, 200, 10)], cap=120) == 1   # cache shorter than prefix + len
     g = lib.mocap_chunk_attn_varlen_append
     items = (VarlenItem * 2)(VarlenItem(0, 0, 0, 10), VarlenItem(10, 500, 20, 10))

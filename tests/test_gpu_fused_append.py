@@ -175,7 +175,7 @@ def test_append_modes_equal_serial_pipeline(m, index, mode):
     q, k, v = workloads.make_qkv(w, dev)
     pu = ChunkedPrefill(w, dev, append_mode="serial")
     pu.run(q, k, v)
-    pf = ChunkedPrefill(w, dev, append_mode=mode)
+    pf = ChunkedPrefill(w, dev, append_mode=mode, chunk_streams=1)
     for t in (pf.out, pf.lse, pf.k_cache, pf.v_cache):
         t.fill_(float("nan"))
     pf.run(q, k, v)
@@ -288,9 +288,10 @@ def test_two_chunk_streams_equal_one(m, index):
     w = workloads.get(index)
     dev = torch.device("cuda")
     q, k, v = workloads.make_qkv(w, dev)
-    p1 = ChunkedPrefill(w, dev)
+    p1 = ChunkedPrefill(w, dev, chunk_streams=1)
     p1.run(q, k, v)
     p2 = ChunkedPrefill(w, dev, chunk_streams=2)
+    assert ChunkedPrefill(w, dev).chunk_streams == 2  # the default with overlapped appends
     for _ in range(2):
         for t in (p2.out, p2.lse, p2.k_cache, p2.v_cache):
             t.fill_(float("nan"))
