@@ -297,7 +297,9 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     // the item's rows start at q_row of the packed out / lse (0 for a
     // single-chunk call)
     const int64_t len = items[0].len, q_row = items[0].q_row;
-    const dim3 grid(static_cast<unsigned>(len), static_cast<unsigned>((sh.n_q_heads + 7) / 8));
+    const dim3 grid(static_cast<unsigned>(len),
+                    static_cast<unsigned>((sh.n_q_heads + kCombineHeadsPerBlock - 1) /
+                                          kCombineHeadsPerBlock));
     attn_combine_kernel<D><<<grid, 256, 0, stream>>>(
         prm.o_part, prm.lse_part, sp.splits, len, sh.n_q_heads,
         prm.out + q_row * sh.n_q_heads * D, lse + q_row, lse_stride, status);
@@ -366,7 +368,8 @@ mocap::SplitPlan plan_for(int64_t prefix, int64_t len, int32_t n_q_heads, int32_
   if (mocap::check_shape(sh, 1.0f) != MOCAP_OK || prefix < 0 || len <= 0 ||
       prefix > mocap::kMaxRows - len)
     return mocap::SplitPlan();
-  if (n_q_heads > 8 * 65535) return mocap::SplitPlan();  // the combine's grid has y <= 65535
+  if (n_q_heads > mocap::kCombineHeadsPerBlock * 65535)  // the combine's grid has y <= 65535
+    return mocap::SplitPlan();
   int splits =
       mocap::choose_splits(prefix, len, n_q_heads, n_kv_heads, head_dim, mocap::device_sm_count());
   // MOCAP_SPLIT_KV: 0 never splits; 1..4 forces that count (tests, tuning),
