@@ -18,7 +18,7 @@ namespace {
 // do not depend on the weights), so the DRAM round trips overlap.  Like the
 // attention launch before it, it does nothing once a bounded wait has
 // expired (the status word is set), so the outputs keep their contents.
-constexpr int kCombineHeadsPerWarp = 1;
+constexpr int kCombineHeadsPerWarp = 2;
 constexpr int kCombineHeadsPerBlock = 8 * kCombineHeadsPerWarp;
 
 template <int D>
