@@ -300,7 +300,16 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     const dim3 grid(static_cast<unsigned>(len),
                     static_cast<unsigned>((sh.n_q_heads + kCombineHeadsPerBlock - 1) /
                                           kCombineHeadsPerBlock));
-    attn_combine_kernel<D><<<grid, 256, 0, stream>>>(
+    static bool combine_done[64] = {};  // shared-memory limit set, per device
+    if (!combine_done[dev]) {
+      if (cudaFuncSetAttribute(attn_combine_kernel<D>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(combine_smem_bytes<D>(kMaxSplits))) !=
+          cudaSuccess)
+        return MOCAP_ECUDA;
+      combine_done[dev] = true;
+    }
+    attn_combine_kernel<D><<<grid, kCombineThreads, combine_smem_bytes<D>(sp.splits), stream>>>(
         prm.o_part, prm.lse_part, sp.splits, len, sh.n_q_heads,
         prm.out + q_row * sh.n_q_heads * D, lse + q_row, lse_stride, status);
     if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
