@@ -201,3 +201,126 @@ def dp_objective(bounds: List[int], granularity: int, num_stages: int,
     costs = [evaluate_chunk(units[i + 1] - units[i], units[i], model, gemm_weight)
              for i in range(len(units) - 1)]
     return sum(costs) + (num_stages - 1) * max(costs)
+
+
+# ---------------------------------------------------------------------------
+# Algorithm 1, stage 1 with EvaluateChunk as a compute-latency model of the
+# chunk attention kernel (Sec. 4.2: "EvaluateChunk returns the compute
+# latency t").  The model, in integer picoseconds so that it is exact:
+#   * a chunk of `length` rows at `prefix` has ceil(length / 128) query row
+#     blocks; row block qb sees keys up to min(prefix + 128 (qb + 1),
+#     prefix + length), i.e. tiles(qb) = ceil(that / 128) key tiles of 128;
+#   * each row block is Hkv * ceil((Hq / Hkv) / 2) CTAs (two query heads per
+#     CTA), each split into `splits` contiguous key ranges of
+#     floor((j + 1) tiles / splits) - floor(j tiles / splits) tiles;
+#   * a CTA costs CTA_PS + TILE_PS * (d / 128) per tile; CTAs are taken
+#     heaviest row block first and each goes to a least-loaded SM of `sms`
+#     (list scheduling); the chunk's time is the largest SM load;
+#   * with splits > 1 the merge adds COMBINE_FIXED_PS + (bytes moved) / 5 ps
+#     (bytes = length Hq (splits (4 d + 4) + 2 d + 4)), and the chunk takes the
+#     split count 1..4 with the smallest time (more than one only when the
+#     chunk has fewer than 8 sms CTAs, and at most the first row block's
+#     tile count);
+# the constants are the ones the library's split planner uses.
+
+TILE_PS = 1400000
+CTA_PS = 4000000
+COMBINE_FIXED_PS = 3000000
+MAX_SPLITS = 4
+
+
+def chunk_latency_ps(prefix: int, length: int, n_q_heads: int, n_kv_heads: int, head_dim: int,
+                     sms: int, splits: int) -> int:
+    """Modelled time of one chunk's attention launch with `splits` key
+    ranges (list scheduling of its CTAs over `sms` SMs), picoseconds."""
+    import heapq
+    group = n_q_heads // n_kv_heads
+    per_block = n_kv_heads * ((group + 1) // 2)
+    tile_ps = TILE_PS * head_dim // 128
+    q_blocks = (length + 127) // 128
+    loads = [0] * sms
+    for qb in range(q_blocks - 1, -1, -1):
+        kv_end = min(prefix + 128 * (qb + 1), prefix + length)
+        tiles = (kv_end + 127) // 128
+        for _ in range(per_block):
+            for j in range(splits):
+                nk = (j + 1) * tiles // splits - j * tiles // splits
+                least = heapq.heappop(loads)
+                heapq.heappush(loads, least + CTA_PS + tile_ps * nk)
+    t = max(loads)
+    if splits > 1:
+        moved = length * n_q_heads * (splits * (4 * head_dim + 4) + 2 * head_dim + 4)
+        t += COMBINE_FIXED_PS + moved // 5
+    return t
+
+
+def chunk_latency_best_ps(prefix: int, length: int, n_q_heads: int, n_kv_heads: int,
+                          head_dim: int, sms: int) -> int:
+    """The model's time with the split count it would choose (see above)."""
+    group = n_q_heads // n_kv_heads
+    ctas = ((length + 127) // 128) * n_kv_heads * ((group + 1) // 2)
+    best = chunk_latency_ps(prefix, length, n_q_heads, n_kv_heads, head_dim, sms, 1)
+    if ctas >= 8 * sms:
+        return best
+    first_tiles = (min(prefix + 128, prefix + length) + 127) // 128
+    for sp in range(2, min(MAX_SPLITS, first_tiles) + 1):
+        best = min(best, chunk_latency_ps(prefix, length, n_q_heads, n_kv_heads, head_dim, sms,
+                                          sp))
+    return best
+
+
+def dp_latency_boundaries(seq_len: int, num_chunks: int, num_stages: int, n_q_heads: int,
+                          n_kv_heads: int, head_dim: int, sms: int, window: int) -> List[int]:
+    """Algorithm 1's stage-1 DP (loops and strict-improvement rule as in
+    dp_tables) with EvaluateChunk = chunk_latency_best_ps, over 128-row units,
+    each interior boundary restricted to `window` units either side of the
+    closed-form split's (``boundaries(seq_len, num_chunks, 128)``).  The last
+    chunk ends at seq_len (absorbing seq_len % 128)."""
+    if window < 0:
+        raise ValueError("window >= 0 required")
+    g = 128
+    units = _check(seq_len, num_chunks, g)
+    M, U, N = num_chunks, units, num_stages
+    if N < 1:
+        raise ValueError("num_stages >= 1 required")
+    closed = [b // g for b in boundaries(seq_len, num_chunks, g)]
+    closed[-1] = U
+
+    def allowed(m):  # unit positions boundary m may take
+        if m == 0:
+            return [0]
+        if m == M:
+            return [U]
+        lo = max(m, closed[m] - window)
+        hi = min(U - (M - m), closed[m] + window)
+        return list(range(lo, hi + 1))
+
+    def evaluate(s, k):
+        length = seq_len - g * s if s + k == U else g * k
+        return chunk_latency_best_ps(g * s, length, n_q_heads, n_kv_heads, head_dim, sms)
+
+    t_max = {(M + 1, U): 0}
+    t_sum = {(M + 1, U): 0}
+    ss = {}
+    for m in range(M, 0, -1):
+        ends = set(allowed(m))
+        for s in sorted(allowed(m - 1), reverse=True):
+            for k in range(1, U - s - (M - m) + 1):
+                if s + k not in ends:
+                    continue
+                nxt = (m + 1, s + k)
+                if nxt not in t_max:
+                    continue
+                t = evaluate(s, k)
+                tmax_new = max(t_max[nxt], t)
+                tsum_new = t_sum[nxt] + t
+                cur = (m, s)
+                if cur not in t_max or \
+                        tsum_new + (N - 1) * tmax_new < t_sum[cur] + (N - 1) * t_max[cur]:
+                    t_max[cur], t_sum[cur], ss[cur] = tmax_new, tsum_new, k
+    out, s = [0], 0
+    for m in range(1, M + 1):
+        s += ss[(m, s)]
+        out.append(g * s)
+    out[-1] = seq_len
+    return out

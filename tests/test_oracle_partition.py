@@ -339,3 +339,89 @@ def test_dp_golden_rows_of_the_32k_shape():
     for s, m, g, n, model, gemm, b in rows:
         assert P.dp_boundaries(s, m, g, n, model, gemm) == b
         _check_invariants(b, s, m, g)
+
+
+# ---------------------------------------------------------------------------
+# Algorithm 1 stage 1 with EvaluateChunk = the kernel's compute-latency model.
+C, T = P.CTA_PS, P.TILE_PS
+
+
+def test_latency_model_hand_worked_cases():
+    # 2 SMs, 1 query head per KV head (one CTA per KV head and row block),
+    # 2 KV heads, 256 rows at prefix 0: row block 1 = 2 CTAs of 2 tiles, row
+    # block 0 = 2 CTAs of 1 tile; list scheduling puts one of each on each SM
+    assert P.chunk_latency_ps(0, 256, 2, 2, 128, 2, 1) == 2 * C + 3 * T
+    # 3 SMs: the third SM takes one 1-tile CTA, then the last one (least loaded)
+    assert P.chunk_latency_ps(0, 256, 2, 2, 128, 3, 1) == 2 * C + 2 * T
+    # d = 64 halves the tile cost
+    assert P.chunk_latency_ps(0, 256, 2, 2, 64, 2, 1) == 2 * C + 3 * (T // 2)
+    # two splits of a one-block chunk with two key tiles: one tile each on two
+    # SMs, plus the merge of 128 rows x 1 head: 3 us + bytes / 5 ps
+    moved = 128 * 1 * (2 * (4 * 128 + 4) + 2 * 128 + 4)
+    assert P.chunk_latency_ps(128, 128, 1, 1, 128, 2, 2) == C + T + P.COMBINE_FIXED_PS + moved // 5
+    # a ragged chunk: 130 rows at prefix 0 = row blocks of 1 and 2 tiles
+    assert P.chunk_latency_ps(0, 130, 1, 1, 128, 1, 1) == 2 * C + 3 * T
+    # four query heads per KV head = two CTAs per KV head and row block
+    assert P.chunk_latency_ps(0, 128, 4, 1, 128, 1, 1) == 2 * (C + T)
+
+
+def test_latency_model_bounds():
+    import random
+    rnd = random.Random(4)
+    for _ in range(200):
+        prefix = rnd.randint(0, 3000)
+        length = rnd.randint(1, 2000)
+        hkv = rnd.choice([1, 2, 4])
+        hq = hkv * rnd.choice([1, 2, 4, 8])
+        sms = rnd.choice([1, 3, 8, 152])
+        t = P.chunk_latency_ps(prefix, length, hq, hkv, 128, sms, 1)
+        q_blocks = (length + 127) // 128
+        per_block = hkv * ((hq // hkv + 1) // 2)
+        jobs = []
+        for qb in range(q_blocks):
+            tiles = (min(prefix + 128 * (qb + 1), prefix + length) + 127) // 128
+            jobs += [C + T * tiles] * per_block
+        assert t >= max(jobs) and t * sms >= sum(jobs)
+        assert t <= sum(jobs) // sms + max(jobs)            # list-scheduling bound
+        best = P.chunk_latency_best_ps(prefix, length, hq, hkv, 128, sms)
+        assert best <= t
+
+
+def test_latency_dp_window_zero_is_the_closed_form():
+    for s, m in [(32768, 16), (8192, 8), (5000, 5)]:
+        assert P.dp_latency_boundaries(s, m, 16, 32, 8, 128, 152, 0) == P.boundaries(s, m, 128)
+
+
+def _lat_costs(sizes, hq, hkv, sms):
+    s, out = 0, []
+    for k in sizes:
+        out.append(P.chunk_latency_best_ps(128 * s, 128 * k, hq, hkv, 128, sms))
+        s += k
+    return out
+
+
+@pytest.mark.parametrize("hq,hkv,sms", [(2, 1, 3), (8, 2, 5), (4, 4, 2)])
+def test_latency_dp_reaches_the_brute_force_optimum(hq, hkv, sms):
+    # windows wider than the prompt: the DP ranges over every split, so with
+    # N = 1 it minimises the total and with (N - 1) above any total it reaches
+    # the minimax chunk latency (the objective's two extremes)
+    for units in range(2, 10):
+        for m in range(1, min(units, 4) + 1):
+            comps = list(_compositions(units, m))
+            b1 = P.dp_latency_boundaries(128 * units, m, 1, hq, hkv, 128, sms, units)
+            got = _lat_costs([(b1[i + 1] - b1[i]) // 128 for i in range(m)], hq, hkv, sms)
+            assert sum(got) == min(sum(_lat_costs(c, hq, hkv, sms)) for c in comps)
+            bn = P.dp_latency_boundaries(128 * units, m, 10 ** 12, hq, hkv, 128, sms, units)
+            got = _lat_costs([(bn[i + 1] - bn[i]) // 128 for i in range(m)], hq, hkv, sms)
+            assert max(got) == min(max(_lat_costs(c, hq, hkv, sms)) for c in comps)
+
+
+def test_latency_dp_stays_in_its_window_and_lowers_the_modelled_maximum():
+    s, m, w = 32768, 16, 6
+    closed = P.boundaries(s, m, 128)
+    dp = P.dp_latency_boundaries(s, m, 10 ** 12, 32, 8, 128, 152, w)
+    _check_invariants(dp, s, m, 128)
+    assert all(abs(a - b) <= 128 * w for a, b in zip(dp, closed))
+    lat = lambda b: [P.chunk_latency_best_ps(b[i], b[i + 1] - b[i], 32, 8, 128, 152)
+                     for i in range(m)]
+    assert max(lat(dp)) <= max(lat(closed))
