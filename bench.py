@@ -575,6 +575,15 @@ def ours_arm(args, rank, world, local):
             line[key] = measure_uniform(w, q, k, v, dev, stream, bounds=[b])
             line[key]["first_chunk_rows"] = b[1] - b[0]
             line[key]["last_chunk_rows"] = b[-1] - b[-2]
+        # the same DP with EvaluateChunk = the kernel's latency model on this
+        # GPU's SM count, boundaries within 8 units of the closed form
+        from paper_2606_22968_gb300.pipeline import latency_balanced_bounds
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        b = latency_balanced_bounds(s_len, n_chunks, w.n_q_heads, w.n_kv_heads, w.head_dim, sms)
+        line["dp_latency_boundaries"] = measure_uniform(w, q, k, v, dev, stream, bounds=[b])
+        line["dp_latency_boundaries"].update({"sms": sms, "window_units": 8,
+                                              "first_chunk_rows": b[1] - b[0],
+                                              "last_chunk_rows": b[-1] - b[-2]})
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         times, flops, done, threads = run_oracle_sample(
             q, k, v, pf.bounds[0], w.scale, 1, args.cpu_rows_per_chunk, 20.0)

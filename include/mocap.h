@@ -12,6 +12,7 @@
  *
  *   mocap_lbcp_partition      chunk boundaries (host, exact integers)
  *   mocap_lbcp_partition_dp   boundaries from Algorithm 1's stage-1 DP (host)
+ *   mocap_lbcp_partition_dp_latency  the same DP with the kernel's latency model
  *   mocap_lbcp_gemm_weight    the DP's GEMM-term weight from measured rates (host)
  *   mocap_kv_append           chunk K/V -> contiguous bf16 KV cache (device)
  *   mocap_kv_append_overlap   the same, sized to run beside an attention launch
@@ -125,6 +126,45 @@ mocap_status mocap_lbcp_partition_dp(int64_t seq_len, int32_t num_chunks,
                                      int32_t granularity, int32_t num_stages,
                                      mocap_cost_model model, int64_t gemm_weight,
                                      int64_t *boundaries);
+
+/*
+ * mocap_lbcp_partition_dp_latency -- Algorithm 1's stage-1 DP (Sec. 4.2) with
+ * EvaluateChunk as the compute latency of this library's chunk attention
+ * kernel on a GPU with `num_sms` SMs, in 128-row units.
+ *
+ * The latency model (integer picoseconds, so the result is bit-exact on
+ * every platform): the chunk's CTAs -- n_kv_heads * ceil((n_q_heads /
+ * n_kv_heads) / 2) per 128-row query block, block qb seeing
+ * ceil(min(prefix + 128 (qb + 1), prefix + len) / 128) key tiles -- are
+ * list-scheduled, heaviest block first, each onto a least-loaded SM; a CTA
+ * costs 4 us plus 1.4 us * (head_dim / 128) per key tile it covers; with
+ * the key range split in s = 2..4 parts (considered only below 8 CTAs per SM)
+ * each CTA covers floor((j+1) T / s) - floor(j T / s) tiles and the merge
+ * adds 3 us + (bytes moved) / (5 bytes per ps); the chunk takes its fastest
+ * split.  These are the costs the split planner of mocap_chunk_attn uses.
+ * Unlike the causal pair count, the model sees how a chunk's CTAs fill the
+ * SMs' waves (measured on GB300: it tracks per-chunk attention latency with
+ * correlation 0.92, the pair count 0.59).
+ *
+ * Loops and tie rule as mocap_lbcp_partition_dp (m down, s down, k up,
+ * strict improvement of t_sum + (N - 1) t_max), with each interior boundary
+ * limited to `window` units either side of mocap_lbcp_partition's
+ * closed-form LBCP boundary (window 0 returns that split).  The last chunk
+ * absorbs seq_len % 128.
+ *
+ *   num_stages   N >= 1;  n_q_heads a multiple of n_kv_heads (<= 4096)
+ *   head_dim     64 or 128 (else MOCAP_EUNSUPPORTED);  num_sms 1 .. 4096
+ *   window       >= 0 units of 128 rows
+ *   boundaries   HOST array of num_chunks + 1 int64, written on success
+ * MOCAP_EINVAL for bad arguments (seq_len < 2^31, num_chunks * 128 <=
+ * seq_len); MOCAP_EUNSUPPORTED when the windows' chunk evaluations would be
+ * too much host work (use a smaller window).  Pure host code.
+ */
+mocap_status mocap_lbcp_partition_dp_latency(int64_t seq_len, int32_t num_chunks,
+                                             int32_t num_stages, int32_t n_q_heads,
+                                             int32_t n_kv_heads, int32_t head_dim,
+                                             int32_t num_sms, int32_t window,
+                                             int64_t *boundaries);
 
 /*
  * mocap_lbcp_gemm_weight -- the gemm_weight argument of

@@ -76,6 +76,20 @@ def mocap_lbcp_partition_dp(seq_len: int, num_chunks: int, granularity: int = 12
     return list(out)
 
 
+def mocap_lbcp_partition_dp_latency(seq_len: int, num_chunks: int, n_q_heads: int,
+                                    n_kv_heads: int, head_dim: int, num_sms: int,
+                                    num_stages: int = 16, window: int = 8) -> List[int]:
+    """Boundaries from Algorithm 1's stage-1 DP with the attention kernel's
+    compute-latency model as EvaluateChunk (128-row units, each boundary
+    within `window` units of the closed-form split)."""
+    out = (ctypes.c_int64 * (num_chunks + 1))()
+    _check(_lib.load().mocap_lbcp_partition_dp_latency(seq_len, num_chunks, num_stages,
+                                                       n_q_heads, n_kv_heads, head_dim, num_sms,
+                                                       window, out),
+           "mocap_lbcp_partition_dp_latency")
+    return list(out)
+
+
 def mocap_lbcp_gemm_weight(attn_s_per_pair: float, gemm_s_per_row: float,
                            granularity: int = 128) -> int:
     """The stage-1 DP's GEMM weight for chunk stages that cost

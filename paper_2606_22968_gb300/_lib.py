@@ -26,6 +26,8 @@ SIGNATURES = {
     "mocap_lbcp_partition": (c_i32, [c_i64, c_i32, c_i32, c_i32, ctypes.POINTER(c_i64)]),
     "mocap_lbcp_partition_dp": (c_i32, [c_i64, c_i32, c_i32, c_i32, c_i32, c_i64,
                                         ctypes.POINTER(c_i64)]),
+    "mocap_lbcp_partition_dp_latency": (c_i32, [c_i64, c_i32, c_i32, c_i32, c_i32, c_i32, c_i32,
+                                                c_i32, ctypes.POINTER(c_i64)]),
     "mocap_lbcp_gemm_weight": (c_i32, [ctypes.c_double, ctypes.c_double, c_i32,
                                        ctypes.POINTER(c_i64)]),
     "mocap_kv_append": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_i64, c_i32, c_i32, c_vp]),

@@ -10,7 +10,10 @@
 //     = (q + 1) / 2 with q = isqrt(floor(4 i U^2 / M)),
 //   b_i = min(max(g n_i, b_{i-1} + g), g (U - (M - i))),  b_0 = 0, b_M = S.
 // Uniform mode: n_i = round_half_up(i U / M) = floor((2 i U + M) / (2 M)).
+#include <algorithm>
 #include <cstdint>
+#include <functional>
+#include <unordered_map>
 #include <vector>
 
 #include "internal.h"
@@ -150,5 +153,167 @@ extern "C" mocap_status mocap_lbcp_gemm_weight(double attn_s_per_pair, double ge
   const double w = 2.0 * gemm_s_per_row / (static_cast<double>(granularity) * attn_s_per_pair);
   if (!(w <= static_cast<double>(int64_t(1) << 40))) return MOCAP_EINVAL;  // inf, too large
   *weight = static_cast<int64_t>(w + 0.5);  // w >= 0: round half up
+  return MOCAP_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Stage 1 of Algorithm 1 with EvaluateChunk as a compute-latency model of the
+// chunk attention kernel (Sec. 4.2: EvaluateChunk returns the compute
+// latency).  The model, in integer picoseconds so that every platform gets
+// the same bits: a chunk's CTAs (Hkv * ceil(group / 2) per 128-row block,
+// each covering split j of the block's key tiles) are list-scheduled,
+// heaviest row block first, each onto a least-loaded SM; a CTA costs
+// kCtaPs + kTilePs * (d / 128) per key tile; a split chunk adds the merge,
+// kCombineFixedPs + (bytes moved) / 5 ps.  The split count is the one of
+// 1..4 with the smallest time (more than one only below 8 CTAs per SM and at
+// most the first row block's tile count).  These are the split planner's
+// own costs.
+namespace {
+
+constexpr int64_t kTilePs = 1400000;
+constexpr int64_t kCtaPs = 4000000;
+constexpr int64_t kCombineFixedPs = 3000000;
+constexpr int kModelMaxSplits = 4;
+
+int64_t chunk_latency_ps(int64_t prefix, int64_t length, int64_t hq, int64_t hkv, int64_t d,
+                         int sms, int splits, std::vector<int64_t> &loads) {
+  const int64_t per_block = hkv * ((hq / hkv + 1) / 2);
+  const int64_t tile_ps = kTilePs * d / 128;
+  const int64_t q_blocks = (length + 127) / 128;
+  loads.assign(static_cast<size_t>(sms), 0);  // a min-heap (std::greater)
+  for (int64_t qb = q_blocks - 1; qb >= 0; --qb) {
+    const int64_t kv_end = std::min(prefix + 128 * (qb + 1), prefix + length);
+    const int64_t tiles = (kv_end + 127) / 128;
+    for (int64_t u = 0; u < per_block; ++u)
+      for (int j = 0; j < splits; ++j) {
+        const int64_t nk = (j + 1) * tiles / splits - j * tiles / splits;
+        std::pop_heap(loads.begin(), loads.end(), std::greater<int64_t>());
+        loads.back() += kCtaPs + tile_ps * nk;
+        std::push_heap(loads.begin(), loads.end(), std::greater<int64_t>());
+      }
+  }
+  int64_t t = *std::max_element(loads.begin(), loads.end());
+  if (splits > 1)
+    t += kCombineFixedPs + length * hq * (splits * (4 * d + 4) + 2 * d + 4) / 5;
+  return t;
+}
+
+int64_t chunk_latency_best_ps(int64_t prefix, int64_t length, int64_t hq, int64_t hkv, int64_t d,
+                              int sms, std::vector<int64_t> &loads) {
+  const int64_t ctas = ((length + 127) / 128) * hkv * ((hq / hkv + 1) / 2);
+  int64_t best = chunk_latency_ps(prefix, length, hq, hkv, d, sms, 1, loads);
+  if (ctas >= 8LL * sms) return best;
+  const int64_t first_tiles = (std::min(prefix + 128, prefix + length) + 127) / 128;
+  for (int sp = 2; sp <= kModelMaxSplits && sp <= first_tiles; ++sp)
+    best = std::min(best, chunk_latency_ps(prefix, length, hq, hkv, d, sms, sp, loads));
+  return best;
+}
+
+}  // namespace
+
+extern "C" mocap_status mocap_lbcp_partition_dp_latency(int64_t seq_len, int32_t num_chunks,
+                                                        int32_t num_stages, int32_t n_q_heads,
+                                                        int32_t n_kv_heads, int32_t head_dim,
+                                                        int32_t num_sms, int32_t window,
+                                                        int64_t *boundaries) {
+  constexpr int64_t g = 128;
+  if (boundaries == nullptr || seq_len <= 0 || seq_len >= (int64_t(1) << 31) ||
+      num_chunks < 1 || num_stages < 1 || window < 0)
+    return MOCAP_EINVAL;
+  if (n_q_heads < 1 || n_kv_heads < 1 || n_q_heads % n_kv_heads != 0 || n_q_heads > 4096)
+    return MOCAP_EINVAL;
+  if (head_dim != 64 && head_dim != 128) return MOCAP_EUNSUPPORTED;
+  if (num_sms < 1 || num_sms > 4096) return MOCAP_EINVAL;
+  if (static_cast<int64_t>(num_chunks) * g > seq_len) return MOCAP_EINVAL;
+  const int64_t U = seq_len / g;
+  const int64_t M = num_chunks;
+  const int64_t W = std::min<int64_t>(window, U);
+  // the closed-form split the windows are centred on
+  std::vector<int64_t> closed(static_cast<size_t>(M + 1));
+  const mocap_status cs = mocap_lbcp_partition(seq_len, num_chunks, static_cast<int32_t>(g),
+                                               MOCAP_PART_LBCP, closed.data());
+  if (cs != MOCAP_OK) return cs;
+  std::vector<int64_t> lo(static_cast<size_t>(M + 1)), hi(static_cast<size_t>(M + 1));
+  for (int64_t m = 0; m <= M; ++m) {
+    if (m == 0) {
+      lo[0] = hi[0] = 0;
+    } else if (m == M) {
+      lo[m] = hi[m] = U;
+    } else {
+      const int64_t c = closed[static_cast<size_t>(m)] / g;
+      lo[m] = std::max(m, c - W);
+      hi[m] = std::min(U - (M - m), c + W);
+    }
+  }
+  // host work: every (start, end) pair of neighbouring windows is one chunk
+  // evaluation of at most (2 W + U / M-ish) row blocks' CTAs
+  const int64_t per_block = n_kv_heads * ((n_q_heads / n_kv_heads + 1) / 2);
+  double work = 0.0;
+  for (int64_t m = 1; m <= M; ++m) {
+    const double pairs = static_cast<double>(hi[m - 1] - lo[m - 1] + 1) * (hi[m] - lo[m] + 1);
+    const double blocks = static_cast<double>(hi[m] - lo[m - 1] + 1);
+    work += pairs * blocks * per_block * kModelMaxSplits;
+  }
+  if (work > 4e9) return MOCAP_EUNSUPPORTED;  // use a smaller window
+
+  std::vector<int64_t> loads;
+  std::unordered_map<int64_t, int64_t> memo;
+  auto evaluate = [&](int64_t s, int64_t k) {
+    const int64_t key = s * (U + 1) + k;
+    const auto it = memo.find(key);
+    if (it != memo.end()) return it->second;
+    const int64_t length = s + k == U ? seq_len - g * s : g * k;
+    const int64_t t = chunk_latency_best_ps(g * s, length, n_q_heads, n_kv_heads, head_dim,
+                                            num_sms, loads);
+    memo.emplace(key, t);
+    return t;
+  };
+  // suffix states (m, s) for s in boundary m-1's window; row M+1 holds only
+  // the terminal (M+1, U)
+  struct State {
+    bool set = false;
+    int64_t t_max = 0, t_sum = 0, k = 0;
+  };
+  std::vector<std::vector<State>> st(static_cast<size_t>(M + 2));
+  for (int64_t m = 1; m <= M; ++m)
+    st[static_cast<size_t>(m)].resize(static_cast<size_t>(hi[m - 1] - lo[m - 1] + 1));
+  State terminal;  // (M + 1, U): t_max = t_sum = 0
+  terminal.set = true;
+  auto suffix = [&](int64_t m, int64_t s) -> const State * {  // state (m, s), s in window m-1
+    if (m == M + 1) return s == U ? &terminal : nullptr;
+    if (s < lo[m - 1] || s > hi[m - 1]) return nullptr;
+    const State &x = st[static_cast<size_t>(m)][static_cast<size_t>(s - lo[m - 1])];
+    return x.set ? &x : nullptr;
+  };
+  const __int128 nm1 = num_stages - 1;
+  for (int64_t m = M; m >= 1; --m) {
+    for (int64_t s = hi[m - 1]; s >= lo[m - 1]; --s) {
+      State &cur = st[static_cast<size_t>(m)][static_cast<size_t>(s - lo[m - 1])];
+      for (int64_t k = 1; k <= U - s - (M - m); ++k) {
+        if (s + k < lo[m] || s + k > hi[m]) continue;
+        const State *nxt = suffix(m + 1, s + k);
+        if (nxt == nullptr) continue;
+        const int64_t t = evaluate(s, k);
+        const int64_t tmax_new = std::max(nxt->t_max, t);
+        const int64_t tsum_new = nxt->t_sum + t;
+        if (!cur.set || static_cast<__int128>(tsum_new) + nm1 * tmax_new <
+                            static_cast<__int128>(cur.t_sum) + nm1 * cur.t_max) {
+          cur.t_max = tmax_new;
+          cur.t_sum = tsum_new;
+          cur.k = k;
+          cur.set = true;
+        }
+      }
+    }
+  }
+  const State *first = suffix(1, 0);
+  if (first == nullptr) return MOCAP_EINVAL;
+  boundaries[0] = 0;
+  int64_t pos = 0;
+  for (int64_t m = 1; m <= M; ++m) {
+    pos += suffix(m, pos)->k;
+    boundaries[m] = g * pos;
+  }
+  boundaries[M] = seq_len;
   return MOCAP_OK;
 }

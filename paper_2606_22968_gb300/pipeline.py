@@ -18,6 +18,7 @@ from . import (MOCAP_COST_CAUSAL, MOCAP_PART_LBCP, MOCAP_PART_UNIFORM, mocap_chu
                mocap_chunk_attn_append, mocap_chunk_attn_varlen, mocap_chunk_attn_varlen_append,
                mocap_chunk_attn_workspace_size, mocap_kv_append, mocap_kv_append_overlap,
                mocap_lbcp_gemm_weight, mocap_lbcp_partition, mocap_lbcp_partition_dp,
+               mocap_lbcp_partition_dp_latency,
                mocap_qkv_rope_append)
 from .workloads import GRANULARITY, Workload, request_offsets
 
@@ -41,6 +42,17 @@ def stage_balanced_bounds(seq_len: int, num_chunks: int, attn_s_per_pair: float,
 
 
 APPEND_MODES = ("serial", "fused", "overlap")
+
+
+def latency_balanced_bounds(seq_len: int, num_chunks: int, n_q_heads: int, n_kv_heads: int,
+                            head_dim: int, num_sms: int, num_stages: int = 16,
+                            window: int = 8) -> List[int]:
+    """Boundaries from stage 1 of Algorithm 1 (Sec. 4.2) with EvaluateChunk =
+    the attention kernel's compute-latency model on `num_sms` SMs, each
+    boundary within `window` 128-row units of the closed-form split
+    (mocap_lbcp_partition_dp_latency)."""
+    return mocap_lbcp_partition_dp_latency(seq_len, num_chunks, n_q_heads, n_kv_heads, head_dim,
+                                           num_sms, num_stages, window)
 
 
 class ChunkedPrefill:

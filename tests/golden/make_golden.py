@@ -7,7 +7,10 @@ Run from the repository root:  python tests/golden/make_golden.py
                             16-chunk and 131072-token / 32-chunk shapes
                             (N = 16 stages; causal cost, Eq. 1's cost, and
                             the causal cost with a GEMM weight of 90)
-The DP rows of the 131072-token shape take a few minutes of pure Python.
+  dp_latency_boundaries.txt the same DP with the attention kernel's latency
+                            model (N = 16, 152 SMs; 32/8 and 64/8 heads,
+                            d = 128; windows of 6 and 8 units)
+The DP rows of the 131072-token shape take several minutes of pure Python.
 """
 import os
 import sys
@@ -45,6 +48,13 @@ DP_CASES = [
 ]
 
 
+# (seq_len, chunks, stages, Hq, Hkv, d, SMs, window)
+DP_LATENCY_CASES = [
+    (32768, 16, 16, 32, 8, 128, 152, 6),
+    (131072, 32, 16, 64, 8, 128, 152, 8),
+]
+
+
 def main():
     here = os.path.dirname(os.path.abspath(__file__))
     with open(os.path.join(here, "partition_boundaries.txt"), "w") as f:
@@ -61,6 +71,14 @@ def main():
         for s, m, g, n, model, gemm in DP_CASES:
             b = P.dp_boundaries(s, m, g, n, model, gemm)
             f.write(f"{s} {m} {g} {n} {model} {gemm}: " + " ".join(str(x) for x in b) + "\n")
+            f.flush()
+    with open(os.path.join(here, "dp_latency_boundaries.txt"), "w") as f:
+        f.write("# seq_len chunks stages n_q_heads n_kv_heads head_dim sms window: b_0 .. b_M\n")
+        f.write("# written by tests/golden/make_golden.py from oracle/partition.py "
+                "(dp_latency_boundaries)\n")
+        for case in DP_LATENCY_CASES:
+            b = P.dp_latency_boundaries(*case)
+            f.write(" ".join(str(x) for x in case) + ": " + " ".join(str(x) for x in b) + "\n")
             f.flush()
 
 

@@ -39,3 +39,16 @@ def dp_boundary_rows():
             s, m, g, n, model, gemm = (int(x) for x in head.split())
             rows.append((s, m, g, n, model, gemm, [int(x) for x in tail.split()]))
     return rows
+
+
+def dp_latency_rows():
+    """Rows of dp_latency_boundaries.txt: ((seq_len, chunks, stages, Hq, Hkv,
+    d, sms, window), boundaries)."""
+    rows = []
+    with open(os.path.join(GOLDEN, "dp_latency_boundaries.txt")) as f:
+        for line in f:
+            if line.startswith("#") or not line.strip():
+                continue
+            head, tail = line.split(":", 1)
+            rows.append((tuple(int(x) for x in head.split()), [int(x) for x in tail.split()]))
+    return rows

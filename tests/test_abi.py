@@ -311,3 +311,50 @@ def test_fused_append_argument_checks(lib):
     arr = (AppendItem * 1)(AppendItem(FAKE, FAKE, 515, 4))  # inside item 1's rows [500, 530)
     assert g(FAKE, FAKE, FAKE, items, 2, 100, 1000, 8, 2, 128, 0.1, FAKE, FAKE, None, 0, arr, 1,
              None) == 1
+
+
+def test_dp_latency_bit_exact_vs_oracle(lib):
+    """Algorithm 1 stage 1 with the kernel's latency model: C++ against the
+    oracle on random small prompts (windows up to the whole prompt)."""
+    rnd = random.Random(23)
+    for _ in range(40):
+        units = rnd.randint(1, 40)
+        m = rnd.randint(1, min(units, 6))
+        s = units * 128 + rnd.choice([0, 0, 1, 77])
+        hkv = rnd.choice([1, 2, 8])
+        hq = hkv * rnd.choice([1, 2, 3, 4, 8])
+        d = rnd.choice([64, 128])
+        sms = rnd.choice([1, 5, 16, 152])
+        n = rnd.choice([1, 2, 16, 10 ** 6])
+        window = rnd.choice([0, 1, 3, units])
+        out = (ctypes.c_int64 * (m + 1))()
+        assert lib.mocap_lbcp_partition_dp_latency(s, m, n, hq, hkv, d, sms, window, out) == 0
+        assert list(out) == P.dp_latency_boundaries(s, m, n, hq, hkv, d, sms, window), \
+            (s, m, n, hq, hkv, d, sms, window)
+
+
+def test_dp_latency_golden_rows(lib):
+    """The workload shapes' rows the oracle wrote (tests/golden/make_golden.py)."""
+    from tests.golden_utils import dp_latency_rows
+    rows = dp_latency_rows()
+    assert {r[0][0] for r in rows} == {32768, 131072}
+    for (s, m, n, hq, hkv, d, sms, window), b in rows:
+        out = (ctypes.c_int64 * (m + 1))()
+        assert lib.mocap_lbcp_partition_dp_latency(s, m, n, hq, hkv, d, sms, window, out) == 0
+        assert list(out) == b
+
+
+def test_dp_latency_argument_checks(lib):
+    out = (ctypes.c_int64 * 40)()
+    f = lib.mocap_lbcp_partition_dp_latency
+    assert f(32768, 16, 16, 32, 8, 96, 152, 4, out) == 3       # head_dim
+    assert f(32768, 16, 16, 32, 6, 128, 152, 4, out) == 1      # Hq % Hkv
+    assert f(32768, 16, 0, 32, 8, 128, 152, 4, out) == 1       # stages
+    assert f(32768, 16, 16, 32, 8, 128, 0, 4, out) == 1        # SMs
+    assert f(32768, 16, 16, 32, 8, 128, 152, -1, out) == 1     # window
+    assert f(1024, 9, 16, 32, 8, 128, 152, 4, out) == 1        # M * 128 > S
+    assert f(1 << 31, 16, 16, 32, 8, 128, 152, 4, out) == 1    # S
+    assert f(32768, 16, 16, 32, 8, 128, 152, 4, None) == 1
+    assert f(1 << 30, 8, 16, 64, 8, 128, 152, 10 ** 6, out) == 3  # too much host work
+    assert f(32768, 16, 16, 32, 8, 128, 152, 0, out) == 0
+    assert list(out)[:17] == P.boundaries(32768, 16, 128)      # window 0: the closed form
