@@ -565,25 +565,30 @@ def ours_arm(args, rank, world, local):
     if not args.no_last_row:
         line["last_row"] = measure_last_row(args, m, w, pf, q, dev, stream, hbm)
     if pf.mode == workloads.MODE_LBCP and pf.single and not args.no_uniform:
-        line["uniform_boundaries"] = measure_uniform(w, q, k, v, dev, stream)
-        # Algorithm 1 stage 1 (the DP over 128-row units, N = 16 pipeline
-        # stages) with the causal cost c (p + c / 2) and with Eq. 1's c (p + c)
-        s_len, n_chunks = w.seq_lens[0], w.num_chunks[0]
-        for key, model in (("dp_causal_boundaries", m.MOCAP_COST_CAUSAL),
-                           ("dp_eq1_boundaries", m.MOCAP_COST_EQ1)):
-            b = m.mocap_lbcp_partition_dp(s_len, n_chunks, 128, 16, model, 0)
-            line[key] = measure_uniform(w, q, k, v, dev, stream, bounds=[b])
-            line[key]["first_chunk_rows"] = b[1] - b[0]
-            line[key]["last_chunk_rows"] = b[-1] - b[-2]
-        # the same DP with EvaluateChunk = the kernel's latency model on this
-        # GPU's SM count, boundaries within 8 units of the closed form
+        # The workload's closed-form LBCP split against uniform chunks and
+        # Algorithm 1's stage-1 DP (128-row units, N = 16 pipeline stages)
+        # with the causal cost c (p + c / 2), Eq. 1's c (p + c), and the
+        # kernel's latency model on this GPU's SM count (boundaries within 8
+        # units of the closed form); all timed interleaved from CUDA graphs.
         from paper_2606_22968_gb300.pipeline import latency_balanced_bounds
+        s_len, n_chunks = w.seq_lens[0], w.num_chunks[0]
         sms = torch.cuda.get_device_properties(dev).multi_processor_count
-        b = latency_balanced_bounds(s_len, n_chunks, w.n_q_heads, w.n_kv_heads, w.head_dim, sms)
-        line["dp_latency_boundaries"] = measure_uniform(w, q, k, v, dev, stream, bounds=[b])
-        line["dp_latency_boundaries"].update({"sms": sms, "window_units": 8,
-                                              "first_chunk_rows": b[1] - b[0],
-                                              "last_chunk_rows": b[-1] - b[-2]})
+        variants = {
+            "workload_boundaries": pf.bounds[0],
+            "uniform_boundaries": m.mocap_lbcp_partition(s_len, n_chunks, 128,
+                                                         m.MOCAP_PART_UNIFORM),
+            "dp_causal_boundaries": m.mocap_lbcp_partition_dp(s_len, n_chunks, 128, 16,
+                                                              m.MOCAP_COST_CAUSAL, 0),
+            "dp_eq1_boundaries": m.mocap_lbcp_partition_dp(s_len, n_chunks, 128, 16,
+                                                           m.MOCAP_COST_EQ1, 0),
+            "dp_latency_boundaries": latency_balanced_bounds(s_len, n_chunks, w.n_q_heads,
+                                                             w.n_kv_heads, w.head_dim, sms),
+        }
+        res = measure_partitions(w, q, k, v, dev, stream, variants)
+        line["partitions"] = {"note": "each split's whole prompt and each of its chunk steps "
+                                      "replayed from CUDA graphs, the splits interleaved; "
+                                      "medians", "sms": sms, "dp_latency_window_units": 8,
+                              **res}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         times, flops, done, threads = run_oracle_sample(
             q, k, v, pf.bounds[0], w.scale, 1, args.cpu_rows_per_chunk, 20.0)
@@ -878,27 +883,50 @@ def measure_last_row(args, m, w, pf, q, dev, stream, hbm):
             "requests": n, "note": "back-to-back calls; K/V may be partly L2-resident"}
 
 
-def measure_uniform(w, q, k, v, dev, stream, reps=3, bounds=None):
-    """Per-chunk attention latency with uniform boundaries (outside the timed
-    region): without latency-balanced chunks the late chunks dominate.  With
-    ``bounds`` the same measurement for that explicit split."""
+def measure_partitions(w, q, k, v, dev, stream, variants, rounds=5):
+    """Per-chunk attention latency and whole-prompt time of several chunk
+    splits of one prompt (outside the timed region): each split's whole
+    prompt and each of its chunk steps are captured as CUDA graphs and the
+    splits are replayed interleaved, round after round (the GPU's clock under
+    its power cap moves between short bursts; interleaving gives every split
+    the same conditions).  Medians over the rounds."""
     import torch
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
-    from paper_2606_22968_gb300 import workloads
-    pu = ChunkedPrefill(w, dev, mode=workloads.MODE_UNIFORM, bounds=bounds, chunk_streams=1)
-    n = len(pu.steps())
-    times = []
-    for _ in range(reps):
-        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n)]
-        pu.run(q, k, v, stream, ev)
-        torch.cuda.synchronize(dev)
-        times.append([ev[c][1].elapsed_time(ev[c][2]) for c in range(n)])
-    per_chunk = [statistics.median(t[c] for t in times) for c in range(n)]
-    del pu
-    return {"per_chunk_attn_ms": {"min": min(per_chunk), "max": max(per_chunk),
-                                  "max_over_min": max(per_chunk) / min(per_chunk),
-                                  "cv": statistics.pstdev(per_chunk) / statistics.mean(per_chunk)},
-            "attn_ms_per_step": sum(per_chunk)}
+    state = {}
+    for name, b in variants.items():
+        px = ChunkedPrefill(w, dev, bounds=[b], chunk_streams=1)
+        px.run(q, k, v, stream)
+        state[name] = (px, px.capture(q, k, v), px.capture_steps(q, k, v))
+    torch.cuda.synchronize(dev)
+    whole = {n: [] for n in variants}
+    chunks = {n: [[] for _ in range(len(b) - 1)] for n, b in variants.items()}
+    names = list(variants)
+    for r in range(rounds):
+        for n in (names if r % 2 == 0 else names[::-1]):
+            _, g, gs = state[n]
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(gs) + 1)]
+            ev[0].record(stream)
+            for i, gi in enumerate(gs):
+                gi.replay()
+                ev[i + 1].record(stream)
+            torch.cuda.synchronize(dev)
+            whole[n].append(e0.elapsed_time(e1))
+            for i in range(len(gs)):
+                chunks[n][i].append(ev[i].elapsed_time(ev[i + 1]))
+    out = {}
+    for n, b in variants.items():
+        pc = [statistics.median(x) for x in chunks[n]]
+        out[n] = {"per_chunk_attn_ms": {"min": min(pc), "max": max(pc),
+                                        "max_over_min": max(pc) / min(pc),
+                                        "cv": statistics.pstdev(pc) / statistics.mean(pc)},
+                  "attn_ms_per_step": sum(pc), "graph_ms_per_step": statistics.median(whole[n]),
+                  "first_chunk_rows": b[1] - b[0], "last_chunk_rows": b[-1] - b[-2]}
+    del state
+    return out
 
 
 def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):

@@ -212,7 +212,8 @@ def test_bench_entry_points_exist():
     import bench
     for name in ["profile_case", "profile_case_append", "profile_case_qkv", "profile_case_last_row", "ours_arm",
                  "reference_arm", "measure_e2e", "measure_graph", "measure_projection",
-                 "measure_last_row", "measure_uniform"]:
+                 "measure_last_row", "measure_partitions", "measure_chunk_streams",
+                 "measure_fusion", "measure_append_graph"]:
         assert callable(getattr(bench, name)), name
 
 
