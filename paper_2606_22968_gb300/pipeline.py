@@ -261,10 +261,12 @@ class ChunkedPrefill:
         if events is not None:
             events[2].record(stream)
 
-    def run(self, q, k, v, stream=None, chunk_events=None, landed=None):
+    def run(self, q, k, v, stream=None, chunk_events=None, landed=None, after_step=None):
         """The whole prompt: every step in order.  ``chunk_events`` optionally
         holds one event triple per step (see run_step); ``landed`` optionally
-        one event per step after which its inputs are in q, k, v."""
+        one event per step after which its inputs are in q, k, v;
+        ``after_step(i, st)`` is called once step i has been enqueued on
+        stream ``st`` (e.g. to queue work that waits for it)."""
         main = torch.cuda.current_stream(self.device) if stream is None else stream
         n = len(self.steps())
         ready, side = [None] * n, None
@@ -292,6 +294,8 @@ class ChunkedPrefill:
             with torch.cuda.stream(st):
                 self.run_step(q, k, v, i, st, None if chunk_events is None else chunk_events[i],
                               ready[i], workspace=ws)
+            if after_step is not None:
+                after_step(i, st)
         if second is not None:
             main.wait_stream(second)
         if side is not None:
@@ -326,47 +330,26 @@ class ChunkedPrefill:
         return slice(self.cu[r] + b0, self.cu[r] + b1), b0, b1
 
     def _compute_and_return(self, q, k, v, compute, d2h, landed, host_out, host_lse):
-        """Every step on ``compute`` once its inputs have landed (events
-        ``landed``), each step's O (and a single request's LSE block) copied
-        back on ``d2h`` as soon as that step is done."""
+        """Every step on ``compute`` (and the second compute stream) once its
+        inputs have landed (events ``landed``), each step's O (and a single
+        request's LSE block) copied back on ``d2h`` as soon as that step is
+        done."""
         steps = self.steps()
         hq = self.w.n_q_heads
-        n = len(steps)
-        ready, side = [None] * n, None
-        if self.append_mode == "overlap" and n > 1:
-            ready, side = self.launch_appends(k, v, compute, landed)
-        second = None
-        if self.chunk_streams == 2 and n > 1:
-            # as in run: step 0's chunks first, then two compute streams
-            compute.wait_event(landed[0])
-            for r, c in steps[0]:
-                kr, vr, dst = self._append_rows(k, v, r, c)
-                mocap_kv_append(kr, vr, self.k_cache, self.v_cache, dst, stream=compute)
-            ready[0] = torch.cuda.Event()
-            ready[0].record(compute)
-            second = torch.cuda.Stream(self.device)
-            second.wait_stream(compute)
-        for i, step in enumerate(steps):
-            st, ws = (second, self.workspace2) if (second is not None and i % 2) else (compute, None)
-            st.wait_event(landed[i])
-            if self.append_mode == "fused" and i + 1 < n:
-                st.wait_event(landed[i + 1])  # this launch appends step i + 1's K/V
-            with torch.cuda.stream(st):
-                self.run_step(q, k, v, i, st, ready=ready[i], workspace=ws)
+
+        def copy_back(i, st):
             done = torch.cuda.Event()
             done.record(st)
             d2h.wait_event(done)
             with torch.cuda.stream(d2h):
-                for r, c in step:
+                for r, c in steps[i]:
                     rows, b0, b1 = self._rows(r, c)
                     host_out[rows].copy_(self.out[rows], non_blocking=True)
                     if self.single:
                         host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
                                                         non_blocking=True)
-        if second is not None:
-            compute.wait_stream(second)
-        if side is not None:
-            compute.wait_stream(side)
+
+        self.run(q, k, v, compute, landed=landed, after_step=copy_back)
 
     def run_from_host(self, host_q, host_k, host_v, host_out, host_lse, q, k, v):
         """The whole prompt from (pinned) host memory, overlapping transfers
