@@ -518,6 +518,29 @@ def test_dp_boundaries_pipeline_parity(m):
     check_single_request(pf, q, k, v, rows_fn=lambda n, i: sample_rows(n, every=509, edge=2, seed=i))
 
 
+def test_latency_model_boundaries_pipeline_parity(m):
+    """A prompt split by Algorithm 1's stage-1 DP with the kernel's latency
+    model as EvaluateChunk (bit-exact against the oracle's DP) runs through
+    the default pipeline and matches the attention oracle on sampled rows of
+    every chunk."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill, latency_balanced_bounds
+    w = workloads.get(3)
+    dev = torch.device("cuda")
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    b = latency_balanced_bounds(w.seq_lens[0], w.num_chunks[0], w.n_q_heads, w.n_kv_heads,
+                                w.head_dim, sms, 16, 4)
+    assert b == P.dp_latency_boundaries(w.seq_lens[0], w.num_chunks[0], 16, w.n_q_heads,
+                                        w.n_kv_heads, w.head_dim, sms, 4)
+    q, k, v = workloads.make_qkv(w, dev)
+    pf = ChunkedPrefill(w, dev, bounds=[b])
+    pf.run(q, k, v)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == 0
+    assert torch.equal(pf.k_cache, k) and torch.equal(pf.v_cache, v)
+    check_single_request(pf, q, k, v, rows_fn=lambda n, i: sample_rows(n, every=509, edge=2, seed=i))
+
+
 def test_nvtx_ranges_leave_results_unchanged(m, monkeypatch):
     """MOCAP_NVTX=1 wraps each chunk step in an NVTX range; the launches and
     results are the same."""
