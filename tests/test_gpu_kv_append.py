@@ -1,5 +1,7 @@
-"""GPU: mocap_kv_append writes exactly the chunk rows, bit for bit, and no
-other cache byte (sentinel bit patterns, NaN included, must survive)."""
+"""GPU: mocap_kv_append and mocap_kv_append_overlap (the one-warp kernel that
+runs beside attention launches) write exactly the chunk rows, bit for bit,
+and no other cache byte (sentinel bit patterns, NaN included, must
+survive)."""
 
 import numpy as np
 import pytest
@@ -17,6 +19,10 @@ def m():
     return mod
 
 
+APPENDS = ["mocap_kv_append", "mocap_kv_append_overlap"]
+
+
+@pytest.mark.parametrize("fn", APPENDS)
 @pytest.mark.parametrize("cap,offset,length,hkv,d", [
     (1000, 0, 1000, 8, 128),
     (1000, 3, 1, 8, 128),
@@ -25,7 +31,7 @@ def m():
     (300, 17, 250, 1, 8),
     (70000, 65536, 4464, 8, 128),
 ])
-def test_append_bitwise_with_sentinels(m, cap, offset, length, hkv, d):
+def test_append_bitwise_with_sentinels(m, fn, cap, offset, length, hkv, d):
     dev = torch.device("cuda")
     gen = torch.Generator(device=dev).manual_seed(cap + offset)
     sentinel = torch.randint(-32768, 32767, (cap, hkv, d), generator=gen, device=dev,
@@ -39,7 +45,7 @@ def test_append_bitwise_with_sentinels(m, cap, offset, length, hkv, d):
                       dtype=torch.int16).view(torch.bfloat16)
     kc0 = kc.view(torch.int16).cpu().numpy()
     vc0 = vc.view(torch.int16).cpu().numpy()
-    m.mocap_kv_append(k, v, kc, vc, offset)
+    getattr(m, fn)(k, v, kc, vc, offset)
     torch.cuda.synchronize()
     k_ref = A.kv_append(kc0, k.view(torch.int16).cpu().numpy(), offset)
     v_ref = A.kv_append(vc0, v.view(torch.int16).cpu().numpy(), offset)
@@ -47,16 +53,18 @@ def test_append_bitwise_with_sentinels(m, cap, offset, length, hkv, d):
     assert np.array_equal(vc.view(torch.int16).cpu().numpy(), v_ref)
 
 
-def test_append_rejects_overflow(m):
+@pytest.mark.parametrize("fn", APPENDS)
+def test_append_rejects_overflow(m, fn):
     dev = torch.device("cuda")
     kc = torch.zeros((10, 8, 128), device=dev, dtype=torch.bfloat16)
     k = torch.zeros((4, 8, 128), device=dev, dtype=torch.bfloat16)
     with pytest.raises(m.MocapError):
-        m.mocap_kv_append(k, k, kc, kc.clone(), 7)
+        getattr(m, fn)(k, k, kc, kc.clone(), 7)
 
 
+@pytest.mark.parametrize("fn", APPENDS)
 @pytest.mark.parametrize("case", range(30))
-def test_random_append_sweep(m, case):
+def test_random_append_sweep(m, fn, case):
     """Seeded random appends (rows a whole number of 16-byte vectors):
     bitwise equal to the oracle's copy, every other cache row untouched."""
     rng = np.random.default_rng(60 + case)
@@ -65,4 +73,4 @@ def test_random_append_sweep(m, case):
     length = int(rng.choice([int(rng.integers(1, 64)), int(rng.integers(64, 20000))]))
     offset = int(rng.integers(0, 50000))
     cap = offset + length + int(rng.integers(0, 100))
-    test_append_bitwise_with_sentinels(m, cap, offset, length, hkv, d)
+    test_append_bitwise_with_sentinels(m, fn, cap, offset, length, hkv, d)
