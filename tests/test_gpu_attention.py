@@ -191,13 +191,13 @@ def test_varlen_equals_single_launches_bitwise(m):
 
 
 # ---------------------------------------------------------------- workloads --
-def _workload_parity(m, index, rows_fn, chunks=None, heads_fn=None):
+def _workload_parity(m, index, rows_fn, chunks=None, heads_fn=None, chunk_streams=None):
     from paper_2606_22968_gb300 import workloads
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
     w = workloads.get(index)
     dev = torch.device("cuda")
     q, k, v = workloads.make_qkv(w, dev)
-    pf = ChunkedPrefill(w, dev)
+    pf = ChunkedPrefill(w, dev, chunk_streams=chunk_streams)
     assert pf.bounds[0] == P.boundaries(w.seq_lens[0], w.num_chunks[0], 128, w.mode)
     pf.run(q, k, v)
     torch.cuda.synchronize()
@@ -219,9 +219,11 @@ def test_workload3_32k_lbcp_sampled(m):
 
 
 def test_workload4_128k_lbcp_sampled(m):
-    # the first, a middle and the last three chunks, sparsely sampled
+    # the first, a middle and the last three chunks, sparsely sampled, all
+    # heads; one compute stream with the appends beside it, the launch
+    # configuration bench.py times
     _workload_parity(m, 4, lambda n, i: sample_rows(n, every=1021, edge=2, seed=i)[::3],
-                     chunks=[0, 1, 15, 29, 30, 31])
+                     chunks=[0, 1, 15, 29, 30, 31], chunk_streams=1)
 
 
 def test_workload4_every_chunk_at_every_tile_edge(m):
