@@ -803,6 +803,7 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
     n = len(b) - 1
     ms_gemm = timed(lambda: [project(c) for c in range(n)])
     ms_stage = timed(lambda: pf.run_stage(x, wq, qbuf, stream))
+    ms_stage_overlap = timed(lambda: pf.run_stage(x, wq, qbuf, stream, overlap=True))
     if m.mocap_last_device_status() != m.MOCAP_OK:
         raise RuntimeError("device wait expired in the projection measurement")
     gemm_tf = gemm_flops / (ms_gemm * 1e-3) / 1e12
@@ -810,7 +811,11 @@ def measure_projection(args, m, w, pf, q, dev, stream, attn_flops, peak):
             "ms_per_step": ms_gemm, "tflops": gemm_tf, "frac_of_peak": gemm_tf / peak,
             "stage_ms_per_step": ms_stage,
             "stage_tflops": (gemm_flops + attn_flops) / (ms_stage * 1e-3) / 1e12,
-            "stage_tokens_per_s": w.total_tokens / (ms_stage * 1e-3)}
+            "stage_tokens_per_s": w.total_tokens / (ms_stage * 1e-3),
+            # projections on their own stream, each chunk's attention waiting
+            # only for its own chunk's projection (two compute streams)
+            "stage_overlap_ms_per_step": ms_stage_overlap,
+            "stage_overlap_tflops": (gemm_flops + attn_flops) / (ms_stage_overlap * 1e-3) / 1e12}
 
     # Per-chunk stage latency (projection + attention of one chunk), for the
     # workload's split and for the stage-1 DP of Algorithm 1 fed with this

@@ -302,17 +302,27 @@ class ChunkedPrefill:
             main.wait_stream(side)
 
     def run_stage(self, x, w_qkv, q_buf, stream=None, rope_theta: float = 500000.0,
-                  chunk_events=None):
+                  chunk_events=None, overlap: bool = False):
         """One attention layer's chunk stage for a single request (Eq. 1 with
         its GEMM term): per chunk, in order, the fused QKV projection of the
         chunk's hidden states ``x`` [S, hidden] with ``w_qkv`` [(Hq + 2 Hkv) d,
         hidden] (RoPE at the chunk's global positions; Q to ``q_buf`` [S, Hq,
         d], K and V straight into the caches), then the chunk's attention over
         the cache.  ``chunk_events`` optionally holds one (start, end) event
-        pair per chunk."""
+        pair per chunk.
+
+        ``overlap=True``: the projections run in order on a stream of their
+        own and each chunk's attention, alternating between two compute
+        streams (their own split-KV scratch), waits only for its chunk's
+        projection: chunk c + 1's projection writes rows chunk c's attention
+        never reads, so the two overlap (no ``chunk_events``)."""
         if not self.single:
             raise ValueError("run_stage takes a single-request workload")
         w, b = self.w, self.bounds[0]
+        if overlap:
+            if chunk_events is not None:
+                raise ValueError("chunk_events need overlap=False")
+            return self._run_stage_overlapped(x, w_qkv, q_buf, stream, rope_theta)
         for c in range(len(b) - 1):
             if chunk_events is not None:
                 chunk_events[c][0].record(stream)
@@ -323,6 +333,31 @@ class ChunkedPrefill:
                              workspace=self.workspace, stream=stream)
             if chunk_events is not None:
                 chunk_events[c][1].record(stream)
+
+    def _run_stage_overlapped(self, x, w_qkv, q_buf, stream, rope_theta):
+        w, b = self.w, self.bounds[0]
+        main = torch.cuda.current_stream(self.device) if stream is None else stream
+        proj = torch.cuda.Stream(self.device)
+        second = torch.cuda.Stream(self.device)
+        proj.wait_stream(main)
+        second.wait_stream(main)
+        if self.workspace is not None and self.workspace2 is None:
+            self.workspace2 = torch.empty_like(self.workspace)
+        for c in range(len(b) - 1):
+            with torch.cuda.stream(proj):
+                mocap_qkv_rope_append(x[b[c]:b[c + 1]], w_qkv, q_buf[b[c]:b[c + 1]],
+                                      self.k_cache, self.v_cache, b[c], rope_theta=rope_theta,
+                                      stream=proj)
+            projected = torch.cuda.Event()
+            projected.record(proj)
+            st, ws = (second, self.workspace2) if c % 2 else (main, self.workspace)
+            st.wait_event(projected)
+            with torch.cuda.stream(st):
+                mocap_chunk_attn(q_buf[b[c]:b[c + 1]], self.k_cache, self.v_cache, b[c],
+                                 self.out[b[c]:b[c + 1]], self.chunk_lse(c), w.scale,
+                                 workspace=ws, stream=st)
+        main.wait_stream(second)
+        main.wait_stream(proj)
 
     # -- from host memory ------------------------------------------------------------
     def _rows(self, r, c):

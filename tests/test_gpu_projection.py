@@ -111,13 +111,16 @@ def test_qkv_rope_full_size_sampled_rows(m, length, offset):
                                                                    err.mean())
 
 
-def test_run_stage_projection_then_attention(m):
+@pytest.mark.parametrize("overlap", [False, True])
+def test_run_stage_projection_then_attention(m, overlap):
     """ChunkedPrefill.run_stage: per chunk the fused projection writes Q and
     the chunk's K/V rows, then attention reads the cache.  The projection
     outputs match the projection oracle, and the attention matches the
     attention oracle on the exact Q/K/V bits the projection produced (every
     chunk, sampled rows), so positions and cache rows line up across the
-    two kernels."""
+    two kernels.  ``overlap``: projections on their own stream, attention
+    alternating between two compute streams, each chunk's attention waiting
+    only for its own projection."""
     from oracle import attention as A
     from paper_2606_22968_gb300 import workloads
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
@@ -133,7 +136,7 @@ def test_run_stage_projection_then_attention(m):
     pf = ChunkedPrefill(w, dev)
     qbuf = torch.full((8192, w.n_q_heads, w.head_dim), float("nan"), device=dev,
                       dtype=torch.bfloat16)
-    pf.run_stage(x, wq, qbuf, rope_theta=theta)
+    pf.run_stage(x, wq, qbuf, rope_theta=theta, overlap=overlap)
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == 0
     q_ref, k_ref, v_ref = R.qkv_rope(f64(x), f64(wq), w.n_q_heads, w.n_kv_heads, w.head_dim, 0,
