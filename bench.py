@@ -60,7 +60,7 @@ def parse_args():
                     help="skip the last-row-only attention measurement")
     ap.add_argument("--no-uniform", action="store_true",
                     help="skip the uniform-boundary per-chunk latency comparison")
-    ap.add_argument("--cpu-rows-per-chunk", type=int, default=2)
+    ap.add_argument("--cpu-rows-per-chunk", type=int, default=4)
     ap.add_argument("--case", default=None,
                     help="profiling case 'prefix,len,Hq,Hkv,d': one chunk attention launch "
                          "repeated warmup+steps times (no JSON metric line)")
@@ -510,7 +510,16 @@ def ours_arm(args, rank, world, local):
         "attn_tflops_kernel_only": achieved,
         "attn_frac_of_peak": achieved / peak,
         "per_chunk_attn_ms": {"min": min(per_chunk), "max": max(per_chunk),
-                              "max_over_min": max(per_chunk) / min(per_chunk), "cv": cv},
+                              "max_over_min": max(per_chunk) / min(per_chunk), "cv": cv,
+                              "ms": [round(t, 4) for t in per_chunk],
+                              # each step's attention FLOP / its median launch time,
+                              # and that rate's fraction of the sustained peak
+                              "tflops": [round(f / (t * 1e-3) / 1e12, 1)
+                                         for f, t in zip(step_flops, per_chunk)],
+                              "frac_of_peak_min": min(f / (t * 1e-3) / 1e12 for f, t in
+                                                      zip(step_flops, per_chunk)) / peak,
+                              "frac_of_peak_max": max(f / (t * 1e-3) / 1e12 for f, t in
+                                                      zip(step_flops, per_chunk)) / peak},
         "append": {"bytes_per_step": append_bytes,
                    "standalone_bytes_per_step": standalone_bytes,
                    "fused_bytes_per_step": append_bytes - standalone_bytes,
