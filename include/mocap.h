@@ -19,6 +19,7 @@
  *   mocap_qkv_rope_append     QKV projection + RoPE + KV append (device GEMM)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
+ *   mocap_chunk_attn_varlen_dev  the same with the items in device memory
  *   mocap_chunk_attn_append, mocap_chunk_attn_varlen_append
  *                             the same with the next chunk's KV append in the launch
  *   mocap_last_row_attn       each request's last row only (prefill-only output)
@@ -401,6 +402,64 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
                                      void *workspace, size_t workspace_bytes,
                                      mocap_stream_t stream);
 
+#define MOCAP_VARLEN_DEV_MAX_ITEMS 65536
+
+/*
+ * mocap_chunk_attn_varlen_dev_workspace_size -- bytes of device scratch that
+ * mocap_chunk_attn_varlen_dev needs for up to n_items items over packed
+ * q / out buffers of q_rows_total rows: per item its three TMA tensor maps
+ * (384 B) and descriptor, one 4-byte entry per CTA of the launch's grid
+ * (at most (ceil(q_rows_total / 128) + n_items) x n_kv_heads x
+ * ceil(n_q_heads / n_kv_heads / 2) CTAs) and the CTA count.  0 when
+ * n_items == 0 or an argument is out of range.
+ */
+size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items, int64_t q_rows_total,
+                                                  int32_t n_q_heads, int32_t n_kv_heads,
+                                                  int32_t head_dim);
+
+/*
+ * mocap_chunk_attn_varlen_dev -- mocap_chunk_attn_varlen with the item array
+ * in DEVICE memory (Sec. 2.2: chunk k of every request of a batch in one
+ * launch), so a device-side scheduler, or a CUDA graph replayed with new
+ * item values, supplies the (request, chunk) items without a host round
+ * trip.  Up to MOCAP_VARLEN_DEV_MAX_ITEMS items.
+ *
+ *   items        DEVICE array of n_items mocap_varlen_item (8-byte aligned),
+ *                read by the launch; the caller keeps it unchanged until the
+ *                work queued on `stream` has started past it
+ *   workspace, workspace_bytes: caller-owned device scratch, 128-byte
+ *                aligned, at least mocap_chunk_attn_varlen_dev_workspace_size
+ *                (n_items, q_rows_total, ...) bytes; overwritten by the call
+ *   other arguments as mocap_chunk_attn_varlen.
+ *
+ * Three launches on `stream`: a one-block kernel validates the items, counts
+ * and scans their CTAs and builds each item's tensor maps (tensormap.replace
+ * of the global address and row extent of templates the host encodes over
+ * the whole buffers); a second fills the CTA -> item table; then the
+ * attention kernel, on a grid of the upper bound above, whose surplus CTAs
+ * exit at once.  Per item the results are bitwise those of
+ * mocap_chunk_attn_varlen with two or more items (this form never splits a
+ * key range).  CTAs follow the items in the order given: put the items with
+ * the most keys first (the host-array form sorts them so itself).
+ *
+ * Errors: the host-side checks of mocap_chunk_attn_varlen on the shape,
+ * pointers and totals, n_items outside [0, MOCAP_VARLEN_DEV_MAX_ITEMS], a
+ * null or misaligned items array, a missing, misaligned or short workspace
+ * -> MOCAP_EINVAL.  An item that fails mocap_chunk_attn_varlen's item checks
+ * (negative field, rows outside q_rows_total / kv_rows_total,
+ * prefix + len >= 2^31), or items whose Q rows overlap beyond the grid's
+ * bound, are found on the device: the call then writes nothing and records
+ * MOCAP_EINVAL in the status word that mocap_last_device_status returns (and
+ * clears); until then later launches do nothing, as after an expired wait.
+ * Items must not write overlapping output rows.  n_items == 0 is a no-op.
+ */
+mocap_status mocap_chunk_attn_varlen_dev(const void *q, const void *k_cache, const void *v_cache,
+                                         const mocap_varlen_item *items, int32_t n_items,
+                                         int64_t q_rows_total, int64_t kv_rows_total,
+                                         int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
+                                         float scale, void *out, float *lse, void *workspace,
+                                         size_t workspace_bytes, mocap_stream_t stream);
+
 /*
  * One KV append that an attention launch carries out (see
  * mocap_chunk_attn_append): rows [0, rows) of k_src / v_src (bf16
@@ -503,8 +562,10 @@ mocap_status mocap_last_row_attn(const void *q_last, const void *k_cache, const 
 /*
  * mocap_last_device_status -- synchronises `stream`, then reads and clears
  * the device status word that the kernels set when a bounded wait expires
- * (MOCAP_ETIMEOUT) instead of hanging.  MOCAP_OK when nothing was recorded;
- * MOCAP_ECUDA if the synchronisation itself failed.
+ * (MOCAP_ETIMEOUT) instead of hanging, or when mocap_chunk_attn_varlen_dev
+ * finds an invalid device item (MOCAP_EINVAL); the first recorded value
+ * stays.  MOCAP_OK when nothing was recorded; MOCAP_ECUDA if the
+ * synchronisation itself failed.
  */
 mocap_status mocap_last_device_status(mocap_stream_t stream);
 

@@ -127,6 +127,14 @@ struct AttnParams {
   int64_t app_total;
   int32_t n_app;
   AppendSeg app[kMaxAppends];
+  // Device item descriptors (DEV instantiations, items in device memory):
+  // the item of every CTA, each item's ItemDesc and three tensor maps, and
+  // the launch's CTA count, all written by the prepare kernels before the
+  // launch (attn_varlen_dev.cuh).  CTAs at or past *dev_total exit at once.
+  const ItemDesc *dev_items;
+  const int32_t *dev_cta_item;
+  const CUtensorMap *dev_maps;  // [item][Q, K, V]
+  const int32_t *dev_total;
 };
 
 // Kernel parameters are limited to 32764 bytes (__grid_constant__ block).
@@ -283,7 +291,28 @@ __device__ __noinline__ void append_share(const AttnParams<MAXI> &p, int tid, in
 
 // Warpgroup 0: warp 0 is the TMA producer, warp 1 the MMA issuer (one lane
 // each); warps 2-3 copy this CTA's share of the launch's KV appends, if any.
-template <int D, int MAXI, bool APPEND>
+// The Q, K and V tensor maps of `item`: launch parameters, or (DEV) the maps
+// a prepare kernel built in global memory, acquired for the tensormap proxy
+// before their first use.
+template <bool DEV, int MAXI>
+__device__ __forceinline__ void item_maps(const AttnParams<MAXI> &p, int item,
+                                          const CUtensorMap *&mq, const CUtensorMap *&mk,
+                                          const CUtensorMap *&mv) {
+  if constexpr (DEV) {
+    mq = p.dev_maps + 3 * static_cast<int64_t>(item);
+    mk = mq + 1;
+    mv = mq + 2;
+    tmap_acquire(mq);
+    tmap_acquire(mk);
+    tmap_acquire(mv);
+  } else {
+    mq = &p.tq[item];
+    mk = &p.tk[item];
+    mv = &p.tv[item];
+  }
+}
+
+template <int D, int MAXI, bool APPEND, bool DEV = false>
 __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_t base,
                                               uint32_t bars, uint32_t tmem, uint32_t warp,
                                               uint32_t lane, int item, int g, int h0, int r0,
@@ -293,9 +322,8 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
   if (warp == 0) {
     // ===================== TMA producer =====================================
     if (lane == 0) {
-      const CUtensorMap *mq = &p.tq[item];
-      const CUtensorMap *mk = &p.tk[item];
-      const CUtensorMap *mv = &p.tv[item];
+      const CUtensorMap *mq, *mk, *mv;
+      item_maps<DEV>(p, item, mq, mk, mv);
       prefetch_tmap(mq);
       prefetch_tmap(mk);
       prefetch_tmap(mv);
@@ -425,7 +453,7 @@ __device__ __forceinline__ void control_roles(const AttnParams<MAXI> &p, uint32_
 //   O_s += P_s V    M = 256 (P in each CTA's TMEM), N = 128 dims
 // and its commits arrive on both CTAs' barriers.  Both CTAs' copies count on
 // the first CTA's barriers, and so do both CTAs' P arrivals.
-template <int MAXI, bool APPEND>
+template <int MAXI, bool APPEND, bool DEV = false>
 __device__ __forceinline__ void control_roles_pair(const AttnParams<MAXI> &p, uint32_t base,
                                                    uint32_t bars, uint32_t tmem, uint32_t warp,
                                                    uint32_t lane, uint32_t rank, int item, int g,
@@ -438,9 +466,8 @@ __device__ __forceinline__ void control_roles_pair(const AttnParams<MAXI> &p, ui
   if (warp == 0) {
     // ===================== TMA producer (both CTAs) =========================
     if (lane == 0) {
-      const CUtensorMap *mq = &p.tq[item];
-      const CUtensorMap *mk = &p.tk[item];  // 64-row boxes: this CTA's half K tile
-      const CUtensorMap *mv = &p.tv[item];
+      const CUtensorMap *mq, *mk, *mv;  // K in 64-row boxes: this CTA's half K tile
+      item_maps<DEV>(p, item, mq, mk, mv);
       prefetch_tmap(mq);
       prefetch_tmap(mk);
       prefetch_tmap(mv);
@@ -748,7 +775,8 @@ __device__ __forceinline__ void cta_barrier() {
 // APPEND: the launch carries KV appends (warps 2-3 copy them).  A separate
 // instantiation, so launches without appends run exactly the code they
 // would without this feature.
-template <int D, int MAXI, bool PAIR = false, bool APPEND = false>
+// DEV: the items are device descriptors (the prepare kernels' tables).
+template <int D, int MAXI, bool PAIR = false, bool APPEND = false, bool DEV = false>
 __global__ void __launch_bounds__(kThreads, 1)
     chunk_attn_kernel(const __grid_constant__ AttnParams<MAXI> p) {
   using L = Layout<D, PAIR>;
@@ -774,8 +802,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   // ---- work item --------------------------------------------------------
   int item = 0;
   const int cta = static_cast<int>(blockIdx.x);
-  while (item + 1 < p.n_items && cta >= p.items[item + 1].cta_begin) ++item;
-  const ItemDesc it = p.items[item];
+  if constexpr (DEV) {
+    // the grid is an upper bound; a CTA pair's two CTAs exit together (the
+    // count is a whole number of pairs)
+    if (cta >= *p.dev_total) return;
+    item = p.dev_cta_item[cta];
+  } else {
+    while (item + 1 < p.n_items && cta >= p.items[item + 1].cta_begin) ++item;
+  }
+  const ItemDesc it = DEV ? p.dev_items[item] : p.items[item];
   int w = cta - it.cta_begin;
   // CTA order: head pair fastest, then split, then row block (heaviest
   // first), then KV group slowest, so the CTAs resident at once mostly
@@ -857,7 +892,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (run) {
       if (warp < 4) {
         setmaxnreg_dec<kRegsControl>();
-        control_roles_pair<MAXI, APPEND>(p, base, bar(0), tmem, warp, lane, rank, item, g, h0, r0, nslots,
+        control_roles_pair<MAXI, APPEND, DEV>(p, base, bar(0), tmem, warp, lane, rank, item, g, h0, r0, nslots,
                                  t0, n_kv);
       } else {
         setmaxnreg_inc<kRegsSoftmax>();
@@ -875,7 +910,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     if (warp < 4) {
       setmaxnreg_dec<kRegsControl>();
-      control_roles<D, MAXI, APPEND>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, t0,
+      control_roles<D, MAXI, APPEND, DEV>(p, base, bar(0), tmem, warp, lane, item, g, h0, r0, nslots, t0,
                              n_kv);
       tc_fence_before();
       cta_barrier();

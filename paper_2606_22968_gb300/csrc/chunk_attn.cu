@@ -1,8 +1,8 @@
 // chunk_attn.cu -- host side of the chunked causal GQA prefill attention:
 // tensor maps, the split-KV plan, launches of the attention kernel
 // (attn_kernel.cuh) and of the split-KV combine (attn_combine.cuh), and the
-// C entry points (mocap_chunk_attn, _varlen, _append, _varlen_append,
-// _workspace_size, _noalloc).
+// C entry points (mocap_chunk_attn, _varlen, _varlen_dev, _append,
+// _varlen_append, _workspace_size, _noalloc).
 //
 // Sec. 2.2 / Eq. 1: chunk i's queries (global rows prefix .. prefix+len-1)
 // attend to the KV of every earlier chunk plus a causal block over their own
@@ -26,6 +26,7 @@
 #include "sm103_ptx.cuh"
 #include "attn_kernel.cuh"
 #include "attn_combine.cuh"
+#include "attn_varlen_dev.cuh"
 
 namespace mocap {
 namespace {
@@ -161,6 +162,37 @@ bool pair_enabled() {
   return env == nullptr || std::atoi(env) != 0;
 }
 
+// One attention launch of `kern` with `prm` on `ctas` CTAs, as CTA pairs
+// (clusters of two) or single CTAs.  Once per kernel and device (`done`):
+// the register-count check (the setmaxnreg split assumes kLaunchRegs) and
+// the dynamic shared-memory limit.
+template <typename Kern, typename P>
+mocap_status start_attn(Kern kern, const P &prm, int64_t ctas, bool as_pair, int smem, bool *done,
+                        int dev, cudaStream_t stream) {
+  if (!done[dev]) {
+    cudaFuncAttributes fa{};
+    if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) return MOCAP_ECUDA;
+    if (fa.numRegs != kLaunchRegs) return MOCAP_EUNSUPPORTED;  // split would not balance
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+        cudaSuccess)
+      return MOCAP_ECUDA;
+    done[dev] = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(ctas));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = as_pair ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, prm) == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+}
+
 template <int D, int MAXI>
 mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
                     const std::vector<HostItem> &items, int64_t lse_stride, const Shape &sh,
@@ -235,35 +267,9 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
 
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
-  // one-time per kernel and device: register count check, shared-memory size
-  auto prepare = [&](auto kern, int smem, bool *done) -> mocap_status {
-    if (done[dev]) return MOCAP_OK;
-    cudaFuncAttributes fa{};
-    if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) return MOCAP_ECUDA;
-    if (fa.numRegs != kLaunchRegs) return MOCAP_EUNSUPPORTED;  // split would not balance
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
-        cudaSuccess)
-      return MOCAP_ECUDA;
-    done[dev] = true;
-    return MOCAP_OK;
-  };
   // the CTA-pair or single-CTA form, each with or without the append copy
   auto launch_form = [&](auto kern, bool as_pair, int smem, bool *done) -> mocap_status {
-    const mocap_status st = prepare(kern, smem, done);
-    if (st != MOCAP_OK) return st;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(ctas));
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = static_cast<size_t>(smem);
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = as_pair ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, kern, prm) == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+    return start_attn(kern, prm, ctas, as_pair, smem, done, dev, stream);
   };
   const bool append = prm.n_app > 0;
   mocap_status lst = MOCAP_OK;
@@ -362,6 +368,124 @@ bool pointers_ok(const void *q, const void *k, const void *v, const void *out, c
 }
 
 constexpr int64_t kMaxRows = 0x7fffffffLL;
+
+// ---- mocap_chunk_attn_varlen_dev -------------------------------------------
+// Scratch of the device-descriptor form (offsets in bytes; the tensor maps,
+// three per item, start at 0): ItemDescs, the CTA -> item table of the
+// grid's upper bound, the CTA count.
+struct DevLayout {
+  int64_t max_ctas = 0;
+  size_t descs = 0, cta_item = 0, total = 0, bytes = 0;
+};
+
+size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+
+bool dev_layout(int32_t n_items, int64_t q_rows_total, const Shape &sh, DevLayout *out) {
+  if (n_items < 1 || n_items > MOCAP_VARLEN_DEV_MAX_ITEMS || q_rows_total < 0 ||
+      q_rows_total > kMaxRows)
+    return false;
+  const int64_t group = sh.n_q_heads / sh.n_kv_heads;
+  const int64_t per_block = static_cast<int64_t>(sh.n_kv_heads) * ((group + 1) / 2);
+  // sum over items of ceil(len / 128) <= ceil(q_rows_total / 128) + n_items
+  // when the items' Q rows do not overlap
+  const int64_t blocks = (q_rows_total + kBlockM - 1) / kBlockM + n_items;
+  if (per_block > 0x7fffffffLL / blocks) return false;
+  DevLayout l;
+  l.max_ctas = blocks * per_block;
+  l.descs = align256(static_cast<size_t>(n_items) * 3 * sizeof(CUtensorMap));
+  l.cta_item = align256(l.descs + static_cast<size_t>(n_items) * sizeof(ItemDesc));
+  l.total = align256(l.cta_item + static_cast<size_t>(l.max_ctas) * sizeof(int32_t));
+  l.bytes = l.total + 256;
+  *out = l;
+  return true;
+}
+
+template <int D>
+mocap_status launch_dev(const void *q, const void *k_cache, const void *v_cache,
+                        const mocap_varlen_item *items, int32_t n_items, int64_t q_rows_total,
+                        int64_t kv_rows_total, const Shape &sh, float scale, void *out, float *lse,
+                        const DevLayout &dl, void *workspace, cudaStream_t stream) {
+  static AttnParams<1> prm;  // large: built in static storage, guarded below
+  static DevPrep prep;
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lock(mu);
+  std::memset(&prm, 0, sizeof(prm));
+  std::memset(&prep, 0, sizeof(prep));
+  uint32_t *status = device_status_ptr();
+  if (status == nullptr) return MOCAP_ECUDA;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
+  const int group = sh.n_q_heads / sh.n_kv_heads;
+  const int pairs = (group + 1) / 2;
+  const bool pair = D == 128 && group % 4 == 0 && pair_enabled();
+  // templates over the whole buffers; the prepare kernel sets each item's
+  // first row and row count
+  const int64_t q_rows = std::min<int64_t>(std::max<int64_t>(q_rows_total, 1), kMaxRows);
+  const int64_t kv_rows = std::min<int64_t>(std::max<int64_t>(kv_rows_total, 1), kMaxRows);
+  if (!make_map(&prep.tq, q, q_rows, sh.n_q_heads, D) ||
+      !make_map(&prep.tk, k_cache, kv_rows, sh.n_kv_heads, D, pair ? kBlockN / 2 : kBlockN) ||
+      !make_map(&prep.tv, v_cache, kv_rows, sh.n_kv_heads, D))
+    return MOCAP_ECUDA;
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  int32_t *cta_item = reinterpret_cast<int32_t *>(ws + dl.cta_item);
+  prep.items = items;
+  prep.descs = reinterpret_cast<ItemDesc *>(ws + dl.descs);
+  prep.maps = reinterpret_cast<CUtensorMap *>(ws);
+  prep.total = reinterpret_cast<int32_t *>(ws + dl.total);
+  prep.status = status;
+  prep.q = static_cast<const uint8_t *>(q);
+  prep.k = static_cast<const uint8_t *>(k_cache);
+  prep.v = static_cast<const uint8_t *>(v_cache);
+  prep.q_rows_total = q_rows_total;
+  prep.kv_rows_total = kv_rows_total;
+  prep.qrow_bytes = static_cast<int64_t>(sh.n_q_heads) * D * 2;
+  prep.kvrow_bytes = static_cast<int64_t>(sh.n_kv_heads) * D * 2;
+  prep.max_ctas = dl.max_ctas;
+  prep.n_items = n_items;
+  prep.ctas_per_block = sh.n_kv_heads * pairs;
+  varlen_dev_prepare<<<1, kPrepThreads, 0, stream>>>(prep);
+  if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
+  const int64_t fill_blocks = (dl.max_ctas + kFillThreads - 1) / kFillThreads;
+  varlen_dev_fill<<<static_cast<unsigned>(fill_blocks), kFillThreads, 0, stream>>>(
+      prep.descs, n_items, prep.total, cta_item);
+  if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
+
+  prm.out = static_cast<__nv_bfloat16 *>(out);
+  prm.lse = lse;
+  prm.status = status;
+  prm.lse_stride = q_rows_total;
+  prm.n_items = 1;
+  prm.n_q_heads = sh.n_q_heads;
+  prm.n_kv_heads = sh.n_kv_heads;
+  prm.heads_per_group = group;
+  prm.pairs_per_group = pairs;
+  prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
+  prm.splits = 1;
+  prm.k_cache_vec = static_cast<uint4 *>(const_cast<void *>(k_cache));
+  prm.v_cache_vec = static_cast<uint4 *>(const_cast<void *>(v_cache));
+  prm.dev_items = prep.descs;
+  prm.dev_cta_item = cta_item;
+  prm.dev_maps = prep.maps;
+  prm.dev_total = prep.total;
+  mocap_status st = MOCAP_OK;
+  bool launched = false;
+  if constexpr (D == 128) {
+    if (pair) {
+      if (dl.max_ctas % 2 != 0) return MOCAP_EINVAL;  // whole pairs by construction
+      static bool done[64] = {};
+      st = start_attn(chunk_attn_kernel<D, 1, true, false, true>, prm, dl.max_ctas, true,
+                      Layout<D, true>::kBytes, done, dev, stream);
+      launched = true;
+    }
+  }
+  if (!launched) {
+    static bool done[64] = {};
+    st = start_attn(chunk_attn_kernel<D, 1, false, false, true>, prm, dl.max_ctas, false,
+                    Layout<D>::kBytes, done, dev, stream);
+  }
+  if (st != MOCAP_OK) return st;
+  return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+}
 
 }  // namespace
 
@@ -525,6 +649,44 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
                                                 size_t workspace_bytes, mocap_stream_t stream) {
   return varlen_impl(q, k_cache, v_cache, items, n_items, q_rows_total, kv_rows_total, n_q_heads,
                      n_kv_heads, head_dim, scale, out, lse, workspace, workspace_bytes, stream);
+}
+
+extern "C" size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items,
+                                                             int64_t q_rows_total,
+                                                             int32_t n_q_heads,
+                                                             int32_t n_kv_heads,
+                                                             int32_t head_dim) {
+  const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
+  if (mocap::check_shape(sh, 1.0f) != MOCAP_OK) return 0;
+  mocap::DevLayout dl;
+  return mocap::dev_layout(n_items, q_rows_total, sh, &dl) ? dl.bytes : 0;
+}
+
+extern "C" mocap_status mocap_chunk_attn_varlen_dev(
+    const void *q, const void *k_cache, const void *v_cache, const mocap_varlen_item *items,
+    int32_t n_items, int64_t q_rows_total, int64_t kv_rows_total, int32_t n_q_heads,
+    int32_t n_kv_heads, int32_t head_dim, float scale, void *out, float *lse, void *workspace,
+    size_t workspace_bytes, mocap_stream_t stream) {
+  const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
+  const mocap_status st = mocap::check_shape(sh, scale);
+  if (st != MOCAP_OK) return st;
+  if (n_items < 0 || n_items > MOCAP_VARLEN_DEV_MAX_ITEMS) return MOCAP_EINVAL;
+  if (q_rows_total < 0 || kv_rows_total < 0 || q_rows_total > mocap::kMaxRows)
+    return MOCAP_EINVAL;
+  if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
+  if (n_items == 0) return MOCAP_OK;
+  if (items == nullptr || (reinterpret_cast<uintptr_t>(items) & 7u) != 0) return MOCAP_EINVAL;
+  mocap::DevLayout dl;
+  if (!mocap::dev_layout(n_items, q_rows_total, sh, &dl)) return MOCAP_EINVAL;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 127u) != 0 ||
+      workspace_bytes < dl.bytes)
+    return MOCAP_EINVAL;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (head_dim == 128)
+    return mocap::launch_dev<128>(q, k_cache, v_cache, items, n_items, q_rows_total,
+                                  kv_rows_total, sh, scale, out, lse, dl, workspace, s);
+  return mocap::launch_dev<64>(q, k_cache, v_cache, items, n_items, q_rows_total, kv_rows_total,
+                               sh, scale, out, lse, dl, workspace, s);
 }
 
 extern "C" mocap_status mocap_chunk_attn_varlen_append(

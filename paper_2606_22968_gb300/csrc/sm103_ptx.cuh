@@ -149,6 +149,15 @@ __device__ __forceinline__ void prefetch_tmap(const CUtensorMap *map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// A tensor map that generic-proxy writes built in global memory (for example
+// tensormap.replace in an earlier kernel): order those writes before this
+// thread's tensormap-proxy uses of the 128-byte object.
+__device__ __forceinline__ void tmap_acquire(const CUtensorMap *map) {
+  asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(
+                   reinterpret_cast<uint64_t>(map))
+               : "memory");
+}
+
 // 3-D tiled load into shared memory, completion counted on `bar` in bytes.
 // c0 is the innermost coordinate (elements); it must be a multiple of 8 for
 // bf16 (16-byte rule).  Out-of-range rows are zero-filled by the hardware.

@@ -163,6 +163,45 @@ def test_varlen_rejects_bad_items_before_launch(lib):
     assert call([(0, 0, 5, 0)]) == 0                     # empty item: no-op
 
 
+def test_varlen_dev_argument_checks(lib):
+    """mocap_chunk_attn_varlen_dev: everything checkable on the host fails
+    before any CUDA call; n_items == 0 is a no-op."""
+    f = lib.mocap_chunk_attn_varlen_dev
+    need = lib.mocap_chunk_attn_varlen_dev_workspace_size(3, 1000, 64, 8, 128)
+
+    def call(n=3, items=FAKE, q_rows=1000, ws=FAKE, ws_bytes=None, d=128):
+        return f(FAKE, FAKE, FAKE, items, n, q_rows, 1000, 64, 8, d, 0.1, FAKE, FAKE, ws,
+                 need if ws_bytes is None else ws_bytes, None)
+
+    assert call(n=0) == 0
+    assert call(n=65537) == 1
+    assert call(n=-1) == 1
+    assert call(items=None) == 1
+    assert call(items=FAKE + 4) == 1                     # items not 8-byte aligned
+    assert call(ws=None) == 1
+    assert call(ws=FAKE + 16) == 1                       # workspace not 128-byte aligned
+    assert call(ws_bytes=need - 1) == 1
+    assert call(q_rows=2 ** 31) == 1
+    assert call(d=96) == 3
+
+
+def test_varlen_dev_workspace_layout(lib):
+    """Tensor maps (3 x 128 B per item), 24-byte item descriptors, one int32
+    per CTA of the grid bound (ceil(q_rows / 128) + n) x Hkv x ceil(group / 2),
+    the count; each section 256-byte aligned."""
+    def expect(n, q_rows, hq, hkv):
+        a = lambda x: (x + 255) // 256 * 256
+        ctas = ((q_rows + 127) // 128 + n) * hkv * ((hq // hkv + 1) // 2)
+        return a(a(a(n * 384) + n * 24) + ctas * 4) + 256
+    for n, q_rows, hq, hkv, d in [(3, 1000, 64, 8, 128), (1, 0, 4, 4, 64), (300, 70784, 32, 8, 128),
+                                  (65536, 1 << 20, 6, 2, 128)]:
+        assert lib.mocap_chunk_attn_varlen_dev_workspace_size(n, q_rows, hq, hkv, d) == \
+            expect(n, q_rows, hq, hkv)
+    assert lib.mocap_chunk_attn_varlen_dev_workspace_size(0, 1000, 64, 8, 128) == 0
+    assert lib.mocap_chunk_attn_varlen_dev_workspace_size(65537, 1000, 64, 8, 128) == 0
+    assert lib.mocap_chunk_attn_varlen_dev_workspace_size(3, 1000, 64, 8, 96) == 0
+
+
 def test_workspace_size_split_plan(lib):
     # many row blocks: no split; few long row blocks: a split and its layout
     assert lib.mocap_chunk_attn_workspace_size(0, 23168, 64, 8, 128) == 0
