@@ -263,3 +263,53 @@ def test_no_items_and_empty_items(m):
     assert m.mocap_last_device_status() == 0
     assert bool((out.float() == 5.0).all()) and bool((lse == 5.0).all())
     assert none.numel() == 0
+
+
+@pytest.mark.parametrize("case", range(20))
+def test_random_device_items_sweep(m, monkeypatch, case):
+    """Seeded random launches of 1..400 device items (some empty, random
+    prefixes, items in random order), heads, head dim and kernel form drawn
+    per case: bitwise equal to the host-array form, rows outside every item
+    untouched; in a third of the cases one item is made invalid, and then
+    the call writes nothing and reports MOCAP_EINVAL."""
+    rng = np.random.default_rng(9100 + case)
+    heads = [(4, 4), (8, 2), (16, 2), (32, 8), (16, 1), (6, 2)]
+    hq, hkv = heads[int(rng.integers(len(heads)))]
+    d = 128 if rng.random() < 0.7 else 64
+    monkeypatch.setenv("MOCAP_ATTN_PAIR", str(int(rng.integers(2))))
+    n_req = int(rng.choice([1, int(rng.integers(2, 65)), int(rng.integers(65, 401))]))
+    lens = [int(x) for x in rng.integers(1, 800 if n_req > 64 else 3000, n_req)]
+    cu = np.concatenate([[0], np.cumsum(lens)]).tolist()
+    t = cu[-1]
+    items = []
+    for r, n in enumerate(lens):
+        pre = int(rng.integers(0, n))
+        ln = int(rng.integers(0, n - pre + 1)) if rng.random() < 0.9 else 0
+        items.append((cu[r] + pre, cu[r], pre, ln))
+    items = [items[i] for i in rng.permutation(len(items))]
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(9100 + case)
+    q = torch.randn((t, hq, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    k = torch.randn((t, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    v = torch.randn((t, hkv, d), generator=gen, device=dev, dtype=torch.bfloat16)
+    scale = 1.0 / math.sqrt(d)
+    if case % 3 == 2:
+        j = int(rng.integers(len(items)))
+        qr, kr, pre, ln = items[j]
+        items[j] = (qr, kr, pre, t + 1)  # rows past both buffers
+        out = torch.full((t, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
+        lse = torch.full((hq, t), float("nan"), device=dev, dtype=torch.float32)
+        it = torch.tensor(items, dtype=torch.int64, device=dev)
+        m.mocap_chunk_attn_varlen_dev(q, k, v, it, out, lse, scale)
+        torch.cuda.synchronize()
+        assert m.mocap_last_device_status() == m.MOCAP_EINVAL
+        assert torch.isnan(out.float()).all() and torch.isnan(lse).all()
+        return
+    out_d, lse_d, out_h, lse_h = _run_both(m, q, k, v, items, scale)
+    assert _equal_bits(out_d, out_h) and _equal_bits(lse_d, lse_h)
+    covered = torch.zeros(t, dtype=torch.bool)
+    for (qr, _, _, ln) in items:
+        covered[qr:qr + ln] = True
+    cov = covered.to(dev)
+    assert torch.isnan(out_d[~cov].float()).all() and torch.isnan(lse_d[:, ~cov]).all()
+    assert torch.isfinite(out_d[cov].float()).all()
