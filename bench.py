@@ -568,6 +568,8 @@ def ours_arm(args, rank, world, local):
         if pf.append_mode == "overlap" and len(steps_plan) > 1:
             line["chunk_streams"] = measure_chunk_streams(args, pf, w, q, k, v, dev, stream,
                                                           total_flops)
+    if not pf.single and not args.no_graph:
+        line["varlen_device_items"] = measure_varlen_dev(m, pf, w, q, dev, stream, total_flops)
     if pf.single and not args.no_projection:
         line["qkv_projection"] = measure_projection(args, m, w, pf, q, dev, stream, total_flops,
                                                     peak)
@@ -728,6 +730,73 @@ def measure_chunk_streams(args, pf, w, q, k, v, dev, stream, total_flops, reps=3
             "two_streams_value": total_flops / (two * 1e-3) / 1e12, "unit": "TFLOP/s",
             "note": "attention launches alternating between two compute streams "
                     "(ChunkedPrefill chunk_streams=2), appends beside them; whole prompt "
+                    "replayed from one CUDA graph"}
+
+
+def measure_varlen_dev(m, pf, w, q, dev, stream, total_flops, reps=5):
+    """Multi-request prompts: every step's attention (chunk k of every
+    request, one launch per step, caches already filled by the timed run)
+    with the items as a host array and as a device array
+    (mocap_chunk_attn_varlen_dev: a prepare launch before each attention
+    launch, the grid sized by the step's rows), each prompt replayed from one
+    CUDA graph, interleaved, median of `reps`."""
+    import torch
+    steps = pf.steps()
+    hq, hkv, d = w.n_q_heads, w.n_kv_heads, w.head_dim
+    rows = q.shape[0]
+    host_items, dev_items, spaces = [], [], []
+    for st in steps:
+        its = [(pf.cu[r] + pf.bounds[r][c], pf.cu[r], pf.bounds[r][c],
+                pf.bounds[r][c + 1] - pf.bounds[r][c]) for r, c in st]
+        if len(its) == 1:
+            its.append((0, 0, 0, 0))  # two items: the host form never splits either
+        host_items.append(its)
+        dev_items.append(torch.tensor(its, dtype=torch.int64, device=dev))
+        bound = sum(x[3] for x in its)  # the step's rows: a scheduler's token budget
+        need = m.mocap_chunk_attn_varlen_dev_workspace_size(len(its), bound, hq, hkv, d)
+        spaces.append((torch.empty((need,), device=dev, dtype=torch.uint8), bound))
+    out = torch.empty_like(pf.out)
+    lse = torch.empty((hq, rows), device=dev, dtype=torch.float32)
+
+    def host_prompt():
+        for its in host_items:
+            m.mocap_chunk_attn_varlen(q, pf.k_cache, pf.v_cache, its, out, lse, w.scale)
+
+    def dev_prompt():
+        for it, (ws, bound) in zip(dev_items, spaces):
+            m.mocap_chunk_attn_varlen_dev(q, pf.k_cache, pf.v_cache, it, out, lse, w.scale,
+                                          max_rows=bound, workspace=ws)
+
+    graphs = {}
+    for name, fn in (("host_items", host_prompt), ("device_items", dev_prompt)):
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            fn()
+        stream.wait_stream(side)
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            fn()
+        graphs[name] = g
+    times = {n: [] for n in graphs}
+    for _ in range(reps):
+        for n, g in graphs.items():
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            g.replay()
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            times[n].append(e0.elapsed_time(e1))
+    if m.mocap_last_device_status() != m.MOCAP_OK:
+        raise RuntimeError("device status set in the device-item measurement")
+    res = {n: statistics.median(t) for n, t in times.items()}
+    return {"host_items_ms": res["host_items"], "device_items_ms": res["device_items"],
+            "device_items_tflops": total_flops / (res["device_items"] * 1e-3) / 1e12,
+            "note": "every step's attention launch (one compute stream, no appends), items as "
+                    "a host array vs in device memory (a prepare launch per step, grid bounded "
+                    "by the step's rows); prompt "
                     "replayed from one CUDA graph"}
 
 

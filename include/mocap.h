@@ -406,14 +406,15 @@ mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cache, const v
 
 /*
  * mocap_chunk_attn_varlen_dev_workspace_size -- bytes of device scratch that
- * mocap_chunk_attn_varlen_dev needs for up to n_items items over packed
- * q / out buffers of q_rows_total rows: per item its three TMA tensor maps
- * (384 B) and descriptor, one 4-byte entry per CTA of the launch's grid
- * (at most (ceil(q_rows_total / 128) + n_items) x n_kv_heads x
- * ceil(n_q_heads / n_kv_heads / 2) CTAs) and the CTA count.  0 when
- * n_items == 0 or an argument is out of range.
+ * mocap_chunk_attn_varlen_dev needs for n_items items whose lengths add up
+ * to at most max_rows: per item its three TMA tensor maps (384 B) and
+ * descriptor, one 4-byte entry per CTA of the launch's grid, which has
+ * (ceil(max_rows / 128) + n_items) x n_kv_heads x
+ * ceil(n_q_heads / n_kv_heads / 2) CTAs, and the CTA count.  0 when
+ * n_items == 0 or an argument is out of range (max_rows outside
+ * [0, 2^31 - 1], n_items above MOCAP_VARLEN_DEV_MAX_ITEMS, a bad shape).
  */
-size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items, int64_t q_rows_total,
+size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items, int64_t max_rows,
                                                   int32_t n_q_heads, int32_t n_kv_heads,
                                                   int32_t head_dim);
 
@@ -427,17 +428,21 @@ size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items, int64_t q_row
  *   items        DEVICE array of n_items mocap_varlen_item (8-byte aligned),
  *                read by the launch; the caller keeps it unchanged until the
  *                work queued on `stream` has started past it
+ *   max_rows     an upper bound on the sum of the items' len (a step's token
+ *                budget; q_rows_total always serves).  It sizes the launch
+ *                grid and the workspace: a tight bound spares the launch
+ *                CTAs that find no work and exit.
  *   workspace, workspace_bytes: caller-owned device scratch, 128-byte
  *                aligned, at least mocap_chunk_attn_varlen_dev_workspace_size
- *                (n_items, q_rows_total, ...) bytes; overwritten by the call
+ *                (n_items, max_rows, ...) bytes; overwritten by the call
  *   other arguments as mocap_chunk_attn_varlen.
  *
- * Three launches on `stream`: a one-block kernel validates the items, counts
- * and scans their CTAs and builds each item's tensor maps (tensormap.replace
+ * Two launches on `stream`: a one-block kernel validates the items, counts
+ * and scans their CTAs, builds each item's tensor maps (tensormap.replace
  * of the global address and row extent of templates the host encodes over
- * the whole buffers); a second fills the CTA -> item table; then the
- * attention kernel, on a grid of the upper bound above, whose surplus CTAs
- * exit at once.  Per item the results are bitwise those of
+ * the whole buffers) and fills the CTA -> item table; then the attention
+ * kernel, on the grid above, whose CTAs past the items' count exit at once.
+ * Per item the results are bitwise those of
  * mocap_chunk_attn_varlen with two or more items (this form never splits a
  * key range).  CTAs follow the items in the order given: put the items with
  * the most keys first (the host-array form sorts them so itself).
@@ -447,8 +452,9 @@ size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items, int64_t q_row
  * null or misaligned items array, a missing, misaligned or short workspace
  * -> MOCAP_EINVAL.  An item that fails mocap_chunk_attn_varlen's item checks
  * (negative field, rows outside q_rows_total / kv_rows_total,
- * prefix + len >= 2^31), or items whose Q rows overlap beyond the grid's
- * bound, are found on the device: the call then writes nothing and records
+ * prefix + len >= 2^31), or items that need more CTAs than the grid has
+ * (their lengths exceed max_rows), are found on the device: the call then
+ * writes nothing and records
  * MOCAP_EINVAL in the status word that mocap_last_device_status returns (and
  * clears); until then later launches do nothing, as after an expired wait.
  * Items must not write overlapping output rows.  n_items == 0 is a no-op.
@@ -456,6 +462,7 @@ size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items, int64_t q_row
 mocap_status mocap_chunk_attn_varlen_dev(const void *q, const void *k_cache, const void *v_cache,
                                          const mocap_varlen_item *items, int32_t n_items,
                                          int64_t q_rows_total, int64_t kv_rows_total,
+                                         int64_t max_rows,
                                          int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim,
                                          float scale, void *out, float *lse, void *workspace,
                                          size_t workspace_bytes, mocap_stream_t stream);

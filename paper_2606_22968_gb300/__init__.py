@@ -193,18 +193,20 @@ def mocap_chunk_attn_varlen(q, k_cache, v_cache, items: Sequence[tuple], out, ls
            "mocap_chunk_attn_varlen")
 
 
-def mocap_chunk_attn_varlen_dev_workspace_size(n_items: int, q_rows_total: int, n_q_heads: int,
+def mocap_chunk_attn_varlen_dev_workspace_size(n_items: int, max_rows: int, n_q_heads: int,
                                                n_kv_heads: int, head_dim: int) -> int:
-    """Bytes of scratch mocap_chunk_attn_varlen_dev needs (0: n_items == 0 or out of range)."""
+    """Bytes of scratch mocap_chunk_attn_varlen_dev needs for n_items items of
+    at most max_rows rows in all (0: n_items == 0 or out of range)."""
     return int(_lib.load().mocap_chunk_attn_varlen_dev_workspace_size(
-        n_items, q_rows_total, n_q_heads, n_kv_heads, head_dim))
+        n_items, max_rows, n_q_heads, n_kv_heads, head_dim))
 
 
 def mocap_chunk_attn_varlen_dev(q, k_cache, v_cache, items, out, lse, scale: float,
-                                workspace=None, stream=None):
+                                max_rows=None, workspace=None, stream=None):
     """mocap_chunk_attn_varlen with the items in device memory: ``items`` is a
     contiguous int64 tensor [n, 4] of (q_row, kv_row, prefix, len) rows on the
-    device; lse is [Hq, q_rows_total].  ``workspace``: a uint8 device tensor of
+    device; lse is [Hq, q_rows_total].  ``max_rows`` bounds the items' total
+    length (default: all rows of q).  ``workspace``: a uint8 device tensor of
     at least mocap_chunk_attn_varlen_dev_workspace_size bytes (allocated here
     when None).  An invalid item is reported by mocap_last_device_status."""
     import torch
@@ -214,16 +216,18 @@ def mocap_chunk_attn_varlen_dev(q, k_cache, v_cache, items, out, lse, scale: flo
             not items.is_contiguous():
         raise ValueError("items must be a contiguous int64 tensor [n, 4]")
     n = items.shape[0]
-    need = mocap_chunk_attn_varlen_dev_workspace_size(n, q_rows, n_q, n_kv, d)
+    max_rows = q_rows if max_rows is None else int(max_rows)
+    need = mocap_chunk_attn_varlen_dev_workspace_size(n, max_rows, n_q, n_kv, d)
     if workspace is None:
         workspace = torch.empty((max(need, 128),), device=q.device, dtype=torch.uint8)
     if not workspace.is_contiguous():
         raise ValueError("workspace must be contiguous")
     ws_bytes = workspace.numel() * workspace.element_size()
     _check(_lib.load().mocap_chunk_attn_varlen_dev(_ptr(q), _ptr(k_cache), _ptr(v_cache),
-                                                   _ptr(items), n, q_rows, k_cache.shape[0], n_q,
-                                                   n_kv, d, scale, _ptr(out), _ptr(lse),
-                                                   _ptr(workspace), ws_bytes, _stream(stream)),
+                                                   _ptr(items), n, q_rows, k_cache.shape[0],
+                                                   max_rows, n_q, n_kv, d, scale, _ptr(out),
+                                                   _ptr(lse), _ptr(workspace), ws_bytes,
+                                                   _stream(stream)),
            "mocap_chunk_attn_varlen_dev")
 
 

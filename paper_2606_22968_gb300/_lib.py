@@ -44,8 +44,9 @@ SIGNATURES = {
                                         c_i64, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp, c_vp,
                                         c_vp, c_sz, c_vp]),
     "mocap_chunk_attn_varlen_dev_workspace_size": (c_sz, [c_i32, c_i64, c_i32, c_i32, c_i32]),
-    "mocap_chunk_attn_varlen_dev": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i32, c_i64, c_i64, c_i32,
-                                            c_i32, c_i32, c_f32, c_vp, c_vp, c_vp, c_sz, c_vp]),
+    "mocap_chunk_attn_varlen_dev": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i32, c_i64, c_i64, c_i64,
+                                            c_i32, c_i32, c_i32, c_f32, c_vp, c_vp, c_vp, c_sz,
+                                            c_vp]),
     "mocap_chunk_attn_append": (c_i32, [c_vp, c_vp, c_vp, c_i64, c_i64, c_i32, c_i32, c_i32, c_f32,
                                         c_vp, c_vp, c_vp, c_sz, ctypes.POINTER(AppendItem), c_i32,
                                         c_i64, c_vp]),

@@ -129,7 +129,7 @@ struct AttnParams {
   AppendSeg app[kMaxAppends];
   // Device item descriptors (DEV instantiations, items in device memory):
   // the item of every CTA, each item's ItemDesc and three tensor maps, and
-  // the launch's CTA count, all written by the prepare kernels before the
+  // the launch's CTA count, all written by the prepare kernel before the
   // launch (attn_varlen_dev.cuh).  CTAs at or past *dev_total exit at once.
   const ItemDesc *dev_items;
   const int32_t *dev_cta_item;
@@ -775,7 +775,7 @@ __device__ __forceinline__ void cta_barrier() {
 // APPEND: the launch carries KV appends (warps 2-3 copy them).  A separate
 // instantiation, so launches without appends run exactly the code they
 // would without this feature.
-// DEV: the items are device descriptors (the prepare kernels' tables).
+// DEV: the items are device descriptors (the prepare kernel's tables).
 template <int D, int MAXI, bool PAIR = false, bool APPEND = false, bool DEV = false>
 __global__ void __launch_bounds__(kThreads, 1)
     chunk_attn_kernel(const __grid_constant__ AttnParams<MAXI> p) {

@@ -1,11 +1,11 @@
-// attn_varlen_dev.cuh -- the prepare kernels of mocap_chunk_attn_varlen_dev:
+// attn_varlen_dev.cuh -- the prepare kernel of mocap_chunk_attn_varlen_dev:
 // variable-length attention whose (request, chunk) items live in device
 // memory, so a device-side scheduler or a CUDA graph can supply them.
 //
 // Sec. 2.2 / Eq. 1: one launch serves several (request, chunk) items, each a
 // chunk's queries against its request's KV prefix plus itself.  The host
-// cannot read the items without a synchronisation, so two small kernels turn
-// them into what the attention kernel's DEV instantiation reads:
+// cannot read the items without a synchronisation, so a one-block kernel
+// turns them into what the attention kernel's DEV instantiation reads:
 //   varlen_dev_prepare (one block): validates every item, counts its CTAs
 //     (128-row blocks x KV groups x head pairs), scans the counts into each
 //     item's first CTA, and builds the item's Q, K and V tensor maps from
@@ -14,10 +14,10 @@
 //     zero-fills past the item exactly as the per-item maps of the host form
 //     do; then publishes the CTA count (0 after an invalid item, with
 //     MOCAP_EINVAL in the status word).
-//   varlen_dev_fill: the item of every CTA (binary search over the first
-//     CTAs), so an attention CTA finds its item with one load.
-// The attention launch's grid is an upper bound on the CTA count; CTAs past
-// the count exit at once.
+//   then, in the same block, the item of every CTA (binary search over the
+//     first CTAs), so an attention CTA finds its item with one load.
+// The attention launch's grid is an upper bound on the CTA count, from the
+// caller's bound on the items' total rows; CTAs past the count exit at once.
 #pragma once
 
 #include <cuda.h>
@@ -28,13 +28,13 @@ namespace mocap {
 namespace {
 
 constexpr int kPrepThreads = 1024;
-constexpr int kFillThreads = 256;
 
 struct DevPrep {
   CUtensorMap tq, tk, tv;          // templates over the whole Q / K / V buffers
   const mocap_varlen_item *items;  // device, n_items
   ItemDesc *descs;                 // [n_items]
   CUtensorMap *maps;               // [n_items][3]
+  int32_t *cta_item;               // [max_ctas]: the item of each CTA
   int32_t *total;                  // CTA count of the launch
   uint32_t *status;
   const uint8_t *q, *k, *v;
@@ -106,8 +106,8 @@ __global__ void __launch_bounds__(kPrepThreads) varlen_dev_prepare(const __grid_
       __syncthreads();
     }
     if (i < a.n_items) {
-      // every item gets its first CTA, empty ones too (the fill's search
-      // needs them non-decreasing); clamped, the count check below decides
+      // every item gets its first CTA, empty ones too (the CTA table's
+      // search needs them non-decreasing); clamped, the count check decides
       const int64_t begin = carry + scan[tid] - count;
       a.descs[i].cta_begin = static_cast<int32_t>(begin < 0x7fffffffLL ? begin : 0x7fffffffLL);
     }
@@ -117,32 +117,29 @@ __global__ void __launch_bounds__(kPrepThreads) varlen_dev_prepare(const __grid_
   }
   // the maps' generic-proxy writes before any later tensormap-proxy use
   asm volatile("fence.proxy.tensormap::generic.release.gpu;" ::: "memory");
-  __syncthreads();
+  const bool ok = bad == 0 && carry <= a.max_ctas;
+  const int64_t total = ok ? carry : 0;
   if (tid == 0) {
-    const bool ok = bad == 0 && carry <= a.max_ctas;
-    *a.total = ok ? static_cast<int32_t>(carry) : 0;
+    *a.total = static_cast<int32_t>(total);
     if (!ok) atomicCAS(a.status, 0u, static_cast<uint32_t>(MOCAP_EINVAL));
   }
-}
-
-// cta_item[c] = the last item whose first CTA is <= c (items without CTAs
-// share their successor's first CTA, so the last such item is the one that
-// owns c).
-__global__ void __launch_bounds__(kFillThreads)
-    varlen_dev_fill(const ItemDesc *__restrict__ descs, int32_t n_items,
-                    const int32_t *__restrict__ total, int32_t *__restrict__ cta_item) {
-  const int64_t c = static_cast<int64_t>(blockIdx.x) * kFillThreads + threadIdx.x;
-  if (c >= *total) return;
-  int lo = 0, hi = n_items - 1;  // descs[0].cta_begin == 0 <= c
-  while (lo < hi) {
-    const int mid = lo + (hi - lo + 1) / 2;
-    if (descs[mid].cta_begin <= c) {
-      lo = mid;
-    } else {
-      hi = mid - 1;
+  // cta_item[c] = the last item whose first CTA is <= c (items without CTAs
+  // share their successor's first CTA, so the last such item owns c); the
+  // descriptors' first CTAs were written by this block before the barrier
+  // above, and __syncthreads orders them for every thread of it
+  __syncthreads();
+  for (int64_t c = tid; c < total; c += kPrepThreads) {
+    int lo = 0, hi = a.n_items - 1;  // descs[0].cta_begin == 0 <= c
+    while (lo < hi) {
+      const int mid = lo + (hi - lo + 1) / 2;
+      if (a.descs[mid].cta_begin <= c) {
+        lo = mid;
+      } else {
+        hi = mid - 1;
+      }
     }
+    a.cta_item[c] = lo;
   }
-  cta_item[c] = lo;
 }
 
 }  // namespace

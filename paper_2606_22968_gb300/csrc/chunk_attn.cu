@@ -380,15 +380,14 @@ struct DevLayout {
 
 size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
-bool dev_layout(int32_t n_items, int64_t q_rows_total, const Shape &sh, DevLayout *out) {
-  if (n_items < 1 || n_items > MOCAP_VARLEN_DEV_MAX_ITEMS || q_rows_total < 0 ||
-      q_rows_total > kMaxRows)
+bool dev_layout(int32_t n_items, int64_t max_rows, const Shape &sh, DevLayout *out) {
+  if (n_items < 1 || n_items > MOCAP_VARLEN_DEV_MAX_ITEMS || max_rows < 0 || max_rows > kMaxRows)
     return false;
   const int64_t group = sh.n_q_heads / sh.n_kv_heads;
   const int64_t per_block = static_cast<int64_t>(sh.n_kv_heads) * ((group + 1) / 2);
-  // sum over items of ceil(len / 128) <= ceil(q_rows_total / 128) + n_items
-  // when the items' Q rows do not overlap
-  const int64_t blocks = (q_rows_total + kBlockM - 1) / kBlockM + n_items;
+  // sum over items of ceil(len / 128) <= ceil(max_rows / 128) + n_items when
+  // the items' lengths add up to at most max_rows
+  const int64_t blocks = (max_rows + kBlockM - 1) / kBlockM + n_items;
   if (per_block > 0x7fffffffLL / blocks) return false;
   DevLayout l;
   l.max_ctas = blocks * per_block;
@@ -429,6 +428,7 @@ mocap_status launch_dev(const void *q, const void *k_cache, const void *v_cache,
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   int32_t *cta_item = reinterpret_cast<int32_t *>(ws + dl.cta_item);
   prep.items = items;
+  prep.cta_item = cta_item;
   prep.descs = reinterpret_cast<ItemDesc *>(ws + dl.descs);
   prep.maps = reinterpret_cast<CUtensorMap *>(ws);
   prep.total = reinterpret_cast<int32_t *>(ws + dl.total);
@@ -444,10 +444,6 @@ mocap_status launch_dev(const void *q, const void *k_cache, const void *v_cache,
   prep.n_items = n_items;
   prep.ctas_per_block = sh.n_kv_heads * pairs;
   varlen_dev_prepare<<<1, kPrepThreads, 0, stream>>>(prep);
-  if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
-  const int64_t fill_blocks = (dl.max_ctas + kFillThreads - 1) / kFillThreads;
-  varlen_dev_fill<<<static_cast<unsigned>(fill_blocks), kFillThreads, 0, stream>>>(
-      prep.descs, n_items, prep.total, cta_item);
   if (cudaGetLastError() != cudaSuccess) return MOCAP_ECUDA;
 
   prm.out = static_cast<__nv_bfloat16 *>(out);
@@ -651,33 +647,33 @@ extern "C" mocap_status mocap_chunk_attn_varlen(const void *q, const void *k_cac
                      n_kv_heads, head_dim, scale, out, lse, workspace, workspace_bytes, stream);
 }
 
-extern "C" size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items,
-                                                             int64_t q_rows_total,
+extern "C" size_t mocap_chunk_attn_varlen_dev_workspace_size(int32_t n_items, int64_t max_rows,
                                                              int32_t n_q_heads,
                                                              int32_t n_kv_heads,
                                                              int32_t head_dim) {
   const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
   if (mocap::check_shape(sh, 1.0f) != MOCAP_OK) return 0;
   mocap::DevLayout dl;
-  return mocap::dev_layout(n_items, q_rows_total, sh, &dl) ? dl.bytes : 0;
+  return mocap::dev_layout(n_items, max_rows, sh, &dl) ? dl.bytes : 0;
 }
 
 extern "C" mocap_status mocap_chunk_attn_varlen_dev(
     const void *q, const void *k_cache, const void *v_cache, const mocap_varlen_item *items,
-    int32_t n_items, int64_t q_rows_total, int64_t kv_rows_total, int32_t n_q_heads,
-    int32_t n_kv_heads, int32_t head_dim, float scale, void *out, float *lse, void *workspace,
-    size_t workspace_bytes, mocap_stream_t stream) {
+    int32_t n_items, int64_t q_rows_total, int64_t kv_rows_total, int64_t max_rows,
+    int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim, float scale, void *out, float *lse,
+    void *workspace, size_t workspace_bytes, mocap_stream_t stream) {
   const mocap::Shape sh{n_q_heads, n_kv_heads, head_dim};
   const mocap_status st = mocap::check_shape(sh, scale);
   if (st != MOCAP_OK) return st;
   if (n_items < 0 || n_items > MOCAP_VARLEN_DEV_MAX_ITEMS) return MOCAP_EINVAL;
   if (q_rows_total < 0 || kv_rows_total < 0 || q_rows_total > mocap::kMaxRows)
     return MOCAP_EINVAL;
+  if (max_rows < 0 || max_rows > mocap::kMaxRows) return MOCAP_EINVAL;
   if (!mocap::pointers_ok(q, k_cache, v_cache, out, lse)) return MOCAP_EINVAL;
   if (n_items == 0) return MOCAP_OK;
   if (items == nullptr || (reinterpret_cast<uintptr_t>(items) & 7u) != 0) return MOCAP_EINVAL;
   mocap::DevLayout dl;
-  if (!mocap::dev_layout(n_items, q_rows_total, sh, &dl)) return MOCAP_EINVAL;
+  if (!mocap::dev_layout(n_items, max_rows, sh, &dl)) return MOCAP_EINVAL;
   if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & 127u) != 0 ||
       workspace_bytes < dl.bytes)
     return MOCAP_EINVAL;

@@ -169,9 +169,9 @@ def test_varlen_dev_argument_checks(lib):
     f = lib.mocap_chunk_attn_varlen_dev
     need = lib.mocap_chunk_attn_varlen_dev_workspace_size(3, 1000, 64, 8, 128)
 
-    def call(n=3, items=FAKE, q_rows=1000, ws=FAKE, ws_bytes=None, d=128):
-        return f(FAKE, FAKE, FAKE, items, n, q_rows, 1000, 64, 8, d, 0.1, FAKE, FAKE, ws,
-                 need if ws_bytes is None else ws_bytes, None)
+    def call(n=3, items=FAKE, q_rows=1000, max_rows=1000, ws=FAKE, ws_bytes=None, d=128):
+        return f(FAKE, FAKE, FAKE, items, n, q_rows, 1000, max_rows, 64, 8, d, 0.1, FAKE, FAKE,
+                 ws, need if ws_bytes is None else ws_bytes, None)
 
     assert call(n=0) == 0
     assert call(n=65537) == 1
@@ -182,21 +182,24 @@ def test_varlen_dev_argument_checks(lib):
     assert call(ws=FAKE + 16) == 1                       # workspace not 128-byte aligned
     assert call(ws_bytes=need - 1) == 1
     assert call(q_rows=2 ** 31) == 1
+    assert call(max_rows=-1) == 1
+    assert call(max_rows=2 ** 31) == 1
+    assert call(max_rows=2000) == 1                      # workspace sized for 1000 rows
     assert call(d=96) == 3
 
 
 def test_varlen_dev_workspace_layout(lib):
     """Tensor maps (3 x 128 B per item), 24-byte item descriptors, one int32
-    per CTA of the grid bound (ceil(q_rows / 128) + n) x Hkv x ceil(group / 2),
+    per CTA of the grid (ceil(max_rows / 128) + n) x Hkv x ceil(group / 2),
     the count; each section 256-byte aligned."""
-    def expect(n, q_rows, hq, hkv):
+    def expect(n, max_rows, hq, hkv):
         a = lambda x: (x + 255) // 256 * 256
-        ctas = ((q_rows + 127) // 128 + n) * hkv * ((hq // hkv + 1) // 2)
+        ctas = ((max_rows + 127) // 128 + n) * hkv * ((hq // hkv + 1) // 2)
         return a(a(a(n * 384) + n * 24) + ctas * 4) + 256
-    for n, q_rows, hq, hkv, d in [(3, 1000, 64, 8, 128), (1, 0, 4, 4, 64), (300, 70784, 32, 8, 128),
-                                  (65536, 1 << 20, 6, 2, 128)]:
-        assert lib.mocap_chunk_attn_varlen_dev_workspace_size(n, q_rows, hq, hkv, d) == \
-            expect(n, q_rows, hq, hkv)
+    for n, max_rows, hq, hkv, d in [(3, 1000, 64, 8, 128), (1, 0, 4, 4, 64),
+                                    (300, 70784, 32, 8, 128), (65536, 1 << 20, 6, 2, 128)]:
+        assert lib.mocap_chunk_attn_varlen_dev_workspace_size(n, max_rows, hq, hkv, d) == \
+            expect(n, max_rows, hq, hkv)
     assert lib.mocap_chunk_attn_varlen_dev_workspace_size(0, 1000, 64, 8, 128) == 0
     assert lib.mocap_chunk_attn_varlen_dev_workspace_size(65537, 1000, 64, 8, 128) == 0
     assert lib.mocap_chunk_attn_varlen_dev_workspace_size(3, 1000, 64, 8, 96) == 0

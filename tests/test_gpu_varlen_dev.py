@@ -48,14 +48,17 @@ def _all_chunk_items(starts, bounds):
     return items
 
 
-def _run_both(m, q, k, v, items, scale, host=True):
+def _run_both(m, q, k, v, items, scale, host=True, tight=True):
+    """The device-item call (grid bound: the items' total length when
+    ``tight``, else every row of q) and the host-array form."""
     dev = q.device
     hq, d = q.shape[1], q.shape[2]
     rows = q.shape[0]
     out_d = torch.full((rows, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
     lse_d = torch.full((hq, rows), float("nan"), device=dev, dtype=torch.float32)
     it = torch.tensor(items, dtype=torch.int64, device=dev).reshape(-1, 4)
-    m.mocap_chunk_attn_varlen_dev(q, k, v, it, out_d, lse_d, scale)
+    bound = sum(x[3] for x in items) if tight else None
+    m.mocap_chunk_attn_varlen_dev(q, k, v, it, out_d, lse_d, scale, max_rows=bound)
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == 0
     if not host:
@@ -98,10 +101,11 @@ def test_device_items_bitwise_equal_to_host_items(m, hq, hkv, d, seed):
     items = _all_chunk_items(starts, bounds)
     items.insert(2, (total, 0, 0, 0))  # an empty item in the middle
     scale = 1.0 / math.sqrt(d)
-    out_d, lse_d, out_h, lse_h = _run_both(m, q, k, v, items, scale)
-    assert _equal_bits(out_d, out_h) and _equal_bits(lse_d, lse_h)
-    assert torch.isnan(out_d[total:].float()).all() and torch.isnan(lse_d[:, total:]).all()
-    assert not torch.isnan(out_d[:total].float()).any()
+    for tight in (True, False):
+        out_d, lse_d, out_h, lse_h = _run_both(m, q, k, v, items, scale, tight=tight)
+        assert _equal_bits(out_d, out_h) and _equal_bits(lse_d, lse_h)
+        assert torch.isnan(out_d[total:].float()).all() and torch.isnan(lse_d[:, total:]).all()
+        assert not torch.isnan(out_d[:total].float()).any()
 
 
 def test_three_hundred_items_in_one_launch(m):
@@ -186,9 +190,10 @@ def test_invalid_device_item_is_reported_and_nothing_written(m):
     assert not torch.isnan(out.float()).any()
 
 
-def test_overlapping_items_beyond_the_grid_bound_are_rejected(m):
-    """Items whose Q rows overlap so much that their CTAs exceed the grid's
-    bound: reported as invalid, nothing written."""
+def test_items_beyond_the_grid_bound_are_rejected(m):
+    """Items that need more CTAs than the grid has: overlapping Q rows
+    beyond the default bound, or items longer in all than the caller's
+    max_rows: reported as invalid, nothing written."""
     hq, hkv, d = 8, 2, 128
     dev = torch.device("cuda")
     q = torch.randn((256, hq, d), device=dev).bfloat16()
@@ -201,6 +206,26 @@ def test_overlapping_items_beyond_the_grid_bound_are_rejected(m):
     torch.cuda.synchronize()
     assert m.mocap_last_device_status() == m.MOCAP_EINVAL
     assert torch.isnan(out.float()).all()
+    # a max_rows of 0 leaves one row block per item: 8 items of 32 rows fit
+    items = torch.tensor([(32 * i, 0, 0, 32) for i in range(8)], dtype=torch.int64, device=dev)
+    m.mocap_chunk_attn_varlen_dev(q, k, v, items, out, lse, 0.1, max_rows=0)
+    torch.cuda.synchronize()
+    assert m.mocap_last_device_status() == m.MOCAP_OK
+    assert not torch.isnan(out.float()).any()
+    # two items of 128 and 96 rows (2 row blocks) against max_rows = 0
+    # (0 + 2 = 2 blocks): fit; 129 + 95 rows (3 blocks): do not
+    for rows_a, ok in ((128, True), (129, False)):
+        out.fill_(float("nan"))
+        items = torch.tensor([(0, 0, 0, rows_a), (rows_a, 0, 0, 224 - rows_a)],
+                             dtype=torch.int64, device=dev)
+        m.mocap_chunk_attn_varlen_dev(q, k, v, items, out, lse, 0.1, max_rows=0)
+        torch.cuda.synchronize()
+        if ok:
+            assert m.mocap_last_device_status() == m.MOCAP_OK
+            assert not torch.isnan(out[:224].float()).any()
+        else:
+            assert m.mocap_last_device_status() == m.MOCAP_EINVAL
+            assert torch.isnan(out.float()).all()
 
 
 def test_graph_replay_with_new_device_items(m):
@@ -223,7 +248,7 @@ def test_graph_replay_with_new_device_items(m):
     items = torch.tensor(first, dtype=torch.int64, device=dev)
     out = torch.full((total, hq, d), float("nan"), device=dev, dtype=torch.bfloat16)
     lse = torch.full((hq, total), float("nan"), device=dev, dtype=torch.float32)
-    need = m.mocap_chunk_attn_varlen_dev_workspace_size(len(first), total, hq, hkv, d)
+    need = m.mocap_chunk_attn_varlen_dev_workspace_size(len(first), total, hq, hkv, d)  # max_rows = all rows
     ws = torch.empty((need,), device=dev, dtype=torch.uint8)
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
@@ -255,7 +280,7 @@ def test_no_items_and_empty_items(m):
     lib = m._lib.load()
     stream = torch.cuda.current_stream().cuda_stream
     assert lib.mocap_chunk_attn_varlen_dev(q.data_ptr(), k.data_ptr(), k.data_ptr(), None, 0, 64,
-                                           64, 8, 2, 128, 0.1, out.data_ptr(), lse.data_ptr(),
+                                           64, 64, 8, 2, 128, 0.1, out.data_ptr(), lse.data_ptr(),
                                            None, 0, stream) == 0
     empty = torch.tensor([(0, 0, 10, 0), (5, 3, 0, 0)], dtype=torch.int64, device=dev)
     m.mocap_chunk_attn_varlen_dev(q, k, k, empty, out, lse, 0.1)
