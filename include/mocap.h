@@ -40,6 +40,12 @@
  *   - Arguments are validated before any launch; on MOCAP_EINVAL or
  *     MOCAP_EUNSUPPORTED nothing was enqueued.  MOCAP_ECUDA reports a failed
  *     CUDA call or launch (the launch error is consumed).
+ *   - Per-device state (the status word's address, kernel attributes set on
+ *     first use, the no-allocation scratch address) is cached by device
+ *     ordinal: the library works in each device's primary context, the one
+ *     the CUDA runtime API uses, not in a context the caller created.
+ *   - Entry points may be called from several host threads; launches that
+ *     share a caller workspace must not overlap on the GPU.
  */
 #ifndef MOCAP_H_
 #define MOCAP_H_
