@@ -40,10 +40,12 @@
  *   - Arguments are validated before any launch; on MOCAP_EINVAL or
  *     MOCAP_EUNSUPPORTED nothing was enqueued.  MOCAP_ECUDA reports a failed
  *     CUDA call or launch (the launch error is consumed).
- *   - Per-device state (the status word's address, kernel attributes set on
- *     first use, the no-allocation scratch address) is cached by device
- *     ordinal: the library works in each device's primary context, the one
- *     the CUDA runtime API uses, not in a context the caller created.
+ *   - Calls run in the CUDA context current on the calling thread: the
+ *     device's primary context (the CUDA runtime API's), or one the caller
+ *     made current with the driver API.  State that belongs to a context
+ *     (the status word's address, kernel attributes set on first use, the
+ *     no-allocation scratch address) is set up once per context, on its
+ *     first call, which should come before any stream capture.
  *   - Entry points may be called from several host threads; launches that
  *     share a caller workspace must not overlap on the GPU.
  */
@@ -343,14 +345,11 @@ size_t mocap_chunk_attn_workspace_size(int64_t prefix, int64_t len, int32_t n_q_
  *     too small a workspace: the same results up to fp32 rounding order, but
  *     a late chunk's last wave may leave SMs idle.  Shapes that need no split
  *     run the single-pass kernel too and use no scratch.
- *   - Every GPU that loads the library holds the array until the process
- *     exits.  The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress, once per device, that device current); make
- *     that first call before any stream capture.  The address is kept per
- *     device ordinal: the entry point assumes each device's primary context
- *     (the one the CUDA runtime API uses), not a context the caller created
- *     with the driver API.
- *   - All calls on a device share the array.  A call writes every scratch
+ *   - Every CUDA context that loads the library holds its own copy of the
+ *     array until the context ends.  The first call in a context looks up
+ *     the array's device address (cudaGetSymbolAddress, once per context);
+ *     make that first call before any stream capture.
+ *   - All calls in a context share the array.  A call writes every scratch
  *     byte it reads, so nothing has to start at zero, but calls whose work
  *     overlaps on the GPU (e.g. on different streams) race on the array.
  */

@@ -163,20 +163,22 @@ bool pair_enabled() {
 }
 
 // One attention launch of `kern` with `prm` on `ctas` CTAs, as CTA pairs
-// (clusters of two) or single CTAs.  Once per kernel and device (`done`):
+// (clusters of two) or single CTAs.  Once per kernel and context (`once`):
 // the register-count check (the setmaxnreg split assumes kLaunchRegs) and
 // the dynamic shared-memory limit.
 template <typename Kern, typename P>
-mocap_status start_attn(Kern kern, const P &prm, int64_t ctas, bool as_pair, int smem, bool *done,
-                        int dev, cudaStream_t stream) {
-  if (!done[dev]) {
+mocap_status start_attn(Kern kern, const P &prm, int64_t ctas, bool as_pair, int smem,
+                        ContextOnce &once, cudaStream_t stream) {
+  const uint64_t ctx = current_context();
+  if (ctx == 0) return MOCAP_ECUDA;
+  if (!once.done(ctx)) {
     cudaFuncAttributes fa{};
     if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess) return MOCAP_ECUDA;
     if (fa.numRegs != kLaunchRegs) return MOCAP_EUNSUPPORTED;  // split would not balance
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
         cudaSuccess)
       return MOCAP_ECUDA;
-    done[dev] = true;
+    once.mark(ctx);
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(ctas));
@@ -265,11 +267,9 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     prm.app_total += 2 * g.n_vec;
   }
 
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
   // the CTA-pair or single-CTA form, each with or without the append copy
-  auto launch_form = [&](auto kern, bool as_pair, int smem, bool *done) -> mocap_status {
-    return start_attn(kern, prm, ctas, as_pair, smem, done, dev, stream);
+  auto launch_form = [&](auto kern, bool as_pair, int smem, ContextOnce &once) -> mocap_status {
+    return start_attn(kern, prm, ctas, as_pair, smem, once, stream);
   };
   const bool append = prm.n_app > 0;
   mocap_status lst = MOCAP_OK;
@@ -279,22 +279,22 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
       if (ctas % 2 != 0) return MOCAP_EINVAL;  // whole pairs by construction
       constexpr int kSmem = Layout<D, true>::kBytes;
       if (append) {
-        static bool done[64] = {};
-        lst = launch_form(chunk_attn_kernel<D, MAXI, true, true>, true, kSmem, done);
+        static ContextOnce once;
+        lst = launch_form(chunk_attn_kernel<D, MAXI, true, true>, true, kSmem, once);
       } else {
-        static bool done[64] = {};
-        lst = launch_form(chunk_attn_kernel<D, MAXI, true, false>, true, kSmem, done);
+        static ContextOnce once;
+        lst = launch_form(chunk_attn_kernel<D, MAXI, true, false>, true, kSmem, once);
       }
       launched = true;
     }
   }
   if (!launched) {
     if (append) {
-      static bool done[64] = {};
-      lst = launch_form(chunk_attn_kernel<D, MAXI, false, true>, false, L::kBytes, done);
+      static ContextOnce once;
+      lst = launch_form(chunk_attn_kernel<D, MAXI, false, true>, false, L::kBytes, once);
     } else {
-      static bool done[64] = {};
-      lst = launch_form(chunk_attn_kernel<D, MAXI, false, false>, false, L::kBytes, done);
+      static ContextOnce once;
+      lst = launch_form(chunk_attn_kernel<D, MAXI, false, false>, false, L::kBytes, once);
     }
   }
   if (lst != MOCAP_OK) return lst;
@@ -306,14 +306,16 @@ mocap_status launch(const void *q, const void *k_cache, const void *v_cache,
     const dim3 grid(static_cast<unsigned>(len),
                     static_cast<unsigned>((sh.n_q_heads + kCombineHeadsPerBlock - 1) /
                                           kCombineHeadsPerBlock));
-    static bool combine_done[64] = {};  // shared-memory limit set, per device
-    if (!combine_done[dev]) {
+    static ContextOnce combine_once;  // shared-memory limit set, per context
+    const uint64_t ctx = current_context();
+    if (ctx == 0) return MOCAP_ECUDA;
+    if (!combine_once.done(ctx)) {
       if (cudaFuncSetAttribute(attn_combine_kernel<D>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize,
                                static_cast<int>(combine_smem_bytes<D>(kMaxSplits))) !=
           cudaSuccess)
         return MOCAP_ECUDA;
-      combine_done[dev] = true;
+      combine_once.mark(ctx);
     }
     attn_combine_kernel<D><<<grid, kCombineThreads, combine_smem_bytes<D>(sp.splits), stream>>>(
         prm.o_part, prm.lse_part, sp.splits, len, sh.n_q_heads,
@@ -412,8 +414,6 @@ mocap_status launch_dev(const void *q, const void *k_cache, const void *v_cache,
   std::memset(&prep, 0, sizeof(prep));
   uint32_t *status = device_status_ptr();
   if (status == nullptr) return MOCAP_ECUDA;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
   const int group = sh.n_q_heads / sh.n_kv_heads;
   const int pairs = (group + 1) / 2;
   const bool pair = D == 128 && group % 4 == 0 && pair_enabled();
@@ -468,16 +468,16 @@ mocap_status launch_dev(const void *q, const void *k_cache, const void *v_cache,
   if constexpr (D == 128) {
     if (pair) {
       if (dl.max_ctas % 2 != 0) return MOCAP_EINVAL;  // whole pairs by construction
-      static bool done[64] = {};
+      static ContextOnce once;
       st = start_attn(chunk_attn_kernel<D, 1, true, false, true>, prm, dl.max_ctas, true,
-                      Layout<D, true>::kBytes, done, dev, stream);
+                      Layout<D, true>::kBytes, once, stream);
       launched = true;
     }
   }
   if (!launched) {
-    static bool done[64] = {};
+    static ContextOnce once;
     st = start_attn(chunk_attn_kernel<D, 1, false, false, true>, prm, dl.max_ctas, false,
-                    Layout<D>::kBytes, done, dev, stream);
+                    Layout<D>::kBytes, once, stream);
   }
   if (st != MOCAP_OK) return st;
   return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
@@ -701,32 +701,33 @@ extern "C" mocap_status mocap_chunk_attn_varlen_append(
 // device memory.  The split-KV partials go to a fixed scratch array that is
 // part of this library's device image; nothing is allocated per call.
 //
-// The array belongs to every device that loads the library, from load until
-// process exit, and all calls on a device share it.  Every byte a call reads
-// from it was written earlier in the same call, so nothing needs clearing;
-// two calls whose work overlaps on the GPU (for example on two streams)
-// would overwrite each other's partials.
+// Every context that loads the library holds its own copy of the array, from
+// load until the context ends, and all calls in a context share it.  Every
+// byte a call reads from it was written earlier in the same call, so nothing
+// needs clearing; two calls whose work overlaps on the GPU (for example on
+// two streams) would overwrite each other's partials.
 static __device__ __align__(256) uint8_t g_noalloc_scratch[MOCAP_NOALLOC_SCRATCH_BYTES];
 
 namespace {
-uint8_t *g_noalloc_ptr[64] = {};
+std::vector<std::pair<uint64_t, uint8_t *>> g_noalloc_ptr;  // per context ID
 std::mutex g_noalloc_mu;
 
-// Device address of g_noalloc_scratch on the current device.  The name is
+// Device address of g_noalloc_scratch in the current context.  The name is
 // only a host-side handle in host code, so the address is looked up once per
-// device (that device current) and cached; nullptr if the lookup fails.  The
-// cache is keyed by device ordinal, i.e. it assumes the CUDA runtime's primary
-// context of each device (the context every runtime-API caller uses).
+// context and cached; nullptr if the lookup fails.  The status word is
+// resolved first, which binds the runtime's context to the thread if none
+// was current.
 uint8_t *noalloc_scratch() {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  if (mocap::device_status_ptr() == nullptr) return nullptr;
+  const uint64_t ctx = mocap::current_context();
+  if (ctx == 0) return nullptr;
   std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (g_noalloc_ptr[dev] == nullptr) {
-    void *ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess) return nullptr;
-    g_noalloc_ptr[dev] = static_cast<uint8_t *>(ptr);
-  }
-  return g_noalloc_ptr[dev];
+  for (const auto &e : g_noalloc_ptr)
+    if (e.first == ctx) return e.second;
+  void *ptr = nullptr;
+  if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess) return nullptr;
+  g_noalloc_ptr.emplace_back(ctx, static_cast<uint8_t *>(ptr));
+  return static_cast<uint8_t *>(ptr);
 }
 }  // namespace
 

@@ -553,24 +553,24 @@ extern "C" mocap_status mocap_last_row_attn(const void *q_last, const void *k_ca
                       st) != cudaSuccess)
     return MOCAP_ECUDA;
   const dim3 grid(splits, n_req, n_kv_heads);
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
-  // the shared-memory size is a per-device attribute of each kernel
-  auto prepare = [&](auto kern, int smem, bool *done) -> bool {
-    if (done[dev]) return true;
+  const uint64_t ctx = current_context();
+  if (ctx == 0) return MOCAP_ECUDA;
+  // the shared-memory size is a per-context attribute of each kernel
+  auto prepare = [&](auto kern, int smem, ContextOnce &once) -> bool {
+    if (once.done(ctx)) return true;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
         cudaSuccess)
       return false;
-    done[dev] = true;
+    once.mark(ctx);
     return true;
   };
   if (head_dim == 128) {
-    static bool done[64] = {};
-    if (!prepare(last_row_kernel<128>, LrLayout<128>::kBytes, done)) return MOCAP_ECUDA;
+    static ContextOnce once;
+    if (!prepare(last_row_kernel<128>, LrLayout<128>::kBytes, once)) return MOCAP_ECUDA;
     last_row_kernel<128><<<grid, kThreads, LrLayout<128>::kBytes, st>>>(prm);
   } else {
-    static bool done[64] = {};
-    if (!prepare(last_row_kernel<64>, LrLayout<64>::kBytes, done)) return MOCAP_ECUDA;
+    static ContextOnce once;
+    if (!prepare(last_row_kernel<64>, LrLayout<64>::kBytes, once)) return MOCAP_ECUDA;
     last_row_kernel<64><<<grid, kThreads, LrLayout<64>::kBytes, st>>>(prm);
   }
   return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;

@@ -405,15 +405,17 @@ extern "C" mocap_status mocap_qkv_rope_append(const void *x, const void *w_qkv, 
   const int64_t tiles = static_cast<int64_t>(prm.m_pairs) * prm.n_tiles;
   const int grid = 2 * static_cast<int>(std::min<int64_t>(tiles, std::max(1, device_sm_count() / 2)));
   auto launch = [&](auto kern) -> mocap_status {
-    static bool attr_done[2][64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOCAP_ECUDA;
-    const int which = head_dim == 128 ? 1 : 0;
-    if (!attr_done[which][dev]) {
+    // one flag set per kernel: both kernels have the same type, so this
+    // lambda has one instantiation and indexes its flags by head_dim
+    static ContextOnce once[2];
+    ContextOnce &kern_once = once[head_dim == 128 ? 1 : 0];
+    const uint64_t ctx = current_context();
+    if (ctx == 0) return MOCAP_ECUDA;
+    if (!kern_once.done(ctx)) {
       if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                QkvLayout::kBytes) != cudaSuccess)
         return MOCAP_ECUDA;
-      attr_done[which][dev] = true;
+      kern_once.mark(ctx);
     }
     kern<<<grid, kThreads, QkvLayout::kBytes, reinterpret_cast<cudaStream_t>(stream)>>>(prm);
     return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;

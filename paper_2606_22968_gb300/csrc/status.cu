@@ -1,6 +1,6 @@
-// status.cu -- per-device runtime state shared by the kernels' host code:
-// the status word for bounded-wait timeouts, the SM count, the tensor-map
-// encoder; status strings.
+// status.cu -- runtime state shared by the kernels' host code: the current
+// context, the status word for bounded-wait timeouts (per context), the SM
+// count (per device), the tensor-map encoder; status strings.
 #include <atomic>
 #include <mutex>
 
@@ -8,10 +8,10 @@
 #include "sm103_ptx.cuh"
 
 namespace {
-__device__ uint32_t g_device_status;  // 0 = OK, MOCAP_ETIMEOUT after an expired wait
+__device__ uint32_t g_device_status;  // 0 = OK, else the first error a kernel recorded
 
 constexpr int kMaxDevices = 64;
-uint32_t *g_status_ptr[kMaxDevices] = {};
+std::vector<std::pair<uint64_t, uint32_t *>> g_status_ptr;  // per context ID
 std::mutex g_status_mu;
 }  // namespace
 
@@ -45,16 +45,47 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
+uint64_t current_context() {
+  static PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
+  static PFN_cuCtxGetId_v12000 get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *ptr = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(ptr);
+    ptr = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(ptr);
+  });
+  CUcontext c = nullptr;
+  unsigned long long id = 0;
+  if (get_current == nullptr || get_id == nullptr || get_current(&c) != CUDA_SUCCESS ||
+      c == nullptr || get_id(c, &id) != CUDA_SUCCESS)
+    return 0;
+  return static_cast<uint64_t>(id);
+}
+
 uint32_t *device_status_ptr() {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
   std::lock_guard<std::mutex> lock(g_status_mu);
-  if (g_status_ptr[dev] == nullptr) {
-    void *p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
-    g_status_ptr[dev] = static_cast<uint32_t *>(p);
-  }
-  return g_status_ptr[dev];
+  uint64_t c = current_context();
+  if (c != 0)
+    for (const auto &e : g_status_ptr)
+      if (e.first == c) return e.second;
+  // resolving the symbol binds the runtime's context to this thread if
+  // none was current yet
+  void *p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
+  c = current_context();
+  if (c == 0) return nullptr;
+  for (const auto &e : g_status_ptr)
+    if (e.first == c) return e.second;
+  g_status_ptr.emplace_back(c, static_cast<uint32_t *>(p));
+  return static_cast<uint32_t *>(p);
 }
 
 }  // namespace mocap
