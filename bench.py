@@ -31,6 +31,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "chunk-attn TFLOP/s & % GB300 BF16 tensor peak; prefill tokens/s"
 FALLBACK_PEAK_TFLOPS = 1700.0  # sustained bf16, used only without MEASURED_PEAKS.json
+FALLBACK_BURST_TFLOPS = 1900.0  # burst bf16, likewise
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -480,7 +481,16 @@ def ours_arm(args, rank, world, local):
     value = replica_throughput(total_flops, ms_step, world) / 1e12
     tokens_per_s = replica_throughput(w.total_tokens, ms_step, world)
     peaks, peak_src = load_peaks()
-    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAK_TFLOPS))
+    # The denominator for a run held by the power cap is the sustained cuBLAS
+    # figure (measured under the same cap, at a known clock); a run that
+    # never reached the cap is compared with the burst figure.
+    capped = "sw_power_cap" in (clk.get("reasons") or [])
+    if capped:
+        peak_name = "bf16_tflops_sustained"
+        peak = float(peaks.get(peak_name, FALLBACK_PEAK_TFLOPS))
+    else:
+        peak_name = "bf16_tflops"
+        peak = float(peaks.get(peak_name, FALLBACK_BURST_TFLOPS))
     attn_avg_ms = statistics.mean(attn_step_ms)
     achieved = total_flops / (attn_avg_ms * 1e-3) / 1e12
     traffic = ncu_traffic(pf.bounds[0], w.n_q_heads, w.n_kv_heads, w.head_dim) \
@@ -492,7 +502,7 @@ def ours_arm(args, rank, world, local):
     # bench's median clock the same tensor pipe delivers peak * f / f_peak.
     peak_mhz = (peaks.get("clocks_under_load") or {}).get("sm_mhz_median")
     frac_clock = None
-    if peak_mhz and clk.get("sm_mhz"):
+    if capped and peak_mhz and clk.get("sm_mhz"):
         frac_clock = achieved / (peak * clk["sm_mhz"] / float(peak_mhz))
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     app_gbs = standalone_bytes / (statistics.mean(app_step_ms) * 1e-3) / 1e9
@@ -530,10 +540,13 @@ def ours_arm(args, rank, world, local):
                            f"append_mode {pf.append_mode}"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak,
-                     "peak_source": f"bf16_tflops_sustained ({peak_src})",
+                     "peak_source": f"{peak_name} ({peak_src}; "
+                                    f"{'power cap active' if capped else 'power cap not reached'}"
+                                    " in the timed region)",
                      "frac_at_peak_clock": frac_clock,
                      "clock_note": (f"achieved / (peak x bench median SM clock {clk.get('sm_mhz')}"
-                                    f" MHz / peak's median SM clock {peak_mhz} MHz)"),
+                                    f" MHz / peak's median SM clock {peak_mhz} MHz)") if capped
+                     else "the burst peak's clock is not recorded: no clock-scaled fraction",
                      "kernel": "chunk_attn_kernel",
                      "traffic": None if traffic is None else traffic["traffic"],
                      "algorithmic_bytes": alg_bytes,
