@@ -1048,7 +1048,10 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
         pf.partition()
         pf.run_from_host(hq, hk, hv, ho, hl, dq, dk, dv)
 
-    step()
+    # the same warm-up as the device-resident timing: the first uploads after
+    # device-resident work run slowly until the host path has settled
+    for _ in range(max(1, args.warmup)):
+        step()
     torch.cuda.synchronize(dev)
     barrier(world)
     t0 = torch.cuda.Event(enable_timing=True)
