@@ -1048,21 +1048,35 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
         pf.partition()
         pf.run_from_host(hq, hk, hv, ho, hl, dq, dk, dv)
 
-    # the same warm-up as the device-resident timing: the first uploads after
-    # device-resident work run slowly until the host path has settled
+    # the same warm-up as the device-resident timing
     for _ in range(max(1, args.warmup)):
         step()
     torch.cuda.synchronize(dev)
     barrier(world)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
-    t0.record(stream)
-    for _ in range(args.e2e_steps):
-        step()
-    t1.record(stream)
-    torch.cuda.synchronize(dev)
-    barrier(world)
-    ms = max_over_ranks(t0.elapsed_time(t1) / args.e2e_steps, world, dev)
+    upload = pf.upload
+
+    def timed_block(mode):
+        pf.upload = mode
+        barrier(world)
+        t0.record(stream)
+        for _ in range(args.e2e_steps):
+            step()
+        t1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        return max_over_ranks(t0.elapsed_time(t1) / args.e2e_steps, world, dev)
+
+    # blocks of single-prompt steps with the default uploads (SM copy
+    # kernels) and with copy-engine uploads, interleaved; medians
+    blocks = {upload: [], "copy_engine": []}
+    for _ in range(3):
+        for mode in blocks:
+            blocks[mode].append(timed_block(mode))
+    pf.upload = upload
+    ms = statistics.median(blocks[upload])
+    ms_ce = statistics.median(blocks["copy_engine"])
     if not torch.equal(ho.to(dev), pf.out) or not torch.equal(hl.to(dev), pf.lse):
         raise RuntimeError("e2e: host copies of O / LSE differ from the device results")
     # The same steps as a stream of prompts: prompt p + 1's inputs go up while
@@ -1087,8 +1101,14 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
     del bufs
     return {"value": replica_throughput(total_flops, ms, world) / 1e12, "unit": "TFLOP/s",
             "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "overlap": "per-chunk H2D, compute (two streams, appends beside them) and D2H "
-                       "overlapped; ChunkedPrefill defaults",
+            "upload": upload,
+            "overlap": "per-chunk H2D (SM copy kernels reading pinned host memory), compute "
+                       "(two streams, appends beside them) and D2H overlapped; ChunkedPrefill "
+                       "defaults",
+            "blocks": "median of 3 blocks of e2e steps, interleaved with the same blocks "
+                      "using copy-engine uploads",
+            "copy_engine_uploads": {"value": replica_throughput(total_flops, ms_ce, world) / 1e12,
+                                    "ms_per_step": ms_ce},
             "streamed": {"value": replica_throughput(total_flops, ms_s, world) / 1e12,
                          "ms_per_step": ms_s, "prompts": args.e2e_steps,
                          "overlap": "also the next prompt's H2D under this prompt's compute"}}

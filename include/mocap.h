@@ -16,6 +16,7 @@
  *   mocap_lbcp_gemm_weight    the DP's GEMM-term weight from measured rates (host)
  *   mocap_kv_append           chunk K/V -> contiguous bf16 KV cache (device)
  *   mocap_kv_append_overlap   the same, sized to run beside an attention launch
+ *   mocap_copy_from_host      host -> device copies by the SMs (prompt uploads)
  *   mocap_qkv_rope_append     QKV projection + RoPE + KV append (device GEMM)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
@@ -229,6 +230,45 @@ mocap_status mocap_kv_append_overlap(const void *k_chunk, const void *v_chunk,
                                      int64_t cache_capacity, int64_t offset, int64_t len,
                                      int32_t n_kv_heads, int32_t head_dim,
                                      mocap_stream_t stream);
+
+/*
+ * One host -> device copy of mocap_copy_from_host: `bytes` bytes (a multiple
+ * of 16) from page-locked host memory at `src` to device memory at `dst`,
+ * both 16-byte aligned.
+ */
+typedef struct {
+  void *dst;
+  const void *src;
+  int64_t bytes;
+} mocap_copy_item;
+
+#define MOCAP_COPY_MAX_ITEMS 8
+
+/*
+ * mocap_copy_from_host -- up to MOCAP_COPY_MAX_ITEMS host -> device copies
+ * in one kernel launch on `stream`, done by the SMs reading the host pages
+ * through their device mapping (a prompt's Q/K/V on their way to the chunk
+ * pipeline, Sec. 2.2).  On GB300 the copy engines' uploads from page-locked
+ * memory ran at about 20 GB/s right after heavy device work in most trials,
+ * where SM loads of the same pages kept the link's ~200 GB/s.
+ *
+ *   beside_kernels  0: all SMs (the GPU otherwise idle, e.g. a prompt's
+ *                   first chunk); nonzero: one warp per SM with at most 32
+ *                   registers and no shared memory, which fits beside a
+ *                   running attention launch (as mocap_kv_append_overlap).
+ *
+ * Each source range must lie in one page-locked allocation (cudaHostAlloc,
+ * cudaMallocHost or cudaHostRegister) that the device sees at the same
+ * address (unified addressing), each destination in device memory; both
+ * ends of every range are checked with cudaPointerGetAttributes.  The host
+ * memory must stay valid and unchanged until the copy has run.
+ * MOCAP_EINVAL: n_items outside [0, MOCAP_COPY_MAX_ITEMS], a null item
+ * array, a null or misaligned pointer, bytes < 0 or not a multiple of 16, a
+ * source that is not such host memory or a destination that is not device
+ * memory.  Items of 0 bytes are skipped.
+ */
+mocap_status mocap_copy_from_host(const mocap_copy_item *items, int32_t n_items,
+                                  int32_t beside_kernels, mocap_stream_t stream);
 
 /*
  * mocap_qkv_rope_append -- a chunk's QKV projection, rotary embedding and KV

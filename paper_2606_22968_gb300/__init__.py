@@ -13,13 +13,14 @@ import ctypes
 from typing import List, Sequence
 
 from . import _lib
-from ._lib import AppendItem, VarlenItem
+from ._lib import AppendItem, CopyItem, VarlenItem
 
 MOCAP_OK, MOCAP_EINVAL, MOCAP_ECUDA, MOCAP_EUNSUPPORTED, MOCAP_ETIMEOUT = 0, 1, 2, 3, 4
 MOCAP_PART_UNIFORM, MOCAP_PART_LBCP = 0, 1
 MOCAP_VARLEN_MAX_ITEMS = 64
 MOCAP_VARLEN_DEV_MAX_ITEMS = 65536
 MOCAP_FUSED_APPEND_MAX = 64
+MOCAP_COPY_MAX_ITEMS = 8
 
 
 class MocapError(RuntimeError):
@@ -121,6 +122,26 @@ def mocap_kv_append_overlap(k_chunk, v_chunk, k_cache, v_cache, offset: int, str
                                                _ptr(v_cache), k_cache.shape[0], offset, length,
                                                n_kv, d, _stream(stream)),
            "mocap_kv_append_overlap")
+
+
+def mocap_copy_from_host(pairs, beside_kernels: bool = False, stream=None):
+    """Host -> device copies by the SMs: ``pairs`` is a sequence of up to
+    MOCAP_COPY_MAX_ITEMS (device_tensor, pinned_host_tensor) of equal byte
+    size, each contiguous."""
+    arr = (CopyItem * max(1, len(pairs)))()
+    for i, (dst, src) in enumerate(pairs):
+        nbytes = dst.numel() * dst.element_size()
+        if src.numel() * src.element_size() != nbytes:
+            raise ValueError("copy source and destination differ in size")
+        if not dst.is_contiguous() or not src.is_contiguous():
+            raise ValueError("copy tensors must be contiguous")
+        if src.is_cuda or not dst.is_cuda:
+            raise ValueError("copies go from host tensors to device tensors")
+        arr[i] = CopyItem(dst.data_ptr() if nbytes else None, src.data_ptr() if nbytes else None,
+                          nbytes)
+    _check(_lib.load().mocap_copy_from_host(arr, len(pairs), int(bool(beside_kernels)),
+                                            _stream(stream)),
+           "mocap_copy_from_host")
 
 
 def mocap_qkv_rope_append(x, w_qkv, q_out, k_cache, v_cache, offset: int,

@@ -22,6 +22,10 @@ class AppendItem(ctypes.Structure):
     _fields_ = [("k_src", c_vp), ("v_src", c_vp), ("dst_row", c_i64), ("rows", c_i64)]
 
 
+class CopyItem(ctypes.Structure):
+    _fields_ = [("dst", c_vp), ("src", c_vp), ("bytes", c_i64)]
+
+
 SIGNATURES = {
     "mocap_lbcp_partition": (c_i32, [c_i64, c_i32, c_i32, c_i32, ctypes.POINTER(c_i64)]),
     "mocap_lbcp_partition_dp": (c_i32, [c_i64, c_i32, c_i32, c_i32, c_i32, c_i64,
@@ -43,6 +47,7 @@ SIGNATURES = {
     "mocap_chunk_attn_varlen": (c_i32, [c_vp, c_vp, c_vp, ctypes.POINTER(VarlenItem), c_i32,
                                         c_i64, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp, c_vp,
                                         c_vp, c_sz, c_vp]),
+    "mocap_copy_from_host": (c_i32, [ctypes.POINTER(CopyItem), c_i32, c_i32, c_vp]),
     "mocap_chunk_attn_varlen_dev_workspace_size": (c_sz, [c_i32, c_i64, c_i32, c_i32, c_i32]),
     "mocap_chunk_attn_varlen_dev": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i32, c_i64, c_i64, c_i64,
                                             c_i32, c_i32, c_i32, c_f32, c_vp, c_vp, c_vp, c_sz,

@@ -14,12 +14,12 @@ from typing import List, Optional
 
 import torch
 
-from . import (MOCAP_COST_CAUSAL, MOCAP_PART_LBCP, MOCAP_PART_UNIFORM, mocap_chunk_attn,
-               mocap_chunk_attn_append, mocap_chunk_attn_varlen, mocap_chunk_attn_varlen_append,
-               mocap_chunk_attn_workspace_size, mocap_kv_append, mocap_kv_append_overlap,
+from . import (MOCAP_COPY_MAX_ITEMS, MOCAP_COST_CAUSAL, MOCAP_PART_LBCP, MOCAP_PART_UNIFORM,
+               mocap_chunk_attn, mocap_chunk_attn_append, mocap_chunk_attn_varlen,
+               mocap_chunk_attn_varlen_append, mocap_chunk_attn_workspace_size,
+               mocap_copy_from_host, mocap_kv_append, mocap_kv_append_overlap,
                mocap_lbcp_gemm_weight, mocap_lbcp_partition, mocap_lbcp_partition_dp,
-               mocap_lbcp_partition_dp_latency,
-               mocap_qkv_rope_append)
+               mocap_lbcp_partition_dp_latency, mocap_qkv_rope_append)
 from .workloads import GRANULARITY, Workload, request_offsets
 
 
@@ -42,6 +42,7 @@ def stage_balanced_bounds(seq_len: int, num_chunks: int, attn_s_per_pair: float,
 
 
 APPEND_MODES = ("serial", "fused", "overlap")
+UPLOAD_MODES = ("kernel", "copy_engine")
 
 
 def latency_balanced_bounds(seq_len: int, num_chunks: int, n_q_heads: int, n_kv_heads: int,
@@ -67,7 +68,7 @@ class ChunkedPrefill:
 
     def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True,
                  bounds: Optional[List[List[int]]] = None, append_mode: str = "overlap",
-                 chunk_streams: Optional[int] = None):
+                 chunk_streams: Optional[int] = None, upload: str = "kernel"):
         """``bounds`` (one boundary list per request) replaces the workload's
         partition rule, e.g. with the Algorithm 1 stage-1 DP's split.
 
@@ -90,9 +91,18 @@ class ChunkedPrefill:
         compute stream has its own split-KV workspace.  Steps are still
         issued in order; per-step events then time overlapping launches.
         Needs append_mode "overlap": every step then waits for an event that
-        says its rows (and all earlier rows) are in the cache."""
+        says its rows (and all earlier rows) are in the cache.
+
+        ``upload`` says how ``run_from_host`` / ``run_prompts_from_host``
+        bring Q/K/V up from pinned host memory: "kernel" (mocap_copy_from_host:
+        the SMs read the host pages, all of them for the first step of a
+        prompt with nothing else running, one warp per SM beside the attention
+        launches after that) or "copy_engine" (cudaMemcpyAsync)."""
         if append_mode not in APPEND_MODES:
             raise ValueError(f"append_mode must be one of {APPEND_MODES}")
+        if upload not in UPLOAD_MODES:
+            raise ValueError(f"upload must be one of {UPLOAD_MODES}")
+        self.upload = upload
         if chunk_streams is None:
             chunk_streams = 2 if append_mode == "overlap" else 1
         if chunk_streams not in (1, 2):
@@ -386,6 +396,20 @@ class ChunkedPrefill:
 
         self.run(q, k, v, compute, landed=landed, after_step=copy_back)
 
+    def _upload_step(self, step, dev_qkv, host_qkv, stream, beside):
+        """Copy one step's Q/K/V rows from pinned host memory on ``stream``."""
+        pairs = []
+        for r, c in step:
+            rows, _, _ = self._rows(r, c)
+            pairs += [(d[rows], h[rows]) for d, h in zip(dev_qkv, host_qkv)]
+        if self.upload == "copy_engine":
+            for d, h in pairs:
+                d.copy_(h, non_blocking=True)
+            return
+        for a in range(0, len(pairs), MOCAP_COPY_MAX_ITEMS):
+            mocap_copy_from_host(pairs[a:a + MOCAP_COPY_MAX_ITEMS], beside_kernels=beside,
+                                 stream=stream)
+
     def run_from_host(self, host_q, host_k, host_v, host_out, host_lse, q, k, v):
         """The whole prompt from (pinned) host memory, overlapping transfers
         with compute.
@@ -399,7 +423,9 @@ class ChunkedPrefill:
         requests a chunk's LSE columns are strided in the ``[Hq, T]`` array, so
         the whole LSE (4 Hq T bytes) goes back in one contiguous copy after the
         last step instead.  The caller's current stream waits for everything
-        before this returns."""
+        before this returns; the host tensors must stay alive and unchanged
+        until that work has finished (with ``upload="kernel"`` the GPU reads
+        them in place)."""
         compute = torch.cuda.current_stream(self.device)
         h2d = torch.cuda.Stream(self.device)
         d2h = torch.cuda.Stream(self.device)
@@ -408,12 +434,10 @@ class ChunkedPrefill:
         landed = []
         h2d.wait_stream(compute)  # device buffers are free of earlier work
         with torch.cuda.stream(h2d):
-            for step in steps:
-                for r, c in step:
-                    rows, _, _ = self._rows(r, c)
-                    q[rows].copy_(host_q[rows], non_blocking=True)
-                    k[rows].copy_(host_k[rows], non_blocking=True)
-                    v[rows].copy_(host_v[rows], non_blocking=True)
+            for i, step in enumerate(steps):
+                # step 0 goes up with nothing else running; later steps
+                # beside the attention launches
+                self._upload_step(step, (q, k, v), (host_q, host_k, host_v), h2d, beside=i > 0)
                 ev = torch.cuda.Event()
                 ev.record(h2d)
                 landed.append(ev)
@@ -460,12 +484,10 @@ class ChunkedPrefill:
             with torch.cuda.stream(h2d):
                 if computed[p % 2] is not None:
                     h2d.wait_event(computed[p % 2])
-                for step in steps:
-                    for r, c in step:
-                        rows, _, _ = self._rows(r, c)
-                        q[rows].copy_(host_q[rows], non_blocking=True)
-                        k[rows].copy_(host_k[rows], non_blocking=True)
-                        v[rows].copy_(host_v[rows], non_blocking=True)
+                for i, step in enumerate(steps):
+                    # only the first prompt's first step goes up alone
+                    self._upload_step(step, (q, k, v), (host_q, host_k, host_v), h2d,
+                                      beside=p > 0 or i > 0)
                     ev = torch.cuda.Event()
                     ev.record(h2d)
                     evs.append(ev)

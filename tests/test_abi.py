@@ -205,6 +205,28 @@ def test_varlen_dev_workspace_layout(lib):
     assert lib.mocap_chunk_attn_varlen_dev_workspace_size(3, 1000, 64, 8, 96) == 0
 
 
+def test_copy_from_host_argument_checks(lib):
+    """mocap_copy_from_host rejects what it can see on the host before any
+    CUDA call; an empty batch is a no-op."""
+    from paper_2606_22968_gb300._lib import CopyItem
+    f = lib.mocap_copy_from_host
+
+    def call(items, n=None):
+        arr = (CopyItem * max(1, len(items)))(*[CopyItem(*x) for x in items])
+        return f(arr, len(items) if n is None else n, 0, None)
+
+    assert call([]) == 0
+    assert f(None, 0, 1, None) == 0
+    assert f(None, 1, 0, None) == 1                       # null item array
+    assert call([(FAKE, FAKE, 32)], n=9) == 1             # above MOCAP_COPY_MAX_ITEMS
+    assert call([(FAKE, FAKE, 32)], n=-1) == 1
+    assert call([(FAKE, FAKE, 17)]) == 1                  # not whole 16-byte vectors
+    assert call([(FAKE, FAKE, -16)]) == 1
+    assert call([(None, FAKE, 32)]) == 1
+    assert call([(FAKE, FAKE + 8, 32)]) == 1              # misaligned source
+    assert call([(FAKE, FAKE, 0)]) == 0                   # empty item skipped
+
+
 def test_workspace_size_split_plan(lib):
     # many row blocks: no split; few long row blocks: a split and its layout
     assert lib.mocap_chunk_attn_workspace_size(0, 23168, 64, 8, 128) == 0
