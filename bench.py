@@ -1055,10 +1055,10 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
     barrier(world)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
-    upload = pf.upload
+    mode0 = pf.host_copies
 
     def timed_block(mode):
-        pf.upload = mode
+        pf.host_copies = mode
         barrier(world)
         t0.record(stream)
         for _ in range(args.e2e_steps):
@@ -1068,14 +1068,15 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
         barrier(world)
         return max_over_ranks(t0.elapsed_time(t1) / args.e2e_steps, world, dev)
 
-    # blocks of single-prompt steps with the default uploads (SM copy
-    # kernels) and with copy-engine uploads, interleaved; medians
-    blocks = {upload: [], "copy_engine": []}
+    # blocks of single-prompt steps with the default host copies (SM copy
+    # kernels, both directions) and with copy-engine copies, interleaved;
+    # medians
+    blocks = {mode0: [], "copy_engine": []}
     for _ in range(3):
         for mode in blocks:
             blocks[mode].append(timed_block(mode))
-    pf.upload = upload
-    ms = statistics.median(blocks[upload])
+    pf.host_copies = mode0
+    ms = statistics.median(blocks[mode0])
     ms_ce = statistics.median(blocks["copy_engine"])
     if not torch.equal(ho.to(dev), pf.out) or not torch.equal(hl.to(dev), pf.lse):
         raise RuntimeError("e2e: host copies of O / LSE differ from the device results")
@@ -1101,13 +1102,13 @@ def measure_e2e(args, m, w, pf, q, k, v, dev, stream, total_flops, world):
     del bufs
     return {"value": replica_throughput(total_flops, ms, world) / 1e12, "unit": "TFLOP/s",
             "ms_per_step": ms, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "upload": upload,
-            "overlap": "per-chunk H2D (SM copy kernels reading pinned host memory), compute "
-                       "(two streams, appends beside them) and D2H overlapped; ChunkedPrefill "
-                       "defaults",
+            "host_copies": mode0,
+            "overlap": "per-chunk H2D and D2H by SM copy kernels through the pinned host pages' "
+                       "device mapping, overlapped with compute (two streams, appends beside "
+                       "them); ChunkedPrefill defaults",
             "blocks": "median of 3 blocks of e2e steps, interleaved with the same blocks "
-                      "using copy-engine uploads",
-            "copy_engine_uploads": {"value": replica_throughput(total_flops, ms_ce, world) / 1e12,
+                      "using copy-engine host copies",
+            "copy_engine_host_copies": {"value": replica_throughput(total_flops, ms_ce, world) / 1e12,
                                     "ms_per_step": ms_ce},
             "streamed": {"value": replica_throughput(total_flops, ms_s, world) / 1e12,
                          "ms_per_step": ms_s, "prompts": args.e2e_steps,

@@ -16,7 +16,9 @@
  *   mocap_lbcp_gemm_weight    the DP's GEMM-term weight from measured rates (host)
  *   mocap_kv_append           chunk K/V -> contiguous bf16 KV cache (device)
  *   mocap_kv_append_overlap   the same, sized to run beside an attention launch
- *   mocap_copy_from_host      host -> device copies by the SMs (prompt uploads)
+ *   mocap_copy_from_host, mocap_copy_to_host
+ *                             host <-> device copies by the SMs (a prompt's
+ *                             inputs up, its results back)
  *   mocap_qkv_rope_append     QKV projection + RoPE + KV append (device GEMM)
  *   mocap_chunk_attn          one chunk's GQA attention over cache[0, prefix+len)
  *   mocap_chunk_attn_varlen   the same for many (request, chunk) items in one launch
@@ -269,6 +271,17 @@ typedef struct {
  */
 mocap_status mocap_copy_from_host(const mocap_copy_item *items, int32_t n_items,
                                   int32_t beside_kernels, mocap_stream_t stream);
+
+/*
+ * mocap_copy_to_host -- the same in the other direction: each item copies
+ * `bytes` from device memory at `src` to page-locked host memory at `dst`
+ * (a chunk's O and LSE on their way back), with the SMs storing through the
+ * host pages' device mapping; the copy engines' returns slowed the same way
+ * after heavy device work.  Same launch forms, checks (device source,
+ * mapped page-locked destination) and errors as mocap_copy_from_host.
+ */
+mocap_status mocap_copy_to_host(const mocap_copy_item *items, int32_t n_items,
+                                int32_t beside_kernels, mocap_stream_t stream);
 
 /*
  * mocap_qkv_rope_append -- a chunk's QKV projection, rotary embedding and KV

@@ -124,10 +124,7 @@ def mocap_kv_append_overlap(k_chunk, v_chunk, k_cache, v_cache, offset: int, str
            "mocap_kv_append_overlap")
 
 
-def mocap_copy_from_host(pairs, beside_kernels: bool = False, stream=None):
-    """Host -> device copies by the SMs: ``pairs`` is a sequence of up to
-    MOCAP_COPY_MAX_ITEMS (device_tensor, pinned_host_tensor) of equal byte
-    size, each contiguous."""
+def _copy_array(pairs, to_host):
     arr = (CopyItem * max(1, len(pairs)))()
     for i, (dst, src) in enumerate(pairs):
         nbytes = dst.numel() * dst.element_size()
@@ -135,13 +132,28 @@ def mocap_copy_from_host(pairs, beside_kernels: bool = False, stream=None):
             raise ValueError("copy source and destination differ in size")
         if not dst.is_contiguous() or not src.is_contiguous():
             raise ValueError("copy tensors must be contiguous")
-        if src.is_cuda or not dst.is_cuda:
-            raise ValueError("copies go from host tensors to device tensors")
+        if (dst.is_cuda, src.is_cuda) != ((False, True) if to_host else (True, False)):
+            raise ValueError("copies go between host and device tensors in the named direction")
         arr[i] = CopyItem(dst.data_ptr() if nbytes else None, src.data_ptr() if nbytes else None,
                           nbytes)
-    _check(_lib.load().mocap_copy_from_host(arr, len(pairs), int(bool(beside_kernels)),
-                                            _stream(stream)),
+    return arr
+
+
+def mocap_copy_from_host(pairs, beside_kernels: bool = False, stream=None):
+    """Host -> device copies by the SMs: ``pairs`` is a sequence of up to
+    MOCAP_COPY_MAX_ITEMS (device_tensor, pinned_host_tensor) of equal byte
+    size, each contiguous."""
+    _check(_lib.load().mocap_copy_from_host(_copy_array(pairs, False), len(pairs),
+                                            int(bool(beside_kernels)), _stream(stream)),
            "mocap_copy_from_host")
+
+
+def mocap_copy_to_host(pairs, beside_kernels: bool = False, stream=None):
+    """Device -> host copies by the SMs: ``pairs`` of (pinned_host_tensor,
+    device_tensor)."""
+    _check(_lib.load().mocap_copy_to_host(_copy_array(pairs, True), len(pairs),
+                                          int(bool(beside_kernels)), _stream(stream)),
+           "mocap_copy_to_host")
 
 
 def mocap_qkv_rope_append(x, w_qkv, q_out, k_cache, v_cache, offset: int,

@@ -20,7 +20,7 @@ OBJDIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmocap.so")
 
 SOURCES = ["lbcp.cpp", "status.cu", "kv_append.cu", "chunk_attn.cu", "qkv_rope.cu",
-           "last_row_attn.cu", "h2d_copy.cu"]
+           "last_row_attn.cu", "host_copy.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr",
          "-I" + INCLUDE, "-I" + CSRC]

@@ -48,6 +48,7 @@ SIGNATURES = {
                                         c_i64, c_i64, c_i32, c_i32, c_i32, c_f32, c_vp, c_vp,
                                         c_vp, c_sz, c_vp]),
     "mocap_copy_from_host": (c_i32, [ctypes.POINTER(CopyItem), c_i32, c_i32, c_vp]),
+    "mocap_copy_to_host": (c_i32, [ctypes.POINTER(CopyItem), c_i32, c_i32, c_vp]),
     "mocap_chunk_attn_varlen_dev_workspace_size": (c_sz, [c_i32, c_i64, c_i32, c_i32, c_i32]),
     "mocap_chunk_attn_varlen_dev": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i32, c_i64, c_i64, c_i64,
                                             c_i32, c_i32, c_i32, c_f32, c_vp, c_vp, c_vp, c_sz,

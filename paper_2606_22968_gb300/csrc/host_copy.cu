@@ -1,16 +1,18 @@
-// h2d_copy.cu -- host -> device copies by the SMs, reading page-locked host
-// memory through its device mapping.
+// host_copy.cu -- copies between page-locked host memory and device memory
+// done by the SMs, through the host pages' device mapping.
 //
 // A prompt's Q/K/V reach the GPU from host memory before its chunks run
 // (Sec. 2.2: the chunks of a prefill-only request stream through the
 // pipeline).  On the GB300 machines this library runs on, copy-engine uploads
 // from page-locked memory right after heavy device work ran at about
 // 20 GB/s (15-28 ms for 475 MB) in 12 of 16 trials, while SM loads of the
-// same pages ran at the link's 200 GB/s in 15 of 16.  So the pipeline
-// uploads with these kernels: all SMs while nothing else runs, or one warp
-// per SM (32 registers, no shared memory: what an attention CTA leaves free)
-// beside the attention launches.  Each launch copies up to
-// MOCAP_COPY_MAX_ITEMS ranges (for example a chunk's Q, K and V rows).
+// same pages ran at the link's 200 GB/s in 15 of 16; returns (380 MB back)
+// behaved the same way, 14 of 16 slow on the copy engines against 2 of 16
+// with SM stores.  So the pipeline moves a prompt's data with these kernels:
+// all SMs while nothing else runs, or one warp per SM (32 registers, no
+// shared memory: what an attention CTA leaves free) beside the attention
+// launches.  Each launch copies up to MOCAP_COPY_MAX_ITEMS ranges (for
+// example a chunk's Q, K and V rows).
 #include <algorithm>
 
 #include "internal.h"
@@ -49,17 +51,17 @@ __device__ __forceinline__ void copy_segment(const CopySeg &s) {
   }
 }
 
-__global__ void __launch_bounds__(kThreads) h2d_copy_kernel(const __grid_constant__ CopyParams p) {
+__global__ void __launch_bounds__(kThreads) host_copy_kernel(const __grid_constant__ CopyParams p) {
   copy_segment<kThreads>(p.seg[blockIdx.y]);
 }
 
-__global__ void __maxnreg__(32) h2d_copy_beside_kernel(const __grid_constant__ CopyParams p) {
+__global__ void __maxnreg__(32) host_copy_beside_kernel(const __grid_constant__ CopyParams p) {
   copy_segment<kBesideThreads>(p.seg[blockIdx.y]);
 }
 
-// The source must be page-locked host memory mapped at the same address on
-// the device (unified addressing); the destination device memory.
-bool host_source_ok(const void *src, int64_t bytes) {
+// Page-locked host memory mapped at the same address on the device (unified
+// addressing), checked at both ends of the range.
+bool host_range_ok(const void *src, int64_t bytes) {
   for (const char *p : {static_cast<const char *>(src), static_cast<const char *>(src) + bytes - 1}) {
     cudaPointerAttributes a{};
     if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
@@ -71,7 +73,8 @@ bool host_source_ok(const void *src, int64_t bytes) {
   return true;
 }
 
-bool device_dest_ok(const void *dst, int64_t bytes) {
+// Device (or managed) memory at both ends of the range.
+bool device_range_ok(const void *dst, int64_t bytes) {
   for (const char *p : {static_cast<const char *>(dst), static_cast<const char *>(dst) + bytes - 1}) {
     cudaPointerAttributes a{};
     if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
@@ -83,10 +86,8 @@ bool device_dest_ok(const void *dst, int64_t bytes) {
   return true;
 }
 
-}  // namespace
-
-extern "C" mocap_status mocap_copy_from_host(const mocap_copy_item *items, int32_t n_items,
-                                             int32_t beside_kernels, mocap_stream_t stream) {
+mocap_status copy_items(const mocap_copy_item *items, int32_t n_items, int32_t beside_kernels,
+                        mocap_stream_t stream, bool to_host) {
   if (n_items < 0 || n_items > MOCAP_COPY_MAX_ITEMS) return MOCAP_EINVAL;
   if (n_items > 0 && items == nullptr) return MOCAP_EINVAL;
   CopyParams prm{};
@@ -97,8 +98,9 @@ extern "C" mocap_status mocap_copy_from_host(const mocap_copy_item *items, int32
     if (it.bytes == 0) continue;
     if (!it.dst || !it.src || !mocap::aligned16(it.dst) || !mocap::aligned16(it.src))
       return MOCAP_EINVAL;
-    if (!host_source_ok(it.src, it.bytes) || !device_dest_ok(it.dst, it.bytes))
-      return MOCAP_EINVAL;
+    const bool ok = to_host ? device_range_ok(it.src, it.bytes) && host_range_ok(it.dst, it.bytes)
+                            : host_range_ok(it.src, it.bytes) && device_range_ok(it.dst, it.bytes);
+    if (!ok) return MOCAP_EINVAL;
     CopySeg &s = prm.seg[prm.n_seg++];
     s.src = static_cast<const uint4 *>(it.src);
     s.dst = static_cast<uint4 *>(it.dst);
@@ -112,12 +114,24 @@ extern "C" mocap_status mocap_copy_from_host(const mocap_copy_item *items, int32
     // one warp per SM in all, shared among the segments
     const int64_t want = (most + kBesideThreads * kUnroll - 1) / (kBesideThreads * kUnroll);
     const int per = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(want, sms / prm.n_seg)));
-    h2d_copy_beside_kernel<<<dim3(per, prm.n_seg), kBesideThreads, 0, st>>>(prm);
+    host_copy_beside_kernel<<<dim3(per, prm.n_seg), kBesideThreads, 0, st>>>(prm);
   } else {
     const int64_t want = (most + kThreads * kUnroll - 1) / (kThreads * kUnroll);
     const int per = static_cast<int>(
         std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)sms * kCtasPerSm / prm.n_seg)));
-    h2d_copy_kernel<<<dim3(per, prm.n_seg), kThreads, 0, st>>>(prm);
+    host_copy_kernel<<<dim3(per, prm.n_seg), kThreads, 0, st>>>(prm);
   }
   return cudaGetLastError() == cudaSuccess ? MOCAP_OK : MOCAP_ECUDA;
+}
+
+}  // namespace
+
+extern "C" mocap_status mocap_copy_from_host(const mocap_copy_item *items, int32_t n_items,
+                                             int32_t beside_kernels, mocap_stream_t stream) {
+  return copy_items(items, n_items, beside_kernels, stream, false);
+}
+
+extern "C" mocap_status mocap_copy_to_host(const mocap_copy_item *items, int32_t n_items,
+                                           int32_t beside_kernels, mocap_stream_t stream) {
+  return copy_items(items, n_items, beside_kernels, stream, true);
 }

@@ -17,7 +17,8 @@ import torch
 from . import (MOCAP_COPY_MAX_ITEMS, MOCAP_COST_CAUSAL, MOCAP_PART_LBCP, MOCAP_PART_UNIFORM,
                mocap_chunk_attn, mocap_chunk_attn_append, mocap_chunk_attn_varlen,
                mocap_chunk_attn_varlen_append, mocap_chunk_attn_workspace_size,
-               mocap_copy_from_host, mocap_kv_append, mocap_kv_append_overlap,
+               mocap_copy_from_host, mocap_copy_to_host, mocap_kv_append,
+               mocap_kv_append_overlap,
                mocap_lbcp_gemm_weight, mocap_lbcp_partition, mocap_lbcp_partition_dp,
                mocap_lbcp_partition_dp_latency, mocap_qkv_rope_append)
 from .workloads import GRANULARITY, Workload, request_offsets
@@ -42,7 +43,7 @@ def stage_balanced_bounds(seq_len: int, num_chunks: int, attn_s_per_pair: float,
 
 
 APPEND_MODES = ("serial", "fused", "overlap")
-UPLOAD_MODES = ("kernel", "copy_engine")
+HOST_COPY_MODES = ("kernel", "copy_engine")
 
 
 def latency_balanced_bounds(seq_len: int, num_chunks: int, n_q_heads: int, n_kv_heads: int,
@@ -68,7 +69,7 @@ class ChunkedPrefill:
 
     def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True,
                  bounds: Optional[List[List[int]]] = None, append_mode: str = "overlap",
-                 chunk_streams: Optional[int] = None, upload: str = "kernel"):
+                 chunk_streams: Optional[int] = None, host_copies: str = "kernel"):
         """``bounds`` (one boundary list per request) replaces the workload's
         partition rule, e.g. with the Algorithm 1 stage-1 DP's split.
 
@@ -93,16 +94,18 @@ class ChunkedPrefill:
         Needs append_mode "overlap": every step then waits for an event that
         says its rows (and all earlier rows) are in the cache.
 
-        ``upload`` says how ``run_from_host`` / ``run_prompts_from_host``
-        bring Q/K/V up from pinned host memory: "kernel" (mocap_copy_from_host:
-        the SMs read the host pages, all of them for the first step of a
-        prompt with nothing else running, one warp per SM beside the attention
-        launches after that) or "copy_engine" (cudaMemcpyAsync)."""
+        ``host_copies`` says how ``run_from_host`` / ``run_prompts_from_host``
+        move Q/K/V up from pinned host memory and O/LSE back.  "kernel": the
+        uploads by the SMs (mocap_copy_from_host: all SMs for a prompt's first
+        step, one warp per SM beside the attention launches after that); the
+        results by the copy engines while attention runs and by the SMs
+        (mocap_copy_to_host) for the last ones, which nothing hides.
+        "copy_engine": every copy by cudaMemcpyAsync."""
         if append_mode not in APPEND_MODES:
             raise ValueError(f"append_mode must be one of {APPEND_MODES}")
-        if upload not in UPLOAD_MODES:
-            raise ValueError(f"upload must be one of {UPLOAD_MODES}")
-        self.upload = upload
+        if host_copies not in HOST_COPY_MODES:
+            raise ValueError(f"host_copies must be one of {HOST_COPY_MODES}")
+        self.host_copies = host_copies
         if chunk_streams is None:
             chunk_streams = 2 if append_mode == "overlap" else 1
         if chunk_streams not in (1, 2):
@@ -374,11 +377,13 @@ class ChunkedPrefill:
         b0, b1 = self.bounds[r][c], self.bounds[r][c + 1]
         return slice(self.cu[r] + b0, self.cu[r] + b1), b0, b1
 
-    def _compute_and_return(self, q, k, v, compute, d2h, landed, host_out, host_lse):
+    def _compute_and_return(self, q, k, v, compute, d2h, landed, host_out, host_lse,
+                            last_alone=True):
         """Every step on ``compute`` (and the second compute stream) once its
         inputs have landed (events ``landed``), each step's O (and a single
         request's LSE block) copied back on ``d2h`` as soon as that step is
-        done."""
+        done.  ``last_alone``: nothing else computes while the last step's
+        results go back (no next prompt queued behind this one)."""
         steps = self.steps()
         hq = self.w.n_q_heads
 
@@ -386,13 +391,13 @@ class ChunkedPrefill:
             done = torch.cuda.Event()
             done.record(st)
             d2h.wait_event(done)
-            with torch.cuda.stream(d2h):
-                for r, c in steps[i]:
-                    rows, b0, b1 = self._rows(r, c)
-                    host_out[rows].copy_(self.out[rows], non_blocking=True)
-                    if self.single:
-                        host_lse[hq * b0:hq * b1].copy_(self.lse[hq * b0:hq * b1],
-                                                        non_blocking=True)
+            pairs = []
+            for r, c in steps[i]:
+                rows, b0, b1 = self._rows(r, c)
+                pairs.append((host_out[rows], self.out[rows]))
+                if self.single:
+                    pairs.append((host_lse[hq * b0:hq * b1], self.lse[hq * b0:hq * b1]))
+            self._copy_back(pairs, d2h, beside=i + 1 < len(steps) or not last_alone)
 
         self.run(q, k, v, compute, landed=landed, after_step=copy_back)
 
@@ -402,13 +407,28 @@ class ChunkedPrefill:
         for r, c in step:
             rows, _, _ = self._rows(r, c)
             pairs += [(d[rows], h[rows]) for d, h in zip(dev_qkv, host_qkv)]
-        if self.upload == "copy_engine":
-            for d, h in pairs:
-                d.copy_(h, non_blocking=True)
+        self._host_copy(pairs, stream, beside, mocap_copy_from_host)
+
+    def _copy_back(self, pairs, stream, beside):
+        """Copy (pinned host, device) pairs back on ``stream``: by the SMs when
+        nothing else runs (``beside`` false: a prompt's last results, which
+        nothing hides), else by the copy engines, which then work behind the
+        attention launches without taking SM slots from them."""
+        if beside and self.host_copies == "kernel":
+            with torch.cuda.stream(stream):
+                for d, src in pairs:
+                    d.copy_(src, non_blocking=True)
+            return
+        self._host_copy(pairs, stream, beside, mocap_copy_to_host)
+
+    def _host_copy(self, pairs, stream, beside, fn):
+        if self.host_copies == "copy_engine":
+            with torch.cuda.stream(stream):
+                for d, src in pairs:
+                    d.copy_(src, non_blocking=True)
             return
         for a in range(0, len(pairs), MOCAP_COPY_MAX_ITEMS):
-            mocap_copy_from_host(pairs[a:a + MOCAP_COPY_MAX_ITEMS], beside_kernels=beside,
-                                 stream=stream)
+            fn(pairs[a:a + MOCAP_COPY_MAX_ITEMS], beside_kernels=beside, stream=stream)
 
     def run_from_host(self, host_q, host_k, host_v, host_out, host_lse, q, k, v):
         """The whole prompt from (pinned) host memory, overlapping transfers
@@ -424,8 +444,8 @@ class ChunkedPrefill:
         the whole LSE (4 Hq T bytes) goes back in one contiguous copy after the
         last step instead.  The caller's current stream waits for everything
         before this returns; the host tensors must stay alive and unchanged
-        until that work has finished (with ``upload="kernel"`` the GPU reads
-        them in place)."""
+        until that work has finished (with ``host_copies="kernel"`` the GPU
+        reads and writes them in place)."""
         compute = torch.cuda.current_stream(self.device)
         h2d = torch.cuda.Stream(self.device)
         d2h = torch.cuda.Stream(self.device)
@@ -445,8 +465,7 @@ class ChunkedPrefill:
         self._compute_and_return(q, k, v, compute, d2h, landed, host_out, host_lse)
         if not self.single:
             d2h.wait_stream(compute)
-            with torch.cuda.stream(d2h):
-                host_lse.copy_(self.lse, non_blocking=True)
+            self._copy_back([(host_lse, self.lse)], d2h, beside=False)
         compute.wait_stream(d2h)
         compute.wait_stream(h2d)
 
@@ -502,14 +521,14 @@ class ChunkedPrefill:
             host_out, host_lse = prompts[p][3], prompts[p][4]
             if outputs_gone is not None:
                 compute.wait_event(outputs_gone)
-            self._compute_and_return(q, k, v, compute, d2h, landed[p], host_out, host_lse)
+            self._compute_and_return(q, k, v, compute, d2h, landed[p], host_out, host_lse,
+                                     last_alone=p + 1 == len(prompts))
             end = torch.cuda.Event()
             end.record(compute)
             computed[p % 2] = end
             if not self.single:
                 d2h.wait_event(end)
-                with torch.cuda.stream(d2h):
-                    host_lse.copy_(self.lse, non_blocking=True)
+                self._copy_back([(host_lse, self.lse)], d2h, beside=True)
             gone = torch.cuda.Event()
             gone.record(d2h)
             outputs_gone = gone

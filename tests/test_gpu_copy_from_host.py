@@ -1,9 +1,9 @@
-"""GPU: mocap_copy_from_host, host -> device copies by the SMs.  Bytes land
-exactly (both launch forms, ragged sizes, several ranges per launch, bytes
-around the ranges untouched); sources that are not page-locked host memory,
-or destinations that are not device memory, are refused before any launch;
-the host-memory pipeline gives the same bits with kernel and copy-engine
-uploads."""
+"""GPU: mocap_copy_from_host / mocap_copy_to_host, host <-> device copies by
+the SMs.  Bytes land exactly (both launch forms, ragged sizes, several
+ranges per launch, bytes around the ranges untouched); ranges in the wrong
+kind of memory are refused before any launch; the host-memory pipeline
+(one prompt, and prompts streamed) gives the same bits with kernel and
+copy-engine copies."""
 
 import numpy as np
 import pytest
@@ -39,6 +39,24 @@ def test_copies_land_exactly(m, beside, sizes):
         assert bool((got[:16] == 0xA5).all()) and bool((got[16 + n:] == 0xA5).all())
 
 
+@pytest.mark.parametrize("beside", [False, True])
+@pytest.mark.parametrize("sizes", [[16], [4096, 16, 48], [3 << 20, 12345 * 16, 64 << 20]])
+def test_copies_back_land_exactly(m, beside, sizes):
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(sum(sizes) + beside)
+    pairs, checks = [], []
+    for n in sizes:
+        src = torch.randint(0, 256, (n + 64,), generator=gen, device=dev, dtype=torch.uint8)
+        host = torch.full((n + 64,), 0x5A, dtype=torch.uint8).pin_memory()
+        pairs.append((host[16:16 + n], src[32:32 + n]))
+        checks.append((host, src, n))
+    m.mocap_copy_to_host(pairs, beside_kernels=beside)
+    torch.cuda.synchronize()
+    for host, src, n in checks:
+        assert torch.equal(host[16:16 + n], src[32:32 + n].cpu())
+        assert bool((host[:16] == 0x5A).all()) and bool((host[16 + n:] == 0x5A).all())
+
+
 def test_refuses_what_is_not_pinned_host_memory(m):
     dev = torch.device("cuda")
     dst = torch.empty(4096, device=dev, dtype=torch.uint8)
@@ -58,10 +76,21 @@ def test_refuses_what_is_not_pinned_host_memory(m):
     assert call(dst.data_ptr(), pinned.data_ptr()) == m.MOCAP_OK
     torch.cuda.synchronize()
 
+    def back(d, s):
+        arr = (CopyItem * 1)(CopyItem(d, s, 4096))
+        return lib.mocap_copy_to_host(arr, 1, 1, torch.cuda.current_stream().cuda_stream)
+
+    assert back(pageable.data_ptr(), dst.data_ptr()) == m.MOCAP_EINVAL
+    assert back(other.data_ptr(), dst.data_ptr()) == m.MOCAP_EINVAL    # device memory as target
+    assert back(pinned.data_ptr(), pinned.data_ptr()) == m.MOCAP_EINVAL  # host memory as source
+    assert back(pinned.data_ptr(), dst.data_ptr()) == m.MOCAP_OK
+    torch.cuda.synchronize()
+
 
 @pytest.mark.parametrize("index", [3, 5])
-def test_pipeline_uploads_kernel_equals_copy_engine(m, index):
-    """run_from_host with both upload forms: O and LSE bitwise equal."""
+def test_pipeline_host_copies_kernel_equals_copy_engine(m, index):
+    """run_from_host and run_prompts_from_host (three prompts) with both
+    forms of host copies: O and LSE bitwise equal."""
     from paper_2606_22968_gb300 import workloads
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
     w = workloads.get(index)
@@ -69,8 +98,8 @@ def test_pipeline_uploads_kernel_equals_copy_engine(m, index):
     q, k, v = workloads.make_qkv(w, dev)
     hq, hk, hv = (t.cpu().pin_memory() for t in (q, k, v))
     outs = []
-    for upload in ("kernel", "copy_engine"):
-        pf = ChunkedPrefill(w, dev, upload=upload)
+    for mode in ("kernel", "copy_engine"):
+        pf = ChunkedPrefill(w, dev, host_copies=mode)
         ho = torch.full(pf.out.shape, float("nan"), dtype=pf.out.dtype).pin_memory()
         hl = torch.full(pf.lse.shape, float("nan"), dtype=pf.lse.dtype).pin_memory()
         dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
@@ -80,5 +109,21 @@ def test_pipeline_uploads_kernel_equals_copy_engine(m, index):
         assert m.mocap_last_device_status() == 0
         assert torch.equal(dq, q) and torch.equal(dk, k) and torch.equal(dv, v)
         outs.append((ho.view(torch.int16).clone(), hl.clone()))
+        # three prompts streamed (the second and third are the first's inputs
+        # with Q scaled, so every prompt's results differ)
+        hqs = [hq] + [(q * s).cpu().pin_memory() for s in (0.5, 2.0)]
+        prompts = [(x, hk, hv,
+                    torch.full(pf.out.shape, float("nan"), dtype=pf.out.dtype).pin_memory(),
+                    torch.full(pf.lse.shape, float("nan"), dtype=pf.lse.dtype).pin_memory())
+                   for x in hqs]
+        bufs = [(dq, dk, dv), (torch.empty_like(q), torch.empty_like(k), torch.empty_like(v))]
+        pf.partition()
+        pf.run_prompts_from_host(prompts, bufs)
+        torch.cuda.synchronize()
+        assert m.mocap_last_device_status() == 0
+        outs.append(tuple(t.view(torch.int16).clone() if t.dtype == torch.bfloat16 else t.clone()
+                          for pr in prompts for t in pr[3:]))
+    assert all(torch.equal(a, b) for a, b in zip(outs[0], outs[2]))
+    assert all(torch.equal(a, b) for a, b in zip(outs[1], outs[3]))
     assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
-    assert not torch.isnan(outs[0][1]).any()
+    assert not torch.isnan(outs[0][1]).any() and not torch.isnan(outs[1][-1]).any()
