@@ -43,7 +43,12 @@ def stage_balanced_bounds(seq_len: int, num_chunks: int, attn_s_per_pair: float,
 
 
 APPEND_MODES = ("serial", "fused", "overlap")
-HOST_COPY_MODES = ("kernel", "copy_engine")
+HOST_COPY_MODES = ("auto", "kernel", "copy_engine")
+# Bandwidth the one-warp-per-SM upload kernel reached beside the attention
+# launches (varlen workload on GB300), and the attention rate assumed to
+# turn a prompt's FLOP into its compute time, for host_copies="auto".
+BESIDE_UPLOAD_BYTES_PER_S = 80e9
+ATTENTION_FLOP_PER_S = 1.5e15
 
 
 def latency_balanced_bounds(seq_len: int, num_chunks: int, n_q_heads: int, n_kv_heads: int,
@@ -69,7 +74,7 @@ class ChunkedPrefill:
 
     def __init__(self, w: Workload, device, mode: Optional[int] = None, split_kv: bool = True,
                  bounds: Optional[List[List[int]]] = None, append_mode: str = "overlap",
-                 chunk_streams: Optional[int] = None, host_copies: str = "kernel"):
+                 chunk_streams: Optional[int] = None, host_copies: str = "auto"):
         """``bounds`` (one boundary list per request) replaces the workload's
         partition rule, e.g. with the Algorithm 1 stage-1 DP's split.
 
@@ -95,12 +100,16 @@ class ChunkedPrefill:
         says its rows (and all earlier rows) are in the cache.
 
         ``host_copies`` says how ``run_from_host`` / ``run_prompts_from_host``
-        move Q/K/V up from pinned host memory and O/LSE back.  "kernel": the
-        uploads by the SMs (mocap_copy_from_host: all SMs for a prompt's first
-        step, one warp per SM beside the attention launches after that); the
-        results by the copy engines while attention runs and by the SMs
-        (mocap_copy_to_host) for the last ones, which nothing hides.
-        "copy_engine": every copy by cudaMemcpyAsync."""
+        move Q/K/V up from pinned host memory and O/LSE back.  The transfers
+        nothing hides, a prompt's first upload and its last results, go by
+        all SMs (mocap_copy_from_host / mocap_copy_to_host) unless
+        "copy_engine"; results returned while attention runs go by the copy
+        engines (no SM slots taken).  Uploads while attention runs: "kernel"
+        by one warp per SM beside the attention CTAs (about 80 GB/s there);
+        "copy_engine" by cudaMemcpyAsync, as every copy then; "auto" by the
+        kernel when the prompt needs less than half that bandwidth to keep
+        its uploads ahead of its attention (compute-bound prompts), else by
+        the copy engines."""
         if append_mode not in APPEND_MODES:
             raise ValueError(f"append_mode must be one of {APPEND_MODES}")
         if host_copies not in HOST_COPY_MODES:
@@ -401,12 +410,29 @@ class ChunkedPrefill:
 
         self.run(q, k, v, compute, landed=landed, after_step=copy_back)
 
+    def _beside_uploads_by_kernel(self):
+        """host_copies "auto": the upload bandwidth this prompt needs to stay
+        ahead of its attention, against half the beside kernel's."""
+        if self.host_copies != "auto":
+            return self.host_copies == "kernel"
+        w = self.w
+        flop = sum(4 * w.n_q_heads * w.head_dim * (c * p + c * (c + 1) // 2)
+                   for b in self.bounds for p, c in
+                   ((b[i], b[i + 1] - b[i]) for i in range(len(b) - 1)))
+        up = w.total_tokens * (w.n_q_heads + 2 * w.n_kv_heads) * w.head_dim * 2
+        return up / max(flop / ATTENTION_FLOP_PER_S, 1e-9) < 0.5 * BESIDE_UPLOAD_BYTES_PER_S
+
     def _upload_step(self, step, dev_qkv, host_qkv, stream, beside):
         """Copy one step's Q/K/V rows from pinned host memory on ``stream``."""
         pairs = []
         for r, c in step:
             rows, _, _ = self._rows(r, c)
             pairs += [(d[rows], h[rows]) for d, h in zip(dev_qkv, host_qkv)]
+        if beside and self.host_copies != "copy_engine" and not self._beside_uploads_by_kernel():
+            with torch.cuda.stream(stream):
+                for d, src in pairs:
+                    d.copy_(src, non_blocking=True)
+            return
         self._host_copy(pairs, stream, beside, mocap_copy_from_host)
 
     def _copy_back(self, pairs, stream, beside):
@@ -414,7 +440,7 @@ class ChunkedPrefill:
         nothing else runs (``beside`` false: a prompt's last results, which
         nothing hides), else by the copy engines, which then work behind the
         attention launches without taking SM slots from them."""
-        if beside and self.host_copies == "kernel":
+        if beside and self.host_copies != "copy_engine":
             with torch.cuda.stream(stream):
                 for d, src in pairs:
                     d.copy_(src, non_blocking=True)

@@ -89,8 +89,8 @@ def test_refuses_what_is_not_pinned_host_memory(m):
 
 @pytest.mark.parametrize("index", [3, 5])
 def test_pipeline_host_copies_kernel_equals_copy_engine(m, index):
-    """run_from_host and run_prompts_from_host (three prompts) with both
-    forms of host copies: O and LSE bitwise equal."""
+    """run_from_host and run_prompts_from_host (three prompts) with every
+    form of host copies: O and LSE bitwise equal."""
     from paper_2606_22968_gb300 import workloads
     from paper_2606_22968_gb300.pipeline import ChunkedPrefill
     w = workloads.get(index)
@@ -98,7 +98,7 @@ def test_pipeline_host_copies_kernel_equals_copy_engine(m, index):
     q, k, v = workloads.make_qkv(w, dev)
     hq, hk, hv = (t.cpu().pin_memory() for t in (q, k, v))
     outs = []
-    for mode in ("kernel", "copy_engine"):
+    for mode in ("kernel", "copy_engine", "auto"):
         pf = ChunkedPrefill(w, dev, host_copies=mode)
         ho = torch.full(pf.out.shape, float("nan"), dtype=pf.out.dtype).pin_memory()
         hl = torch.full(pf.lse.shape, float("nan"), dtype=pf.lse.dtype).pin_memory()
@@ -123,7 +123,8 @@ def test_pipeline_host_copies_kernel_equals_copy_engine(m, index):
         assert m.mocap_last_device_status() == 0
         outs.append(tuple(t.view(torch.int16).clone() if t.dtype == torch.bfloat16 else t.clone()
                           for pr in prompts for t in pr[3:]))
-    assert all(torch.equal(a, b) for a, b in zip(outs[0], outs[2]))
-    assert all(torch.equal(a, b) for a, b in zip(outs[1], outs[3]))
+    for j in (2, 4):  # every mode gives the bits of the first
+        assert all(torch.equal(a, b) for a, b in zip(outs[0], outs[j]))
+        assert all(torch.equal(a, b) for a, b in zip(outs[1], outs[j + 1]))
     assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
     assert not torch.isnan(outs[0][1]).any() and not torch.isnan(outs[1][-1]).any()
