@@ -68,6 +68,9 @@ def parse_args():
     ap.add_argument("--case-split", choices=["none", "auto"], default="none",
                     help="with --case: 'auto' passes the library's split-KV workspace, as "
                          "the prompt pipeline does (the launch may split and add a combine)")
+    ap.add_argument("--case-host-copy", default=None,
+                    help="profiling case 'bytes,up|down,0|1': one host <-> device copy by the "
+                         "SMs (mocap_copy_from_host / _to_host), repeated (no JSON line)")
     ap.add_argument("--case-append", default=None,
                     help="profiling case 'rows,Hkv,d': one KV append launch repeated "
                          "warmup+steps times")
@@ -1166,6 +1169,31 @@ def profile_case_append(args):
     return 0
 
 
+def profile_case_host_copy(args):
+    """One host <-> device copy by the SMs, repeated (ncu probe):
+    'bytes,up|down,0|1' = size, direction, beside-attention form."""
+    import torch
+    import paper_2606_22968_gb300 as m
+    nbytes, direction, beside = args.case_host_copy.split(",")
+    nbytes, beside = int(nbytes), bool(int(beside))
+    dev = torch.device("cuda")
+    host = torch.randint(0, 256, (nbytes,), dtype=torch.uint8).pin_memory()
+    devbuf = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+    if direction == "up":
+        ms = _repeat_timed(args, lambda: m.mocap_copy_from_host([(devbuf, host)], beside))
+        ok = torch.equal(devbuf.cpu(), host)
+    else:
+        devbuf.copy_(host)
+        back = torch.zeros(nbytes, dtype=torch.uint8).pin_memory()
+        ms = _repeat_timed(args, lambda: m.mocap_copy_to_host([(back, devbuf)], beside))
+        ok = torch.equal(back, host)
+    if not ok:
+        raise RuntimeError("host copy probe: bytes differ")
+    print(json.dumps({"case_host_copy": args.case_host_copy, "ms": ms, "bytes": nbytes,
+                      "gb_per_s": nbytes / ms / 1e6}), flush=True)
+    return 0
+
+
 def _repeat_timed(args, fn, reps=20):
     """Median over `steps` samples of the mean time of `reps` back-to-back
     calls (the host enqueues ahead of the device, so per-call host work stays
@@ -1232,6 +1260,8 @@ def main():
         return profile_case(args)
     if args.case_append:
         return profile_case_append(args)
+    if args.case_host_copy:
+        return profile_case_host_copy(args)
     if args.case_qkv:
         return profile_case_qkv(args)
     if args.case_last_row:

@@ -274,7 +274,8 @@ def test_dp_partition_invalid_and_limits(lib):
 def test_bench_entry_points_exist():
     """bench.py's probe modes and arms are all defined (they are run on the GPU)."""
     import bench
-    for name in ["profile_case", "profile_case_append", "profile_case_qkv", "profile_case_last_row", "ours_arm",
+    for name in ["profile_case", "profile_case_append", "profile_case_qkv", "profile_case_last_row",
+                 "profile_case_host_copy", "measure_varlen_dev", "ours_arm",
                  "reference_arm", "measure_e2e", "measure_graph", "measure_projection",
                  "measure_last_row", "measure_partitions", "measure_chunk_streams",
                  "measure_fusion", "measure_append_graph"]:
