@@ -448,7 +448,11 @@ class ChunkedPrefill:
         self._host_copy(pairs, stream, beside, mocap_copy_to_host)
 
     def _host_copy(self, pairs, stream, beside, fn):
-        if self.host_copies == "copy_engine":
+        # the SM copies read or write the host pages through their device
+        # mapping, which only page-locked memory has: other host tensors go
+        # by cudaMemcpyAsync (torch stages pageable memory itself)
+        pinned = all(t.is_pinned() for pair in pairs for t in pair if not t.is_cuda)
+        if self.host_copies == "copy_engine" or not pinned:
             with torch.cuda.stream(stream):
                 for d, src in pairs:
                     d.copy_(src, non_blocking=True)

@@ -128,3 +128,29 @@ def test_pipeline_host_copies_kernel_equals_copy_engine(m, index):
         assert all(torch.equal(a, b) for a, b in zip(outs[1], outs[j + 1]))
     assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
     assert not torch.isnan(outs[0][1]).any() and not torch.isnan(outs[1][-1]).any()
+
+
+def test_pipeline_with_pageable_host_tensors(m):
+    """Host tensors that are not page-locked have no device mapping: the
+    pipeline moves them with the copy engines instead, same bits."""
+    from paper_2606_22968_gb300 import workloads
+    from paper_2606_22968_gb300.pipeline import ChunkedPrefill
+    w = workloads.get(2)
+    dev = torch.device("cuda")
+    q, k, v = workloads.make_qkv(w, dev)
+    res = []
+    for pin in (True, False):
+        hq, hk, hv = (t.cpu() for t in (q, k, v))
+        pf = ChunkedPrefill(w, dev)
+        ho = torch.full(pf.out.shape, float("nan"), dtype=pf.out.dtype)
+        hl = torch.full(pf.lse.shape, float("nan"), dtype=pf.lse.dtype)
+        if pin:
+            hq, hk, hv, ho, hl = (t.pin_memory() for t in (hq, hk, hv, ho, hl))
+        dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+        pf.partition()
+        pf.run_from_host(hq, hk, hv, ho, hl, dq, dk, dv)
+        torch.cuda.synchronize()
+        assert m.mocap_last_device_status() == 0
+        res.append((ho.view(torch.int16).clone(), hl.clone()))
+    assert torch.equal(res[0][0], res[1][0]) and torch.equal(res[0][1], res[1][1])
+    assert not torch.isnan(res[1][1]).any()
